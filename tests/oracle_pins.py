@@ -1,0 +1,453 @@
+"""Pins that tie the fp64 oracle to the paper and to mathematics.
+
+Each ``check_*`` function raises AssertionError when the oracle disagrees
+with something fixed independently of it: a worked example printed in the
+paper, a closed form, an invariant, a brute-force restatement on tiny
+inputs, or a special case with a known answer.  ``test_oracle_pins.py`` runs
+them against the oracle; ``test_oracle_mutations.py`` plants plausible
+mistakes in the oracle and checks that some pin fails for each.
+"""
+
+from __future__ import annotations
+
+import math
+import os
+import random
+
+import numpy as np
+
+import oracle
+from oracle import heterofold_oracle as O
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+
+
+def _read_golden(name):
+    out = {}
+    with open(os.path.join(HERE, "golden", name)) as f:
+        for line in f:
+            line = line.strip()
+            if not line or line.startswith("#"):
+                continue
+            if ":" in line:
+                k, v = line.split(":", 1)
+                out[k.strip()] = v.strip()
+            else:
+                out.setdefault("_rows", []).append(line.split())
+    return out
+
+
+def _ends(lengths):
+    return list(np.cumsum(lengths).astype(int))
+
+
+def _random_segmentation(rng, n_chars, lo, hi):
+    ends, e = [], 0
+    while e < n_chars:
+        e = min(n_chars, e + rng.randint(lo, hi))
+        ends.append(e)
+    return ends
+
+
+# ---------------------------------------------------------------------------
+# Token alignment
+# ---------------------------------------------------------------------------
+
+def check_ta_worked_example():
+    """Section 3.1's table: Qwen3 vs Ministral-3 tokenisations of
+    "The unbelievable result." give a = [1,1,1,2,3,4] and [1,4,5,6]."""
+    g = _read_golden("ta_worked_example.txt")
+    qwen = [int(x) for x in g["qwen3_ends"].split()]
+    mini = [int(x) for x in g["ministral3_ends"].split()]
+    q2m = [int(x) for x in g["qwen3_to_ministral3"].split()]
+    m2q = [int(x) for x in g["ministral3_to_qwen3"].split()]
+    assert list(O.token_alignment(qwen, mini) + 1) == q2m
+    assert list(O.token_alignment(mini, qwen) + 1) == m2q
+
+
+def check_ta_literal_shared_boundary():
+    """Reading of "latest preceding shared boundary": sender ends
+    {1,2,4,6}, receiver ends {1,3,6}; the shared boundaries are {1,6}, so
+    the receiver token ending at 3 takes the sender token ending at 1
+    (zero-based 0), not the sender-only boundary at 2."""
+    assert list(O.token_alignment([1, 2, 4, 6], [1, 3, 6])) == [0, 0, 3]
+
+
+def _ta_brute(s_end, r_end):
+    # For every receiver token scan all shared boundaries not after it.
+    shared = [e for e in r_end if e in s_end]
+    out = []
+    for e in r_end:
+        before = [x for x in shared if x <= e]
+        out.append(s_end.index(max(before)) if before else 0)
+    return out
+
+
+def check_ta_brute_force(trials=300, seed=7):
+    rng = random.Random(seed)
+    for _ in range(trials):
+        n = rng.randint(1, 60)
+        s = _random_segmentation(rng, n, 1, rng.randint(1, 7))
+        r = _random_segmentation(rng, n, 1, rng.randint(1, 7))
+        a = list(O.token_alignment(s, r))
+        assert a == _ta_brute(s, r), (s, r, a)
+        # invariants: non-decreasing, end of text maps to end of text
+        assert all(x <= y for x, y in zip(a, a[1:]))
+        assert a[-1] == len(s) - 1
+
+
+def check_ta_identity():
+    rng = random.Random(3)
+    for _ in range(50):
+        s = _random_segmentation(rng, rng.randint(1, 80), 1, 6)
+        assert list(O.token_alignment(s, s)) == list(range(len(s)))
+
+
+def check_same_index():
+    """Appendix B.1: a(j) = min(j, n_S) with one-based indices."""
+    for n_s in range(1, 7):
+        for n_r in range(0, 9):
+            a = O.same_index_alignment(n_s, n_r)
+            assert [int(x) + 1 for x in a] == [min(j, n_s) for j in range(1, n_r + 1)]
+
+
+def _overlap_brute(s_end, r_end):
+    # Token spans as explicit character sets; overlap = non-empty intersection.
+    def spans(ends):
+        out, prev = [], 0
+        for e in ends:
+            out.append(set(range(prev + 1, e + 1)))
+            prev = e
+        return out
+    S, R = spans(s_end), spans(r_end)
+    return [[k for k, sk in enumerate(S) if sk & rj] for rj in R]
+
+
+def check_overlap_brute_force(trials=300, seed=11):
+    rng = random.Random(seed)
+    for _ in range(trials):
+        n = rng.randint(1, 60)
+        s = _random_segmentation(rng, n, 1, rng.randint(1, 7))
+        r = _random_segmentation(rng, n, 1, rng.randint(1, 7))
+        rows = O.overlap_alignment(s, r)
+        assert rows == _overlap_brute(s, r), (s, r)
+        csr = O.alignment_csr(O.ALIGN_OVERLAP_MEAN, [0, len(s)], [0, len(r)], s, r)
+        for j in range(len(r)):
+            w = csr.w[csr.row_ptr[j]:csr.row_ptr[j + 1]]
+            assert abs(w.sum() - 1.0) < 1e-12  # a mean
+        # the common refinement has one piece per overlapping pair
+        assert csr.nnz == len(set(s) | set(r))
+
+
+def check_csr_batching():
+    """Concatenating requests offsets sender columns by the request start."""
+    s1, r1 = [3, 16, 23, 24], [3, 9, 12, 16, 23, 24]
+    s2, r2 = [2, 5], [1, 5]
+    csr = O.alignment_csr(O.ALIGN_TA, [0, 4, 6], [0, 6, 8], s1 + s2, r1 + r2)
+    assert list(csr.row_ptr) == list(range(9))
+    assert list(csr.col) == [0, 0, 0, 1, 2, 3, 4, 5]
+    assert np.all(csr.w == 1.0)
+
+
+# ---------------------------------------------------------------------------
+# Layer alignment
+# ---------------------------------------------------------------------------
+
+def check_layer_alignment_closed_form():
+    """Eq. 1 properties: pi(1) = 1, pi(L_R) = L_S, monotone, identity when
+    the depths agree, and the clip at the ends."""
+    for L_s in range(1, 45):
+        for L_r in range(2, 45):
+            pis = [O.proportional_depth(l, L_s, L_r) for l in range(1, L_r + 1)]
+            assert pis[0] == 1 and pis[-1] == L_s
+            assert all(a <= b for a, b in zip(pis, pis[1:]))
+            # |pi - (1 + exact)| <= 1/2
+            for l, p in zip(range(1, L_r + 1), pis):
+                exact = 1 + (l - 1) * (L_s - 1) / (L_r - 1)
+                assert abs(p - exact) <= 0.5 + 1e-12
+            if L_s == L_r:
+                assert pis == list(range(1, L_r + 1))
+            for trip in O.layer_alignment(L_s, L_r):
+                assert all(0 <= t < L_s for t in trip)
+                assert trip[0] <= trip[1] <= trip[2]
+
+
+def check_layer_alignment_hand_tables():
+    """Tables worked by hand from Eq. 1 (one-based pi)."""
+    # L_S = 4 -> L_R = 6: (l-1)*3/5 = 0, .6, 1.2, 1.8, 2.4, 3
+    assert [O.proportional_depth(l, 4, 6) for l in range(1, 7)] == [1, 2, 2, 3, 3, 4]
+    # Llama (32) -> Ministral (40): (l-1)*31/39
+    assert [O.proportional_depth(l, 32, 40) for l in range(1, 9)] == [1, 2, 3, 3, 4, 5, 6, 7]
+    # the neighbourhood of receiver layer 1 is clip(-3, 1, 5) = (1, 1, 5)
+    assert O.layer_alignment(32, 40)[0] == (0, 0, 4)
+    # last receiver layer: pi = 32 -> clip(28, 32, 36) = (28, 32, 32)
+    assert O.layer_alignment(32, 40)[-1] == (27, 31, 31)
+    # Ministral (40) -> Llama (32): (l-1)*39/31, l = 2 -> 1.258 -> 1 -> pi 2
+    assert [O.proportional_depth(l, 40, 32) for l in range(1, 5)] == [1, 2, 4, 5]
+
+
+def check_layer_interpolation():
+    for L_s in range(1, 41):
+        for L_r in range(2, 41):
+            rows = O.layer_interpolation(L_s, L_r)
+            assert len(rows) == L_r
+            assert rows[0] == [(0, 1.0)]
+            assert rows[-1] == [(L_s - 1, 1.0)]
+            for l, terms in enumerate(rows):
+                assert abs(sum(w for _, w in terms) - 1.0) < 1e-12
+                assert all(0.0 <= w <= 1.0 for _, w in terms)
+                p = sum(t * w for t, w in terms)  # the blend position
+                assert abs(p - l * (L_s - 1) / (L_r - 1)) < 1e-9
+
+
+def check_mapper_size_table_f():
+    """Appendix F's Table: 2 L_R (3 d_S d_R + d_R) parameters, in millions."""
+    g = _read_golden("mapper_size_table_f.txt")
+    for row in g["_rows"]:
+        _, _, _Ls, Lr, ds, dr, millions = row
+        n = O.mapper_parameter_count(int(Lr), int(ds), int(dr), n_seg=3)
+        assert round(n / 1e6) == int(millions), (row, n)
+        # and the same count from the segment structure of Eq. 1-2
+        segs = O.layer_segments(O.LAYER_PAPER3, int(_Ls), int(Lr))
+        assert sum(2 * (len(s) * int(ds) * int(dr) + int(dr)) for s in segs) == n
+
+
+# ---------------------------------------------------------------------------
+# RoPE and key norm
+# ---------------------------------------------------------------------------
+
+def check_rope_two_dim_rotation():
+    """D = 2, inv_freq = [1]: a plane rotation by angle p."""
+    inv = O.rope_inv_freq(10000.0, 2)
+    assert inv.tolist() == [1.0]
+    rng = np.random.default_rng(0)
+    x = rng.normal(size=(5, 1, 2))
+    pos = np.array([0, 1, 7, 1000, 131071])
+    y = O.rope(x, pos, inv)
+    for n, p in enumerate(pos):
+        c, s = math.cos(p), math.sin(p)
+        a, b = x[n, 0]
+        assert abs(y[n, 0, 0] - (a * c - b * s)) < 1e-12
+        assert abs(y[n, 0, 1] - (b * c + a * s)) < 1e-12
+
+
+def check_rope_complex_form():
+    """Rotate-half RoPE equals multiplying z_i = x_i + 1j x_{i+D/2} by
+    exp(1j p f_i); it preserves pair norms and is the identity at p = 0."""
+    rng = np.random.default_rng(1)
+    D = 16
+    inv = O.rope_inv_freq(500000.0, D)
+    x = rng.normal(size=(6, 3, D))
+    pos = np.array([0, 3, 17, 4095, 32767, 131071])
+    y = O.rope(x, pos, inv)
+    z = x[..., : D // 2] + 1j * x[..., D // 2:]
+    zr = z * np.exp(1j * pos[:, None, None] * inv[None, None, :])
+    assert np.allclose(y[..., : D // 2], zr.real, atol=1e-9)
+    assert np.allclose(y[..., D // 2:], zr.imag, atol=1e-9)
+    assert np.allclose(np.abs(zr), np.abs(z))
+    assert np.array_equal(y[0], x[0])
+
+
+def check_rope_relative_position():
+    """<RoPE_m q, RoPE_n k> depends only on m - n."""
+    rng = np.random.default_rng(2)
+    D = 8
+    inv = O.rope_inv_freq(10000.0, D)
+    q = rng.normal(size=(1, 1, D))
+    k = rng.normal(size=(1, 1, D))
+    for m, n in [(5, 3), (100, 98), (40000, 39998)]:
+        lhs = float(np.sum(O.rope(q, np.array([m]), inv) * O.rope(k, np.array([n]), inv)))
+        rhs = float(np.sum(O.rope(q, np.array([m - n]), inv) * k))
+        assert abs(lhs - rhs) < 1e-8
+
+
+def check_inv_freq():
+    inv = O.rope_inv_freq(10000.0, 128)
+    assert inv[0] == 1.0
+    assert inv[32] == float(np.float32(0.01))  # 10000 ** (-64/128)
+    assert all(a > b for a, b in zip(inv, inv[1:]))
+    assert np.all(inv.astype(np.float32).astype(np.float64) == inv)  # fp32 values
+
+
+def check_key_norm():
+    rng = np.random.default_rng(4)
+    x = rng.normal(size=(4, 2, 32)) * 3.0
+    g = np.ones(32)
+    y = O.key_norm(x, g, 0.0)
+    assert np.allclose(np.mean(y * y, axis=-1), 1.0)
+    assert np.allclose(O.key_norm(5.0 * x, g, 0.0), y)  # scale invariant
+    g2 = rng.uniform(0.5, 2.0, size=32)
+    assert np.allclose(O.key_norm(x, g2, 0.0), y * g2)
+
+
+# ---------------------------------------------------------------------------
+# The transfer
+# ---------------------------------------------------------------------------
+
+def _tiny_problem(seed, align_mode, layer_mode, L_s=3, L_r=4, H_s=2, D_s=4, H_r=2, D_r=4,
+                  n_chars=23):
+    rng = random.Random(seed)
+    nrng = np.random.default_rng(seed)
+    s_end = _random_segmentation(rng, n_chars, 1, 5)
+    r_end = _random_segmentation(rng, n_chars, 1, 4)
+    d_s, d_r = H_s * D_s, H_r * D_r
+    sender = nrng.normal(size=(L_s, 2, len(s_end), d_s))
+    segs = O.layer_segments(layer_mode, L_s, L_r)
+    K = len(segs[0]) * d_s
+    A = nrng.normal(size=(L_r, 2, K, d_r)) / math.sqrt(K)
+    b = nrng.normal(size=(L_r, 2, d_r)) * 0.1
+    r = nrng.uniform(0.5, 2.0, size=(L_r, 2))
+    csr = O.alignment_csr(align_mode, [0, len(s_end)], [0, len(r_end)], s_end, r_end)
+    inv = O.rope_inv_freq(10000.0, D_r)
+    pos = O.receiver_positions([0, len(r_end)], [5])
+    return dict(sender=sender, segs=segs, A=A, b=b, r=r, csr=csr, inv=inv, pos=pos,
+                H_r=H_r, D_r=D_r, d_s=d_s, s_end=s_end, r_end=r_end)
+
+
+def _transfer_brute(P, knorm_g=None, eps=1e-6):
+    """Every output element from the definitions, with Python loops."""
+    sender, segs, A, b, r, csr = P["sender"], P["segs"], P["A"], P["b"], P["r"], P["csr"]
+    H_r, D_r, d_s, inv, pos = P["H_r"], P["D_r"], P["d_s"], P["inv"], P["pos"]
+    out = {}
+    for l in range(len(segs)):
+        for c in (0, 1):
+            res = np.zeros((csr.n_rows, H_r, D_r))
+            for j in range(csr.n_rows):
+                y = []
+                for n in range(H_r * D_r):
+                    acc = 0.0
+                    for s, seg in enumerate(segs[l]):
+                        for (t, omega) in seg:
+                            for e in range(csr.row_ptr[j], csr.row_ptr[j + 1]):
+                                k, wk = csr.col[e], csr.w[e]
+                                for d in range(d_s):
+                                    acc += omega * wk * sender[t, c, k, d] * A[l, c, s * d_s + d, n]
+                    y.append(acc / r[l, c] + b[l, c, n])
+                for h in range(H_r):
+                    v = y[h * D_r:(h + 1) * D_r]
+                    if c == 0:
+                        if knorm_g is not None:
+                            rms = math.sqrt(sum(t * t for t in v) / D_r + eps)
+                            v = [t / rms * knorm_g[i] for i, t in enumerate(v)]
+                        half = D_r // 2
+                        w_ = list(v)
+                        for i in range(half):
+                            ang = pos[j] * inv[i]
+                            w_[i] = v[i] * math.cos(ang) - v[i + half] * math.sin(ang)
+                            w_[i + half] = v[i + half] * math.cos(ang) + v[i] * math.sin(ang)
+                        v = w_
+                    res[j, h] = v
+            out[(l, c)] = res
+    return out
+
+
+def _run_oracle(P, **kw):
+    return O.transfer(P["sender"], P["csr"], P["segs"], P["A"], P["b"], P["r"],
+                      H_r=P["H_r"], D_r=P["D_r"], pos=P["pos"], inv_freq_r=P["inv"], **kw)
+
+
+def check_transfer_brute_force():
+    for seed, am, lm in [(0, O.ALIGN_TA, O.LAYER_PAPER3),
+                         (1, O.ALIGN_OVERLAP_MEAN, O.LAYER_INTERP),
+                         (2, O.ALIGN_OVERLAP_MEAN, O.LAYER_PAPER3),
+                         (3, O.ALIGN_TA, O.LAYER_INTERP),
+                         (4, O.ALIGN_SAME_INDEX, O.LAYER_PAPER3)]:
+        P = _tiny_problem(seed, am, lm)
+        got = _run_oracle(P)
+        ref = _transfer_brute(P)
+        for key in ref:
+            assert np.allclose(got[key], ref[key], rtol=1e-10, atol=1e-10), (seed, key)
+    P = _tiny_problem(5, O.ALIGN_TA, O.LAYER_PAPER3)
+    g = np.random.default_rng(9).uniform(0.5, 1.5, size=P["D_r"])
+    got = _run_oracle(P, knorm_g=g, knorm_eps=1e-6)
+    ref = _transfer_brute(P, knorm_g=g, eps=1e-6)
+    for key in ref:
+        assert np.allclose(got[key], ref[key], rtol=1e-10, atol=1e-10)
+
+
+def check_identity_map_reproduces_input():
+    """Same depth, same tokenisation, A = [0; I; 0] (the middle block reads
+    sender layer pi(l) = l), b = 0, r = 1: V is the sender V, K is the sender K
+    rotated to its receiver position (the identity at position 0)."""
+    L, H, D = 5, 2, 8
+    d = H * D
+    rng = np.random.default_rng(5)
+    ends = _ends([2, 1, 3, 4, 1, 2, 5])
+    sender = rng.normal(size=(L, 2, len(ends), d))
+    segs = O.layer_segments(O.LAYER_PAPER3, L, L)
+    A = np.zeros((L, 2, 3 * d, d))
+    A[:, :, d:2 * d, :] = np.eye(d)
+    b = np.zeros((L, 2, d))
+    r = np.ones((L, 2))
+    csr = O.alignment_csr(O.ALIGN_TA, [0, len(ends)], [0, len(ends)], ends, ends)
+    inv = O.rope_inv_freq(10000.0, D)
+    pos = O.receiver_positions([0, len(ends)])
+    out = O.transfer(sender, csr, segs, A, b, r, H_r=H, D_r=D, pos=pos, inv_freq_r=inv)
+    for l in range(L):
+        assert np.array_equal(out[(l, 1)].reshape(len(ends), d), sender[l, 1])
+        assert np.array_equal(out[(l, 0)][0].reshape(d), sender[l, 0, 0])
+        z = sender[l, 0].reshape(len(ends), H, D)
+        zc = z[..., : D // 2] + 1j * z[..., D // 2:]
+        zc = zc * np.exp(1j * pos[:, None, None] * inv[None, None, :])
+        assert np.allclose(out[(l, 0)][..., : D // 2], zc.real)
+        assert np.allclose(out[(l, 0)][..., D // 2:], zc.imag)
+
+
+def check_affine_structure():
+    """Eq. 9 is affine in the sender features with slope 1/r: zero input gives
+    the bias; scaling the sender scales (y - b); doubling r halves it."""
+    P = _tiny_problem(6, O.ALIGN_OVERLAP_MEAN, O.LAYER_PAPER3)
+    base = _run_oracle(P, roles=(1,))
+    P0 = dict(P, sender=np.zeros_like(P["sender"]))
+    zero = _run_oracle(P0, roles=(1,))
+    for (l, c), y in zero.items():
+        assert np.allclose(y.reshape(y.shape[0], -1), P["b"][l, c][None, :])
+    P2 = dict(P, sender=2.5 * P["sender"])
+    scaled = _run_oracle(P2, roles=(1,))
+    Pr = dict(P, r=2.0 * P["r"])
+    halved = _run_oracle(Pr, roles=(1,))
+    for (l, c), y in base.items():
+        bb = P["b"][l, c].reshape(1, P["H_r"], P["D_r"])
+        assert np.allclose(scaled[(l, c)] - bb, 2.5 * (y - bb))
+        assert np.allclose(halved[(l, c)] - bb, 0.5 * (y - bb))
+
+
+def check_segment_blocks():
+    """Segment s multiplies rows [s d_S, (s+1) d_S) of A: zeroing all but one
+    block equals mapping that sender layer alone with that block."""
+    P = _tiny_problem(8, O.ALIGN_TA, O.LAYER_PAPER3)
+    d_s = P["d_s"]
+    for s in range(3):
+        A1 = np.zeros_like(P["A"])
+        A1[:, :, s * d_s:(s + 1) * d_s, :] = P["A"][:, :, s * d_s:(s + 1) * d_s, :]
+        got = _run_oracle(dict(P, A=A1), roles=(1,))
+        for (l, c), y in got.items():
+            t = P["segs"][l][s][0][0]
+            a = P["csr"].col[P["csr"].row_ptr[:-1]]
+            x = P["sender"][t, c][a]
+            ref = x @ P["A"][l, c, s * d_s:(s + 1) * d_s, :] / P["r"][l, c] + P["b"][l, c]
+            assert np.allclose(y.reshape(len(a), -1), ref)
+
+
+ALL_CHECKS = [
+    check_ta_worked_example, check_ta_literal_shared_boundary, check_ta_brute_force,
+    check_ta_identity, check_same_index, check_overlap_brute_force, check_csr_batching,
+    check_layer_alignment_closed_form, check_layer_alignment_hand_tables,
+    check_layer_interpolation, check_mapper_size_table_f,
+    check_rope_two_dim_rotation, check_rope_complex_form, check_rope_relative_position,
+    check_inv_freq, check_key_norm,
+    check_transfer_brute_force, check_identity_map_reproduces_input,
+    check_affine_structure, check_segment_blocks,
+]
+
+
+def run_all():
+    failures = []
+    for chk in ALL_CHECKS:
+        try:
+            chk()
+        except AssertionError as e:  # pragma: no cover - reported by the caller
+            failures.append((chk.__name__, repr(e)[:200]))
+        except Exception as e:  # a mutated oracle may also raise
+            failures.append((chk.__name__, repr(e)[:200]))
+    return failures

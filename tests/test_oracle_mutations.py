@@ -1,0 +1,137 @@
+"""Plant plausible mistakes in the oracle (on the CPU) and check that the
+pins catch every one of them: evidence that the pins constrain each part of
+the oracle, not just its happy path."""
+import math
+
+import numpy as np
+import pytest
+
+import oracle_pins as pins
+from oracle import heterofold_oracle as O
+
+
+def _ta_any_sender_boundary(s_end, r_end):
+    # wrong reading: latest *sender* boundary, shared or not
+    s, r = list(s_end), list(r_end)
+    out = []
+    for e in r:
+        before = [i for i, x in enumerate(s) if x <= e]
+        out.append(before[-1] if before else 0)
+    return np.asarray(out)
+
+
+def _ta_next_boundary(s_end, r_end):
+    # wrong: the sender token that contains the receiver token's end
+    s = list(s_end)
+    return np.asarray([next(i for i, x in enumerate(s) if x >= e) for e in r_end])
+
+
+def _depth_floor(l1, L_s, L_r):
+    if L_r == 1:
+        return 1
+    return 1 + ((l1 - 1) * (L_s - 1)) // (L_r - 1)
+
+
+def _layer_alignment_offsets3(L_s, L_r):
+    return [tuple(min(max(O.proportional_depth(l, L_s, L_r) + o, 1), L_s) - 1
+                  for o in (-3, 0, 3)) for l in range(1, L_r + 1)]
+
+
+def _rope_sign(x, pos, inv):
+    D = x.shape[-1]
+    h = D // 2
+    ang = np.asarray(pos, dtype=np.float64)[:, None] * inv[None, :]
+    c, s = np.cos(ang)[:, None, :], np.sin(ang)[:, None, :]
+    return np.concatenate([x[..., :h] * c + x[..., h:] * s, x[..., h:] * c - x[..., :h] * s], -1)
+
+
+def _rope_interleaved(x, pos, inv):
+    ang = np.asarray(pos, dtype=np.float64)[:, None] * inv[None, :]
+    c, s = np.cos(ang)[:, None, :], np.sin(ang)[:, None, :]
+    y = x.copy()
+    y[..., 0::2] = x[..., 0::2] * c - x[..., 1::2] * s
+    y[..., 1::2] = x[..., 1::2] * c + x[..., 0::2] * s
+    return y
+
+
+def _inv_freq_wrong(theta, D):
+    return np.array([np.float32(float(theta) ** (-(1.0 * i) / D)) for i in range(D // 2)],
+                    dtype=np.float64)
+
+
+def _key_norm_no_weight(x, g, eps):
+    return x / np.sqrt(np.mean(x * x, axis=-1, keepdims=True) + eps)
+
+
+def _interp_swapped(L_s, L_r):
+    out = []
+    for l in range(L_r):
+        p = (l * (L_s - 1)) / (L_r - 1) if L_r > 1 else 0.0
+        i0 = int(math.floor(p))
+        f = p - i0
+        terms = [(i0, f)] if f > 0 else [(i0, 1.0)]
+        if f > 0:
+            terms.append((min(i0 + 1, L_s - 1), 1.0 - f))
+        out.append(terms)
+    return out
+
+
+def _overlap_closed(s_end, r_end):
+    # wrong: spans that merely touch count as overlapping
+    s, r = list(s_end), list(r_end)
+    rows = []
+    for j, e in enumerate(r):
+        st = r[j - 1] if j else 0
+        rows.append([k for k in range(len(s)) if (s[k - 1] if k else 0) <= e and s[k] >= st])
+    return rows
+
+
+def _pool_unweighted(sender_lc, csr, rows):
+    out = []
+    for j in rows:
+        idx = csr.col[csr.row_ptr[j]:csr.row_ptr[j + 1]]
+        out.append(np.asarray(sender_lc[idx], dtype=np.float64).sum(axis=0))
+    return np.asarray(out)
+
+
+_orig_map_input = O.map_input
+_orig_transfer = O.transfer
+
+
+def _map_input_reversed(sender, csr, segments_l, role, rows):
+    return _orig_map_input(sender, csr, list(reversed(segments_l)), role, rows)
+
+
+def _transfer_no_bias(sender, csr, segments, A, b, r, **kw):
+    return _orig_transfer(sender, csr, segments, A, np.zeros_like(np.asarray(b, dtype=np.float64)), r, **kw)
+
+
+def _transfer_times_r(sender, csr, segments, A, b, r, **kw):
+    r2 = 1.0 / np.asarray(r, dtype=np.float64)
+    return _orig_transfer(sender, csr, segments, A, b, r2, **kw)
+
+
+MUTATIONS = {
+    "ta_any_sender_boundary": ("token_alignment", _ta_any_sender_boundary),
+    "ta_next_boundary": ("token_alignment", _ta_next_boundary),
+    "depth_floor": ("proportional_depth", _depth_floor),
+    "offsets_3": ("layer_alignment", _layer_alignment_offsets3),
+    "rope_sign": ("rope", _rope_sign),
+    "rope_interleaved": ("rope", _rope_interleaved),
+    "inv_freq_exponent": ("rope_inv_freq", _inv_freq_wrong),
+    "key_norm_weight_dropped": ("key_norm", _key_norm_no_weight),
+    "interp_weights_swapped": ("layer_interpolation", _interp_swapped),
+    "overlap_touching": ("overlap_alignment", _overlap_closed),
+    "pool_unweighted": ("pooled_features", _pool_unweighted),
+    "segments_reversed": ("map_input", _map_input_reversed),
+    "bias_dropped": ("transfer", _transfer_no_bias),
+    "r_multiplies": ("transfer", _transfer_times_r),
+}
+
+
+@pytest.mark.parametrize("name", sorted(MUTATIONS))
+def test_pins_catch_planted_mistake(name, monkeypatch):
+    attr, fn = MUTATIONS[name]
+    monkeypatch.setattr(O, attr, fn)
+    failures = pins.run_all()
+    assert failures, f"no pin caught the planted mistake {name!r}"
