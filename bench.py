@@ -1,0 +1,405 @@
+"""Benchmark of the HeteroFold transfer hot path on GB300.
+
+A step is one pass of the whole path over one batch: alignment CSR
+(hf_align_build), plan metadata (hf_plan_create), the fused map
+(hf_transfer).  Default workload: the 32K-receiver-token Llama-3.1-8B-shaped
+-> Ministral-shaped transfer (Token Alignment + three-layer neighbourhood,
+bf16 caches and maps, fp32 accumulation).
+
+Prints one JSON line (rank 0).  --impl reference times the fp64 CPU oracle
+on a bounded sample of the same workload instead.
+"""
+
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "transferred receiver-KV tokens/sec and µs per 32K transfer; % of roofline"
+UNIT = "receiver tokens/s"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="llama_to_ministral_32k")
+    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    return ap.parse_args()
+
+
+def workload(name):
+    from paper_2609_32259_gb300 import workloads as W
+    table = {
+        "llama_to_ministral_32k": lambda: W.llama_to_ministral(32768),
+        "llama_to_qwen25_4k": lambda: W.llama_to_qwen25(4096),
+        "qwen25_to_llama_batched_paged": W.qwen25_to_llama_batched,
+        "tiny": W.tiny,
+    }
+    if name.startswith("ministral_to_llama_"):
+        return W.ministral_to_llama(int(name.rsplit("_", 1)[1]))
+    return table[name]()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), float(p["bf16_tflops"]), "measured"
+    return 6800.0, 1900.0, "fallback"
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.proc = None
+        self.gpu = gpu_index
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.QUERY}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (FileNotFoundError, OSError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# algorithmic work of one transfer
+# ---------------------------------------------------------------------------
+def algorithmic_work(w, tok, U, n_distinct_cols):
+    """FLOPs and bytes a transfer cannot avoid.
+
+    FLOP: 2 * (2 L_r) * U * K * d_r, U = distinct alignment rows (rows with
+    identical inputs share one map output before RoPE).
+    Bytes: the receiver cache written once; every referenced sender row read
+    once per sender layer (the three-layer neighbourhoods of these depth
+    pairs touch every sender layer); the maps and biases read once; the CSR
+    and per-row metadata."""
+    e = 2 if w.dtype == "bf16" else 4
+    flops = 2.0 * 2 * w.L_r * U * w.K * w.d_r
+    T_r = tok.T_r
+    bytes_ = (2 * w.L_r * T_r * w.d_r * e            # receiver cache
+              + w.L_s * 2 * n_distinct_cols * w.d_s * e  # sender rows
+              + 2 * w.L_r * w.K * w.d_r * e          # maps
+              + 2 * w.L_r * w.d_r * 4                # bias
+              + T_r * 4 * 6)                         # CSR + run / position / row metadata
+    return flops, float(bytes_)
+
+
+# ---------------------------------------------------------------------------
+# the oracle on host cores (cpu_baseline and --impl reference)
+# ---------------------------------------------------------------------------
+class OracleSample:
+    """A contiguous block of receiver rows of the workload, all layers and
+    roles, with everything the oracle needs already in host memory."""
+
+    def __init__(self, w, tok, sender, Wm, b, r, n_rows, start=None):
+        import numpy as np
+        from oracle import heterofold_oracle as O
+        self.O = O
+        csr = O.alignment_csr(w.align_mode, tok.s_tok_ptr, tok.r_tok_ptr, tok.s_end, tok.r_end)
+        T = tok.T_r
+        n_rows = max(1, min(n_rows, T))
+        j0 = (T - n_rows) // 2 if start is None else start
+        rows = np.arange(j0, j0 + n_rows)
+        e0, e1 = int(csr.row_ptr[j0]), int(csr.row_ptr[j0 + n_rows])
+        cols = csr.col[e0:e1]
+        c_lo, c_hi = int(cols.min()), int(cols.max()) + 1
+        self.csr = O.CSR(csr.row_ptr[j0:j0 + n_rows + 1] - e0, cols - c_lo, csr.w[e0:e1])
+        self.sender = sender[:, :, c_lo:c_hi].float().cpu().numpy()
+        self.A = Wm.float().cpu().numpy().transpose(0, 1, 3, 2)
+        self.b = b.cpu().numpy()
+        self.r = r
+        self.segs = O.layer_segments(w.layer_mode, w.L_s, w.L_r)
+        self.pos = O.receiver_positions(tok.r_tok_ptr)[j0:j0 + n_rows]
+        self.inv = O.rope_inv_freq(w.theta_r, w.D_r)
+        self.w = w
+        self.n_rows = n_rows
+
+    def run(self):
+        return self.O.transfer(self.sender, self.csr, self.segs, self.A, self.b, self.r,
+                               H_r=self.w.H_r, D_r=self.w.D_r, pos=self.pos,
+                               inv_freq_r=self.inv)
+
+
+def blas_threads():
+    for k in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
+        v = os.environ.get(k)
+        if v and v.isdigit():
+            return int(v)
+    return os.cpu_count() or 1
+
+
+def sized_oracle_sample(w, tok, sender, Wm, b, r, seconds):
+    """Calibrates the sample size so one oracle pass takes ~`seconds`."""
+    probe = OracleSample(w, tok, sender, Wm, b, r, 32)
+    t0 = time.perf_counter()
+    probe.run()
+    dt = max(time.perf_counter() - t0, 1e-3)
+    n = int(32 * seconds / dt)
+    n = max(32, min(n, tok.T_r))
+    return OracleSample(w, tok, sender, Wm, b, r, n)
+
+
+# ---------------------------------------------------------------------------
+def run_reference(args):
+    """--impl reference: the fp64 oracle on the host cores, one bounded
+    sample of the workload per step."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    import torch
+    from paper_2609_32259_gb300 import workloads as W
+    w = workload(args.workload)
+    tok = W.tokens(w)
+    dev = torch.device("cuda") if torch.cuda.is_available() else torch.device("cpu")
+    sender = W.sender_kv(w, tok.T_s, dev)
+    Wm, b, r = W.maps(w, dev)
+    per_step = max(1.0, min(8.0, 150.0 / max(1, args.steps + args.warmup)))
+    samp = sized_oracle_sample(w, tok, sender, Wm, b, r, per_step)
+    for _ in range(args.warmup):
+        samp.run()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        samp.run()
+    dt = (time.perf_counter() - t0) / max(1, args.steps)
+    value = samp.n_rows / dt
+    sample = (f"{samp.n_rows} contiguous receiver rows x {w.L_r} layers x K/V of "
+              f"{w.name} per step (dense fp64 numpy, oracle as written)")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": dt * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": w.name, "T_r": tok.T_r, "T_s": tok.T_s,
+                   "mode": f"{w.align_mode}+{w.layer_mode}"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": blas_threads(),
+                         "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_ours(args):
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    if not torch.cuda.is_available():
+        print(json.dumps({"error": "no CUDA device"}))
+        return 1
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+
+    import __graft_entry__ as g
+    if rank == 0:
+        g.build()
+    if world > 1:
+        dist.barrier()
+    from paper_2609_32259_gb300 import pipeline, workloads as W
+
+    w = workload(args.workload)
+    tok = W.tokens(w)
+    sender = W.sender_kv(w, tok.T_s, dev)
+    Wm, b, r = W.maps(w, dev)
+    paged = W.paged_layout(w, tok) if w.paged else None
+    job = pipeline.job_from_workload(w, tok, sender, Wm, b, r, paged=paged, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    for _ in range(max(3, args.warmup)):
+        job.step(stream)
+    torch.cuda.synchronize()
+    status = job.device_status()
+    U = job.distinct_rows()
+    _, col, _ = job.csr()
+    n_cols = int(np.unique(col).size)
+
+    # timed region: K whole steps, plus the transfer kernel alone per step
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for i in range(args.steps):
+        job.align(stream)
+        job.make_plan(stream)
+        ev[i][0].record(stream)
+        job.transfer(stream)
+        ev[i][1].record(stream)
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clk = clocks.stop()
+    step_ms = t_start.elapsed_time(t_end) / args.steps
+    kern_ms = statistics.mean(a.elapsed_time(bb) for a, bb in ev)
+    if world > 1:
+        t = torch.tensor([step_ms, kern_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        step_ms, kern_ms = float(t[0]), float(t[1])
+    value = world * tok.T_r / (step_ms * 1e-3)
+
+    # end to end through the API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        h_sender = torch.empty(sender.shape, dtype=sender.dtype, pin_memory=True)
+        h_sender.copy_(sender)
+        h_recv = torch.empty(job.receiver.shape, dtype=job.receiver.dtype, pin_memory=True)
+        h_s_end = torch.as_tensor(tok.s_end).pin_memory()
+        h_r_end = torch.as_tensor(tok.r_end).pin_memory()
+        n_e2e = max(1, args.e2e_steps)
+        torch.cuda.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        for it in range(n_e2e + 1):  # first pass warms up
+            if it == 1:
+                e0.record(stream)
+            sender.copy_(h_sender, non_blocking=True)
+            job.s_end.copy_(h_s_end, non_blocking=True)
+            job.r_end.copy_(h_r_end, non_blocking=True)
+            job.step(stream)
+            h_recv.copy_(job.receiver, non_blocking=True)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        e2e_ms = e0.elapsed_time(e1) / n_e2e
+        if world > 1:
+            t = torch.tensor([e2e_ms], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e2e_ms = float(t[0])
+        h2d = (sender.numel() * sender.element_size() + h_s_end.numel() * 4 +
+               h_r_end.numel() * 4)
+        d2h = job.receiver.numel() * job.receiver.element_size()
+        e2e = {"value": world * tok.T_r / (e2e_ms * 1e-3), "unit": UNIT, "ms_per_step": e2e_ms,
+               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
+        del h_sender, h_recv
+
+    hbm_gbs, tflops, src = peaks()
+    flops, bytes_ = algorithmic_work(w, tok, U, n_cols)
+    t_k = kern_ms * 1e-3
+    t_tensor = flops / (tflops * 1e12)
+    t_hbm = bytes_ / (hbm_gbs * 1e9)
+    if t_tensor >= t_hbm:
+        roof = {"bound": "tensor", "achieved": flops / t_k / 1e12, "peak": tflops,
+                "unit": "TFLOP/s", "frac": (flops / t_k / 1e12) / tflops}
+    else:
+        roof = {"bound": "hbm", "achieved": bytes_ / t_k / 1e9, "peak": hbm_gbs,
+                "unit": "GB/s", "frac": (bytes_ / t_k / 1e9) / hbm_gbs}
+    roof.update({"traffic": None, "peak_source": src, "kernel": "transfer_kernel",
+                 "kernel_ms": kern_ms, "flop_alg": flops, "bytes_alg": bytes_,
+                 "hbm_achieved_gbs": bytes_ / t_k / 1e9,
+                 "tensor_achieved_tflops": flops / t_k / 1e12,
+                 "roofline_ms": max(t_tensor, t_hbm) * 1e3})
+    traffic_file = os.path.join(ROOT, "profiles", "transfer_traffic.json")
+    if os.path.exists(traffic_file):
+        with open(traffic_file) as f:
+            tr = json.load(f).get(w.name)
+        if tr:
+            roof["traffic"] = tr
+
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        samp = sized_oracle_sample(w, tok, sender, Wm, b, r, args.cpu_seconds)
+        t0 = time.perf_counter()
+        samp.run()
+        dt = time.perf_counter() - t0
+        cpu = {"value": samp.n_rows / dt, "unit": UNIT, "cores": blas_threads(),
+               "kind": "oracle", "seconds": dt,
+               "sample": (f"{samp.n_rows} contiguous receiver rows x {w.L_r} layers x K/V "
+                          f"of {w.name} (dense fp64 numpy oracle as written)")}
+
+    launches_per_step = 3 + 4 + 1  # align (3 kernels), plan (4), transfer (1)
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_ms,
+        "us_per_transfer": step_ms * 1e3, "us_per_transfer_kernel": kern_ms * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": w.dtype, "data": "synthetic",
+        "config": {"workload": w.name, "T_r": tok.T_r, "T_s": tok.T_s,
+                   "distinct_rows": U, "sender": f"{w.L_s}x{w.H_s}x{w.D_s}",
+                   "receiver": f"{w.L_r}x{w.H_r}x{w.D_r}",
+                   "mode": f"{w.align_mode}+{w.layer_mode}",
+                   "l2": "inputs larger than L2 (no flush)",
+                   "parallelism": "replicas" if world > 1 else "single"},
+        "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
+        "gpu_launches": launches_per_step * args.steps, "device_status": status,
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    job.close()
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,229 @@
+/*
+ * heterofold.h — C ABI of the GB300 (sm_103a) HeteroFold transfer library.
+ *
+ * HeteroFold (arxiv 2609.32259) turns a sender model's KV cache into a
+ * receiver model's KV cache without receiver prefill.  At inference time it
+ * applies, per receiver layer l and role c in {K, V}, one folded affine map
+ * (Section 3.3 "Folding for inference", Eq. 9):
+ *
+ *     Phi_{l,c}(x_j) = (x_j / r_{l,c}) A_final_{l,c} + b_final_{l,c}
+ *
+ * to the concatenated features of three sender layers (Eq. 1-2) taken at
+ * the sender token that Token Alignment pairs with receiver token j
+ * (Section 3.1, Appendix B.1); the output is reshaped into the receiver's
+ * KV heads, and keys get the receiver's key normalisation and RoPE at
+ * receiver positions (Section 3 opening paragraph, Appendix B.1).
+ *
+ * Call sequence for one transfer:
+ *   hf_align_build            character-end offsets -> alignment CSR (device)
+ *   hf_plan_workspace_size    bytes of device workspace the plan needs
+ *   hf_plan_create            validates, builds per-transfer metadata (device)
+ *   hf_transfer               one kernel launch: receiver cache <- Phi(sender)
+ *   hf_plan_destroy
+ *
+ * General rules:
+ *  - Every pointer prefixed d_ is device memory; h_ or unprefixed arrays
+ *    documented as "host" are host memory.  The library allocates no device
+ *    memory: all device buffers belong to the caller, who keeps them alive
+ *    and unchanged while work that uses them is in flight.
+ *  - Every device-side function is asynchronous and stream-ordered on the
+ *    given stream (NULL = the legacy default stream); none synchronises the
+ *    host except hf_plan_device_status and hf_plan_distinct_rows.
+ *  - Functions return an hf_status; HF_OK is 0.  On any other value
+ *    hf_last_error() returns a message for the calling host thread.  Invalid
+ *    arguments are caught on the host before any launch.
+ *  - Data-dependent problems that only the device can see (unsorted
+ *    offsets, out-of-range columns or blocks, a wait that timed out) set
+ *    bits in a device status word; kernels skip the offending row or block
+ *    and never trap.  hf_plan_device_status reads the word.
+ *  - A plan may be used by one stream at a time.
+ *  - Requires a GPU of compute capability 10.3 (GB300).
+ */
+#ifndef HETEROFOLD_H
+#define HETEROFOLD_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t. */
+typedef struct CUstream_st* hf_stream_t;
+
+typedef enum {
+  HF_OK = 0,
+  HF_ERR_INVALID_ARGUMENT = 1, /* a host-visible argument is wrong; nothing launched */
+  HF_ERR_UNSUPPORTED = 2,      /* valid but outside what the kernels handle */
+  HF_ERR_CUDA = 3,             /* a CUDA runtime or driver call failed */
+  HF_ERR_DEVICE_CHECK = 5,     /* the device status word has bits set */
+  HF_ERR_WORKSPACE = 6         /* workspace too small or misaligned */
+} hf_status;
+
+/* Token alignment rules (rows of the alignment CSR). */
+typedef enum {
+  /* Token Alignment, Section 3.1 and Appendix B.1: one sender token per
+     receiver token, weight 1: the sender token ending at the latest shared
+     character-end boundary at or before the receiver token's end; the first
+     sender token before the first shared boundary. */
+  HF_ALIGN_TA = 0,
+  /* Mean pooling over every sender token whose character span
+     (end_{k-1}, end_k] overlaps the receiver token's span; weights are the
+     fp32 rounding of 1/n. */
+  HF_ALIGN_OVERLAP_MEAN = 1,
+  /* Same-index pairing, Appendix A and B.1: a(j) = min(j, n_S), one-based. */
+  HF_ALIGN_SAME_INDEX = 2
+} hf_align_mode;
+
+/* Layer alignment rules (map input segments per receiver layer). */
+typedef enum {
+  /* Eq. 1-2: three sender layers N(l) = clip(pi(l)-4, pi(l), pi(l)+4),
+     pi(l) = 1 + round((l-1)(L_S-1)/(L_R-1)), concatenated: K = 3 d_S. */
+  HF_LAYER_PAPER3 = 0,
+  /* One segment: the linear interpolation of sender layers floor(p) and
+     floor(p)+1 at p = l (L_S-1)/(L_R-1) (zero-based l): K = d_S. */
+  HF_LAYER_INTERP = 1
+} hf_layer_mode;
+
+typedef enum {
+  HF_BF16 = 0, /* bf16 K/V and maps; fp32 accumulation (tcgen05 kind::f16) */
+  HF_F32 = 1   /* fp32 K/V and maps; tf32 products, fp32 accumulation */
+} hf_dtype;
+
+/* Bits of the device status word. */
+#define HF_CHECK_BAD_OFFSETS   0x01 /* offsets not strictly increasing, or ends differ */
+#define HF_CHECK_BAD_COLUMN    0x02 /* a CSR column outside the sender tokens */
+#define HF_CHECK_BAD_ROW       0x04 /* an empty CSR row, or a row that is not one
+                                       weight-1 entry where the align mode says so */
+#define HF_CHECK_BAD_BLOCK     0x08 /* a block-table entry outside the pool */
+#define HF_CHECK_CAPACITY      0x10 /* the CSR did not fit the given capacity */
+#define HF_CHECK_TIMEOUT       0x20 /* a pipeline wait gave up (internal error) */
+
+/*
+ * hf_align_build — alignment CSR from character-end offsets (Section 3.1,
+ * Appendix B.1; mode as above).
+ *
+ * n_req      number of requests (1 .. 4096) concatenated in one call.
+ * s_tok_ptr  host int32[n_req+1], non-decreasing, s_tok_ptr[0] = 0: request q
+ *            owns sender tokens [s_tok_ptr[q], s_tok_ptr[q+1]).
+ * r_tok_ptr  host int32[n_req+1], the same for receiver tokens.
+ * d_s_end    device int32[T_s]: character-end offset of every sender token,
+ *            restarting per request; strictly increasing and positive within
+ *            a request (tokens are nonempty).
+ * d_r_end    device int32[T_r]: the same for receiver tokens.  Within a
+ *            request the last sender and receiver ends must be equal (both
+ *            sides tokenise the same text); a request with receiver tokens
+ *            needs at least one sender token.
+ * d_row_ptr  device int32[T_r+1] out: CSR row pointers, global.
+ * d_col      device int32[nnz_capacity] out: global sender token indices.
+ * d_w        device float[nnz_capacity] out: pooling weights.
+ * nnz_capacity  entries available in d_col/d_w; must be >= T_r for TA and
+ *            same-index, >= T_r + T_s for overlap mean pooling.
+ * d_info     device int32[2] out: [0] = nnz, [1] = status bits
+ *            (HF_CHECK_BAD_OFFSETS, HF_CHECK_CAPACITY).
+ * Rows are ordered like the receiver tokens; each row's columns ascend.
+ */
+hf_status hf_align_build(hf_align_mode mode, int32_t n_req, const int32_t* s_tok_ptr,
+                         const int32_t* r_tok_ptr, const int32_t* d_s_end,
+                         const int32_t* d_r_end, int32_t* d_row_ptr, int32_t* d_col,
+                         float* d_w, int64_t nnz_capacity, int32_t* d_info,
+                         hf_stream_t stream);
+
+/* Everything a transfer needs besides the two caches. */
+typedef struct {
+  /* Shapes: layers, KV heads and head width of sender (s) and receiver (r).
+     d_S = H_s * D_s and d_R = H_r * D_r are the flattened feature widths
+     (head-major, index h * D + d). */
+  int32_t L_s, H_s, D_s;
+  int32_t L_r, H_r, D_r;
+  hf_dtype dtype;          /* element type of both caches and of d_W */
+  hf_layer_mode layer_mode;
+  hf_align_mode align_mode; /* the rule the CSR was built with */
+
+  /* Requests (host): as in hf_align_build. */
+  int32_t n_req;
+  const int32_t* s_tok_ptr;     /* host int32[n_req+1] */
+  const int32_t* r_tok_ptr;     /* host int32[n_req+1] */
+  const int32_t* r_pos0;        /* host int32[n_req] receiver position of each
+                                   request's first token, or NULL for 0 */
+
+  /* Alignment CSR (device, from hf_align_build or the caller). */
+  const int32_t* d_row_ptr;     /* int32[T_r+1] */
+  const int32_t* d_col;         /* int32[nnz] */
+  const float* d_w;             /* float[nnz] */
+
+  /* Folded maps (Eq. 9), device.  d_W is A_final transposed:
+     [L_r][2][d_R][K] row-major in `dtype`, K = 3 d_S (PAPER3) or d_S
+     (INTERP); row n of W[l][c] holds column n of A_final, and segment s of
+     the map input occupies W columns [s d_S, (s+1) d_S). */
+  const void* d_W;
+  const float* d_b;             /* float[L_r][2][d_R], b_final */
+  const float* h_r;             /* host float[L_r][2], Eq. 3's r (> 0) */
+
+  /* Receiver key processing. */
+  double theta_r;               /* RoPE base; <= 0 disables RoPE */
+  const float* d_knorm_w;       /* device float[D_r] key RMS-norm weight, or NULL */
+  float knorm_eps;
+
+  /* Receiver cache layout.  paged = 0: receiver_kv is
+     [L_r][2][T_r][H_r][D_r].  paged = 1: receiver_kv is a block pool
+     [L_r][2][n_blocks][block_size][H_r][D_r] and token t of request q goes
+     to block d_block_table[q * max_blocks_per_req + t / block_size], slot
+     t % block_size. */
+  int32_t paged;
+  int32_t block_size;
+  int32_t n_blocks;
+  int32_t max_blocks_per_req;
+  const int32_t* d_block_table; /* device int32[n_req][max_blocks_per_req] */
+} hf_plan_desc;
+
+typedef struct hf_plan_s* hf_plan;
+
+/* Bytes of device workspace hf_plan_create needs for this descriptor. */
+hf_status hf_plan_workspace_size(const hf_plan_desc* desc, size_t* bytes);
+
+/*
+ * hf_plan_create — validate the descriptor and build the per-transfer
+ * metadata on `stream`: the layer table (Eq. 1 or interpolation), RoPE
+ * inverse frequencies fp32(theta_r^(-2i/D_r)), the receiver position and
+ * destination row of every receiver token, and the runs of identical CSR
+ * rows (their map output is identical before RoPE).
+ * d_workspace: device memory of hf_plan_workspace_size bytes, 256-byte
+ * aligned, owned by the caller and reserved for this plan until
+ * hf_plan_destroy.  The plan keeps pointers to d_row_ptr, d_col, d_w,
+ * d_W, d_b, d_knorm_w and d_block_table; host arrays are copied.
+ */
+hf_status hf_plan_create(const hf_plan_desc* desc, void* d_workspace, size_t workspace_bytes,
+                         hf_stream_t stream, hf_plan* out);
+
+/*
+ * hf_transfer — write the receiver cache (one kernel launch on `stream`).
+ * sender_kv:   device [L_s][2][T_s][H_s][D_s] in the plan's dtype, the
+ *              sender's pre-RoPE keys and values (Section 3: keys are mapped
+ *              before key normalisation and RoPE); 16-byte aligned.
+ * receiver_kv: device, layout per desc.paged; 16-byte aligned.  Only the
+ *              rows (contiguous) or block slots (paged) of the plan's
+ *              receiver tokens are written.
+ */
+hf_status hf_transfer(hf_plan plan, const void* sender_kv, void* receiver_kv,
+                      hf_stream_t stream);
+
+/* Frees the plan's host memory.  Does not touch the workspace. */
+hf_status hf_plan_destroy(hf_plan plan);
+
+/* Synchronises `stream` and returns the plan's device status bits in
+   *flags (0 = clean); HF_ERR_DEVICE_CHECK if any bit is set. */
+hf_status hf_plan_device_status(hf_plan plan, hf_stream_t stream, int32_t* flags);
+
+/* Synchronises `stream` and returns the number of distinct alignment rows. */
+hf_status hf_plan_distinct_rows(hf_plan plan, hf_stream_t stream, int32_t* n_rows);
+
+const char* hf_status_string(hf_status status);
+const char* hf_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* HETEROFOLD_H */

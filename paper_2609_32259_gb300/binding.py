@@ -1,0 +1,226 @@
+"""ctypes binding of the C ABI in include/heterofold.h.
+
+Argument marshalling only: every step of the transfer runs in the CUDA
+library.  Device pointers may be given as torch tensors (their data_ptr()) or
+plain integers; host arrays as numpy arrays.  If libheterofold.so has not
+been built, every call raises RuntimeError: there is no fallback path.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional
+
+import numpy as np
+
+PKG_DIR = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(PKG_DIR, "libheterofold.so")
+
+# enums of heterofold.h
+HF_OK = 0
+HF_ERR_INVALID_ARGUMENT = 1
+HF_ERR_UNSUPPORTED = 2
+HF_ERR_CUDA = 3
+HF_ERR_DEVICE_CHECK = 5
+HF_ERR_WORKSPACE = 6
+
+ALIGN_MODES = {"ta": 0, "overlap_mean": 1, "same_index": 2}
+LAYER_MODES = {"paper3": 0, "interp": 1}
+DTYPES = {"bf16": 0, "f32": 1}
+
+CHECK_BITS = {
+    0x01: "HF_CHECK_BAD_OFFSETS", 0x02: "HF_CHECK_BAD_COLUMN", 0x04: "HF_CHECK_BAD_ROW",
+    0x08: "HF_CHECK_BAD_BLOCK", 0x10: "HF_CHECK_CAPACITY", 0x20: "HF_CHECK_TIMEOUT",
+}
+
+EXPORTED = ("hf_align_build", "hf_plan_workspace_size", "hf_plan_create", "hf_transfer",
+            "hf_plan_destroy", "hf_plan_device_status", "hf_plan_distinct_rows",
+            "hf_status_string", "hf_last_error")
+
+_p = ctypes.c_void_p
+_i32p = ctypes.POINTER(ctypes.c_int32)
+_f32p = ctypes.POINTER(ctypes.c_float)
+
+
+class PlanDesc(ctypes.Structure):
+    """Mirror of hf_plan_desc."""
+    _fields_ = [
+        ("L_s", ctypes.c_int32), ("H_s", ctypes.c_int32), ("D_s", ctypes.c_int32),
+        ("L_r", ctypes.c_int32), ("H_r", ctypes.c_int32), ("D_r", ctypes.c_int32),
+        ("dtype", ctypes.c_int), ("layer_mode", ctypes.c_int), ("align_mode", ctypes.c_int),
+        ("n_req", ctypes.c_int32),
+        ("s_tok_ptr", _i32p), ("r_tok_ptr", _i32p), ("r_pos0", _i32p),
+        ("d_row_ptr", _p), ("d_col", _p), ("d_w", _p),
+        ("d_W", _p), ("d_b", _p), ("h_r", _f32p),
+        ("theta_r", ctypes.c_double),
+        ("d_knorm_w", _p), ("knorm_eps", ctypes.c_float),
+        ("paged", ctypes.c_int32), ("block_size", ctypes.c_int32),
+        ("n_blocks", ctypes.c_int32), ("max_blocks_per_req", ctypes.c_int32),
+        ("d_block_table", _p),
+    ]
+
+
+class HFError(RuntimeError):
+    def __init__(self, status: int, where: str, msg: str):
+        super().__init__(f"{where}: status {status}: {msg}")
+        self.status = status
+
+
+_LIB: Optional[ctypes.CDLL] = None
+
+
+def lib() -> ctypes.CDLL:
+    global _LIB
+    if _LIB is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(
+                f"{LIB_PATH} is missing: build it first "
+                "(python -c 'import __graft_entry__ as g; g.build()'); there is no CPU fallback")
+        L = ctypes.CDLL(LIB_PATH)
+        L.hf_align_build.argtypes = [ctypes.c_int, ctypes.c_int32, _i32p, _i32p, _p, _p, _p, _p,
+                                     _p, ctypes.c_int64, _p, _p]
+        L.hf_plan_workspace_size.argtypes = [ctypes.POINTER(PlanDesc), ctypes.POINTER(ctypes.c_size_t)]
+        L.hf_plan_create.argtypes = [ctypes.POINTER(PlanDesc), _p, ctypes.c_size_t, _p,
+                                     ctypes.POINTER(ctypes.c_void_p)]
+        L.hf_transfer.argtypes = [_p, _p, _p, _p]
+        L.hf_plan_destroy.argtypes = [_p]
+        L.hf_plan_device_status.argtypes = [_p, _p, _i32p]
+        L.hf_plan_distinct_rows.argtypes = [_p, _p, _i32p]
+        L.hf_status_string.argtypes = [ctypes.c_int]
+        L.hf_status_string.restype = ctypes.c_char_p
+        L.hf_last_error.argtypes = []
+        L.hf_last_error.restype = ctypes.c_char_p
+        for name in ("hf_align_build", "hf_plan_workspace_size", "hf_plan_create", "hf_transfer",
+                     "hf_plan_destroy", "hf_plan_device_status", "hf_plan_distinct_rows"):
+            getattr(L, name).restype = ctypes.c_int
+        _LIB = L
+    return _LIB
+
+
+def _check(status: int, where: str) -> None:
+    if status != HF_OK:
+        raise HFError(status, where, lib().hf_last_error().decode(errors="replace"))
+
+
+def _dptr(x) -> Optional[int]:
+    """Device pointer of a torch tensor (or an int / None)."""
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    return int(x.data_ptr())
+
+
+def _stream(stream) -> Optional[int]:
+    if stream is None:
+        return None
+    if isinstance(stream, int):
+        return stream
+    return int(stream.cuda_stream)
+
+
+def _host_i32(a) -> np.ndarray:
+    return np.ascontiguousarray(np.asarray(a, dtype=np.int32))
+
+
+def _as_i32p(a: np.ndarray):
+    return a.ctypes.data_as(_i32p)
+
+
+def align_build(mode: str, s_tok_ptr, r_tok_ptr, d_s_end, d_r_end, d_row_ptr, d_col, d_w,
+                nnz_capacity: int, d_info, stream=None) -> None:
+    """hf_align_build.  Host token pointers (numpy), device arrays (torch)."""
+    s = _host_i32(s_tok_ptr)
+    r = _host_i32(r_tok_ptr)
+    st = lib().hf_align_build(ALIGN_MODES[mode], len(r) - 1, _as_i32p(s), _as_i32p(r),
+                              _dptr(d_s_end), _dptr(d_r_end), _dptr(d_row_ptr), _dptr(d_col),
+                              _dptr(d_w), int(nnz_capacity), _dptr(d_info), _stream(stream))
+    _check(st, "hf_align_build")
+
+
+class Desc:
+    """Builds an hf_plan_desc and keeps its host arrays alive."""
+
+    def __init__(self, *, L_s, H_s, D_s, L_r, H_r, D_r, dtype, layer_mode, align_mode,
+                 s_tok_ptr, r_tok_ptr, d_row_ptr, d_col, d_w, d_W, d_b, r, theta_r,
+                 r_pos0=None, d_knorm_w=None, knorm_eps=1e-6, paged=False, block_size=16,
+                 n_blocks=0, max_blocks_per_req=0, d_block_table=None):
+        self._s = _host_i32(s_tok_ptr)
+        self._r = _host_i32(r_tok_ptr)
+        self._pos0 = None if r_pos0 is None else _host_i32(r_pos0)
+        self._hr = np.ascontiguousarray(np.asarray(r, dtype=np.float32).reshape(-1))
+        self.c = PlanDesc(
+            L_s=L_s, H_s=H_s, D_s=D_s, L_r=L_r, H_r=H_r, D_r=D_r,
+            dtype=DTYPES[dtype], layer_mode=LAYER_MODES[layer_mode],
+            align_mode=ALIGN_MODES[align_mode], n_req=len(self._r) - 1,
+            s_tok_ptr=_as_i32p(self._s), r_tok_ptr=_as_i32p(self._r),
+            r_pos0=_as_i32p(self._pos0) if self._pos0 is not None else None,
+            d_row_ptr=_dptr(d_row_ptr), d_col=_dptr(d_col), d_w=_dptr(d_w),
+            d_W=_dptr(d_W), d_b=_dptr(d_b), h_r=self._hr.ctypes.data_as(_f32p),
+            theta_r=float(theta_r), d_knorm_w=_dptr(d_knorm_w), knorm_eps=float(knorm_eps),
+            paged=int(bool(paged)), block_size=int(block_size), n_blocks=int(n_blocks),
+            max_blocks_per_req=int(max_blocks_per_req), d_block_table=_dptr(d_block_table))
+
+
+def plan_workspace_size(desc: Desc) -> int:
+    n = ctypes.c_size_t(0)
+    _check(lib().hf_plan_workspace_size(ctypes.byref(desc.c), ctypes.byref(n)),
+           "hf_plan_workspace_size")
+    return int(n.value)
+
+
+class Plan:
+    """An hf_plan handle; destroy() (or garbage collection) releases it."""
+
+    def __init__(self, handle: int, desc: Desc, workspace):
+        self.handle = handle
+        self.desc = desc
+        self.workspace = workspace
+
+    def destroy(self) -> None:
+        if self.handle:
+            _check(lib().hf_plan_destroy(self.handle), "hf_plan_destroy")
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.destroy()
+        except Exception:
+            pass
+
+
+def plan_create(desc: Desc, workspace, stream=None) -> Plan:
+    h = ctypes.c_void_p(0)
+    nbytes = int(workspace.numel() * workspace.element_size()) if hasattr(workspace, "numel") else 0
+    _check(lib().hf_plan_create(ctypes.byref(desc.c), _dptr(workspace), nbytes, _stream(stream),
+                                ctypes.byref(h)), "hf_plan_create")
+    return Plan(h.value, desc, workspace)
+
+
+def transfer(plan: Plan, sender_kv, receiver_kv, stream=None) -> None:
+    _check(lib().hf_transfer(plan.handle, _dptr(sender_kv), _dptr(receiver_kv), _stream(stream)),
+           "hf_transfer")
+
+
+def plan_device_status(plan: Plan, stream=None) -> int:
+    v = ctypes.c_int32(0)
+    st = lib().hf_plan_device_status(plan.handle, _stream(stream), ctypes.byref(v))
+    if st not in (HF_OK, HF_ERR_DEVICE_CHECK):
+        _check(st, "hf_plan_device_status")
+    return int(v.value)
+
+
+def plan_distinct_rows(plan: Plan, stream=None) -> int:
+    v = ctypes.c_int32(0)
+    _check(lib().hf_plan_distinct_rows(plan.handle, _stream(stream), ctypes.byref(v)),
+           "hf_plan_distinct_rows")
+    return int(v.value)
+
+
+def status_string(status: int) -> str:
+    return lib().hf_status_string(int(status)).decode()
+
+
+def decode_check_bits(bits: int):
+    return [name for b, name in CHECK_BITS.items() if bits & b]

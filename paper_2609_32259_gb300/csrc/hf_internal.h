@@ -1,0 +1,88 @@
+// Internal declarations shared by the library's translation units.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <string>
+
+#include "heterofold.h"
+
+namespace hf {
+
+constexpr int kMaxReq = 1024;        // requests per call
+constexpr int kMaxLayersR = 128;     // receiver layers
+constexpr int kMaxSeg = 3;           // map input segments per receiver layer
+constexpr int kMaxTerms = 2;         // sender layers blended into one segment
+constexpr int kMaxHeadDim = 256;
+
+// One receiver layer's map input: n_seg segments of d_S features each;
+// segment s is sum_t w[s][t] * (pooled sender layer layer[s][t]).
+struct LayerSegs {
+  int32_t n_seg;
+  int32_t n_terms[kMaxSeg];
+  int32_t layer[kMaxSeg][kMaxTerms];
+  float w[kMaxSeg][kMaxTerms];
+};
+
+// Per-plan metadata that lives in the caller's device workspace.
+struct WorkspaceLayout {
+  size_t status;     // int32: device status bits
+  size_t n_distinct; // int32: number of distinct alignment rows U
+  size_t segs;       // LayerSegs[L_r]
+  size_t inv_r;      // float[L_r * 2]  (1 / r)
+  size_t inv_freq;   // float[D_r / 2]
+  size_t r_tok_ptr;  // int32[n_req + 1]
+  size_t r_pos0;     // int32[n_req]
+  size_t run_ptr;    // int32[T_r + 1]: first receiver row of each distinct row
+  size_t ucol;       // int32[T_r]: sender column of each distinct row (one-entry rows)
+  size_t pos;        // int32[T_r]: RoPE position of each receiver row
+  size_t dst_row;    // int32[T_r]: destination row of each receiver row
+  size_t new_flag;   // int32[T_r]: 1 where a receiver row starts a new distinct row
+  size_t total;
+};
+
+WorkspaceLayout workspace_layout(int L_r, int D_r, int n_req, int64_t T_r);
+
+// Constant tables copied into the workspace by the plan kernel (passed by
+// value as a kernel parameter, so plan creation issues no host copies).
+struct PlanTables {
+  int32_t L_r, D_r, n_req;
+  LayerSegs segs[kMaxLayersR];
+  float inv_r[2 * kMaxLayersR];
+  float inv_freq[kMaxHeadDim / 2];
+  int32_t r_tok_ptr[kMaxReq + 1];
+  int32_t r_pos0[kMaxReq];
+};
+
+}  // namespace hf
+
+struct hf_plan_s {
+  hf_plan_desc desc;  // host-array fields are cleared after copying
+  int d_s, d_r, K, n_seg;
+  int64_t T_s, T_r, nnz_hint;
+  int BN, groups, stages;
+  bool gather;  // every map input row is a single unweighted sender row
+  char* ws;
+  size_t ws_bytes;
+  hf::WorkspaceLayout lay;
+  int32_t s_tok_ptr_last;
+};
+
+namespace hf {
+
+void set_error(const std::string& msg);
+hf_status cuda_fail(cudaError_t e, const char* what);
+int device_sm_count();
+
+hf_status launch_plan_kernels(hf_plan_s* p, const PlanTables& tables, cudaStream_t stream);
+hf_status launch_transfer(hf_plan_s* p, const void* sender, void* receiver, cudaStream_t stream);
+
+}  // namespace hf
+
+#define HF_CUDA_TRY(expr, what)                      \
+  do {                                               \
+    cudaError_t e__ = (expr);                        \
+    if (e__ != cudaSuccess) return hf::cuda_fail(e__, what); \
+  } while (0)

@@ -1,0 +1,448 @@
+// Plan creation: descriptor validation, the layer table (Eq. 1 or the
+// interpolation reading), RoPE inverse frequencies, and the per-transfer
+// device metadata (receiver positions and destination rows, runs of
+// identical alignment rows).  Also the error-reporting helpers of the ABI.
+#include <cmath>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+#include <string>
+
+#include "hf_device.cuh"
+#include "hf_internal.h"
+#include "hf_scan.cuh"
+
+namespace hf {
+
+namespace {
+thread_local std::string g_last_error;
+}
+
+void set_error(const std::string& msg) { g_last_error = msg; }
+
+hf_status cuda_fail(cudaError_t e, const char* what) {
+  set_error(std::string(what) + ": " + cudaGetErrorString(e));
+  return HF_ERR_CUDA;
+}
+
+int device_sm_count() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 1;
+  int n = 0;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1)
+    return 1;
+  return n;
+}
+
+static size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+WorkspaceLayout workspace_layout(int L_r, int D_r, int n_req, int64_t T_r) {
+  WorkspaceLayout w{};
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = off;
+    off = align_up(off + bytes, 256);
+    return at;
+  };
+  w.status = take(sizeof(int32_t));
+  w.n_distinct = take(sizeof(int32_t));
+  w.segs = take(sizeof(LayerSegs) * (size_t)L_r);
+  w.inv_r = take(sizeof(float) * 2 * (size_t)L_r);
+  w.inv_freq = take(sizeof(float) * (size_t)(D_r / 2 > 0 ? D_r / 2 : 1));
+  w.r_tok_ptr = take(sizeof(int32_t) * (size_t)(n_req + 1));
+  w.r_pos0 = take(sizeof(int32_t) * (size_t)n_req);
+  w.run_ptr = take(sizeof(int32_t) * (size_t)(T_r + 1));
+  w.ucol = take(sizeof(int32_t) * (size_t)(T_r > 0 ? T_r : 1));
+  w.pos = take(sizeof(int32_t) * (size_t)(T_r > 0 ? T_r : 1));
+  w.dst_row = take(sizeof(int32_t) * (size_t)(T_r > 0 ? T_r : 1));
+  w.new_flag = take(sizeof(int32_t) * (size_t)(T_r > 0 ? T_r : 1));
+  w.total = off;
+  return w;
+}
+
+namespace {
+
+struct PlanDev {
+  int32_t* status;
+  int32_t* n_distinct;
+  LayerSegs* segs;
+  float* inv_r;
+  float* inv_freq;
+  int32_t* r_tok_ptr;
+  int32_t* r_pos0;
+  int32_t* run_ptr;
+  int32_t* ucol;
+  int32_t* pos;
+  int32_t* dst_row;
+  int32_t* new_flag;
+};
+
+PlanDev plan_dev(const hf_plan_s* p) {
+  auto at = [&](size_t off) { return p->ws + off; };
+  PlanDev d;
+  d.status = reinterpret_cast<int32_t*>(at(p->lay.status));
+  d.n_distinct = reinterpret_cast<int32_t*>(at(p->lay.n_distinct));
+  d.segs = reinterpret_cast<LayerSegs*>(at(p->lay.segs));
+  d.inv_r = reinterpret_cast<float*>(at(p->lay.inv_r));
+  d.inv_freq = reinterpret_cast<float*>(at(p->lay.inv_freq));
+  d.r_tok_ptr = reinterpret_cast<int32_t*>(at(p->lay.r_tok_ptr));
+  d.r_pos0 = reinterpret_cast<int32_t*>(at(p->lay.r_pos0));
+  d.run_ptr = reinterpret_cast<int32_t*>(at(p->lay.run_ptr));
+  d.ucol = reinterpret_cast<int32_t*>(at(p->lay.ucol));
+  d.pos = reinterpret_cast<int32_t*>(at(p->lay.pos));
+  d.dst_row = reinterpret_cast<int32_t*>(at(p->lay.dst_row));
+  d.new_flag = reinterpret_cast<int32_t*>(at(p->lay.new_flag));
+  return d;
+}
+
+// Copies the constant tables into the workspace and clears the counters.
+__global__ void plan_init_kernel(PlanTables t, PlanDev d) {
+  const int tid = threadIdx.x;
+  if (tid == 0) {
+    *d.status = 0;
+    *d.n_distinct = 0;
+  }
+  for (int i = tid; i < t.L_r; i += blockDim.x) d.segs[i] = t.segs[i];
+  for (int i = tid; i < 2 * t.L_r; i += blockDim.x) d.inv_r[i] = t.inv_r[i];
+  for (int i = tid; i < t.D_r / 2; i += blockDim.x) d.inv_freq[i] = t.inv_freq[i];
+  for (int i = tid; i <= t.n_req; i += blockDim.x) d.r_tok_ptr[i] = t.r_tok_ptr[i];
+  for (int i = tid; i < t.n_req; i += blockDim.x) d.r_pos0[i] = t.r_pos0[i];
+}
+
+struct RowArgs {
+  PlanDev d;
+  const int32_t* row_ptr;
+  const int32_t* col;
+  const float* w;
+  const int32_t* block_table;
+  int64_t T_r;
+  int64_t T_s;
+  int n_req;
+  int paged, block_size, n_blocks, max_blocks;
+  int single_entry;  // rows must be one entry of weight 1
+};
+
+__device__ __forceinline__ void flag(int32_t* status, int bits) { atomicOr(status, bits); }
+
+// Per receiver row: position, destination row, checks, and whether the row
+// differs from the previous one (starts a new distinct row).
+__global__ void plan_rows_kernel(RowArgs a) {
+  const PlanDev& d = a.d;
+  for (int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; j < a.T_r;
+       j += (int64_t)gridDim.x * blockDim.x) {
+    const int q = find_request(d.r_tok_ptr, a.n_req, j);
+    const int32_t r0 = d.r_tok_ptr[q];
+    const int32_t t = static_cast<int32_t>(j - r0);
+    d.pos[j] = d.r_pos0[q] + t;
+    int32_t dst = static_cast<int32_t>(j);
+    if (a.paged) {
+      const int bi = t / a.block_size;
+      int32_t blk = -1;
+      if (bi < a.max_blocks) blk = a.block_table[(int64_t)q * a.max_blocks + bi];
+      if (blk < 0 || blk >= a.n_blocks) {
+        flag(d.status, HF_CHECK_BAD_BLOCK);
+        dst = -1;
+      } else {
+        dst = blk * a.block_size + t % a.block_size;
+      }
+    }
+    d.dst_row[j] = dst;
+    const int32_t e0 = a.row_ptr[j], e1 = a.row_ptr[j + 1];
+    if (e1 <= e0) flag(d.status, HF_CHECK_BAD_ROW);
+    if (a.single_entry && (e1 - e0 != 1 || a.w[e0] != 1.0f)) flag(d.status, HF_CHECK_BAD_ROW);
+    for (int32_t e = e0; e < e1; ++e) {
+      const int32_t k = a.col[e];
+      if (k < 0 || k >= a.T_s) flag(d.status, HF_CHECK_BAD_COLUMN);
+    }
+    int is_new = (j == r0) ? 1 : 0;
+    if (!is_new) {
+      const int32_t p0 = a.row_ptr[j - 1];
+      if (e1 - e0 != e0 - p0) {
+        is_new = 1;
+      } else {
+        for (int32_t i = 0; i < e1 - e0; ++i) {
+          if (a.col[e0 + i] != a.col[p0 + i] || a.w[e0 + i] != a.w[p0 + i]) {
+            is_new = 1;
+            break;
+          }
+        }
+      }
+    }
+    d.new_flag[j] = is_new;
+  }
+}
+
+// After the inclusive scan new_flag[j] = (index of j's distinct row) + 1.
+__global__ void plan_runs_kernel(RowArgs a) {
+  const PlanDev& d = a.d;
+  for (int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; j < a.T_r;
+       j += (int64_t)gridDim.x * blockDim.x) {
+    const int32_t incl = d.new_flag[j];
+    const bool starts = (j == 0) || (incl != d.new_flag[j - 1]);
+    if (starts) {
+      const int32_t u = incl - 1;
+      d.run_ptr[u] = static_cast<int32_t>(j);
+      int32_t k = a.col[a.row_ptr[j]];
+      if (k < 0 || k >= a.T_s) k = 0;  // flagged by plan_rows_kernel
+      d.ucol[u] = k;
+    }
+    if (j == a.T_r - 1) {
+      d.run_ptr[incl] = static_cast<int32_t>(a.T_r);
+      *d.n_distinct = incl;
+    }
+  }
+}
+
+// Eq. 1: pi(l) = 1 + round((l-1)(L_S-1)/(L_R-1)) (one-based), round half
+// away from zero, computed exactly in integers.
+int proportional_depth(int l1, int L_s, int L_r) {
+  if (L_r == 1) return 1;
+  const long long num = (long long)(l1 - 1) * (L_s - 1);
+  const long long den = L_r - 1;
+  return 1 + static_cast<int>((2 * num + den) / (2 * den));
+}
+
+void build_layer_table(const hf_plan_desc& d, LayerSegs* out) {
+  for (int l = 0; l < d.L_r; ++l) {
+    LayerSegs s;
+    std::memset(&s, 0, sizeof(s));
+    if (d.layer_mode == HF_LAYER_PAPER3) {
+      // N(l) = clip(pi - 4, pi, pi + 4) to [1, L_S], one segment each.
+      const int pi = proportional_depth(l + 1, d.L_s, d.L_r);
+      const int offs[3] = {-4, 0, 4};
+      s.n_seg = 3;
+      for (int k = 0; k < 3; ++k) {
+        int t = pi + offs[k];
+        t = t < 1 ? 1 : (t > d.L_s ? d.L_s : t);
+        s.n_terms[k] = 1;
+        s.layer[k][0] = t - 1;
+        s.w[k][0] = 1.0f;
+      }
+    } else {
+      // p = l (L_S - 1)/(L_R - 1); blend floor(p) and floor(p)+1 by (1-f, f).
+      const double p = d.L_r > 1 ? (double)(l * (d.L_s - 1)) / (double)(d.L_r - 1) : 0.0;
+      const int i0 = static_cast<int>(std::floor(p));
+      const double f = p - i0;
+      s.n_seg = 1;
+      s.layer[0][0] = i0;
+      s.w[0][0] = static_cast<float>(1.0 - f);
+      s.n_terms[0] = 1;
+      if (f > 0.0) {
+        s.n_terms[0] = 2;
+        s.layer[0][1] = i0 + 1 < d.L_s ? i0 + 1 : d.L_s - 1;
+        s.w[0][1] = static_cast<float>(f);
+      }
+    }
+    out[l] = s;
+  }
+}
+
+hf_status validate(const hf_plan_desc* d) {
+  auto bad = [](const char* m) {
+    set_error(std::string("hf_plan_create: ") + m);
+    return HF_ERR_INVALID_ARGUMENT;
+  };
+  auto unsup = [](const char* m) {
+    set_error(std::string("hf_plan_create: unsupported: ") + m);
+    return HF_ERR_UNSUPPORTED;
+  };
+  if (!d) return bad("null descriptor");
+  if (d->L_s < 1 || d->H_s < 1 || d->D_s < 1 || d->L_r < 1 || d->H_r < 1 || d->D_r < 1)
+    return bad("shapes must be positive");
+  if (d->dtype != HF_BF16 && d->dtype != HF_F32) return bad("unknown dtype");
+  if (d->layer_mode != HF_LAYER_PAPER3 && d->layer_mode != HF_LAYER_INTERP)
+    return bad("unknown layer mode");
+  if (d->align_mode != HF_ALIGN_TA && d->align_mode != HF_ALIGN_OVERLAP_MEAN &&
+      d->align_mode != HF_ALIGN_SAME_INDEX)
+    return bad("unknown align mode");
+  if (d->n_req < 1 || d->n_req > kMaxReq) return bad("n_req must be in [1, 1024]");
+  if (!d->s_tok_ptr || !d->r_tok_ptr) return bad("null token pointers");
+  if (d->s_tok_ptr[0] != 0 || d->r_tok_ptr[0] != 0) return bad("token pointers must start at 0");
+  for (int q = 0; q < d->n_req; ++q) {
+    if (d->s_tok_ptr[q + 1] < d->s_tok_ptr[q] || d->r_tok_ptr[q + 1] < d->r_tok_ptr[q])
+      return bad("token pointers must be non-decreasing");
+    if (d->r_tok_ptr[q + 1] > d->r_tok_ptr[q] && d->s_tok_ptr[q + 1] == d->s_tok_ptr[q])
+      return bad("a request has receiver tokens but no sender token");
+  }
+  if (!d->d_row_ptr || !d->d_W || !d->d_b || !d->h_r) return bad("null CSR or map pointer");
+  if (d->r_tok_ptr[d->n_req] > 0 && (!d->d_col || !d->d_w)) return bad("null CSR arrays");
+  for (int i = 0; i < 2 * d->L_r; ++i)
+    if (!(d->h_r[i] > 0.0f) || !std::isfinite(d->h_r[i])) return bad("r must be positive");
+  if (d->L_r > kMaxLayersR) return unsup("more than 128 receiver layers");
+  const int esize = d->dtype == HF_BF16 ? 2 : 4;
+  const int bke = 128 / esize;  // elements per 128-byte k-block
+  const int d_s = d->H_s * d->D_s, d_r = d->H_r * d->D_r;
+  if (d_s % bke) return unsup("d_S must be a multiple of 64 (bf16) or 32 (fp32)");
+  if (d_r % 128) return unsup("d_R must be a multiple of 128");
+  if (d->D_r % 32 || d->D_r > kMaxHeadDim) return unsup("D_r must be a multiple of 32, <= 256");
+  const int BN = (d_r % 256 == 0) ? 256 : 128;
+  if (BN % d->D_r) return unsup("a receiver head must fit one 128/256-column tile");
+  if (d->paged) {
+    if (d->block_size < 1 || d->n_blocks < 1 || d->max_blocks_per_req < 1 || !d->d_block_table)
+      return bad("paged layout needs block_size, n_blocks, max_blocks_per_req, d_block_table");
+  }
+  const long long rows = (long long)d->L_s * 2 * d->s_tok_ptr[d->n_req];
+  if (rows >= (1LL << 31)) return unsup("sender cache has more than 2^31 rows");
+  return HF_OK;
+}
+
+}  // namespace
+
+hf_status launch_plan_kernels(hf_plan_s* p, const PlanTables& tables, cudaStream_t stream) {
+  const PlanDev d = plan_dev(p);
+  plan_init_kernel<<<1, 256, 0, stream>>>(tables, d);
+  HF_CUDA_TRY(cudaGetLastError(), "plan init launch");
+  if (p->T_r == 0) return HF_OK;
+  RowArgs a;
+  a.d = d;
+  a.row_ptr = p->desc.d_row_ptr;
+  a.col = p->desc.d_col;
+  a.w = p->desc.d_w;
+  a.block_table = p->desc.d_block_table;
+  a.T_r = p->T_r;
+  a.T_s = p->T_s;
+  a.n_req = p->desc.n_req;
+  a.paged = p->desc.paged;
+  a.block_size = p->desc.block_size > 0 ? p->desc.block_size : 1;
+  a.n_blocks = p->desc.n_blocks;
+  a.max_blocks = p->desc.max_blocks_per_req;
+  a.single_entry = p->desc.align_mode != HF_ALIGN_OVERLAP_MEAN;
+  const int64_t want = (p->T_r + 255) / 256;
+  const int grid = static_cast<int>(std::min<int64_t>(want, 8LL * device_sm_count()));
+  plan_rows_kernel<<<grid, 256, 0, stream>>>(a);
+  scan_inplace_kernel<ScanSum><<<1, kScanThreads, 0, stream>>>(d.new_flag, p->T_r, nullptr);
+  plan_runs_kernel<<<grid, 256, 0, stream>>>(a);
+  HF_CUDA_TRY(cudaGetLastError(), "plan kernels launch");
+  return HF_OK;
+}
+
+}  // namespace hf
+
+using namespace hf;
+
+extern "C" hf_status hf_plan_workspace_size(const hf_plan_desc* desc, size_t* bytes) {
+  if (!desc || !bytes || !desc->r_tok_ptr || desc->n_req < 1 || desc->n_req > kMaxReq) {
+    set_error("hf_plan_workspace_size: invalid descriptor");
+    return HF_ERR_INVALID_ARGUMENT;
+  }
+  *bytes = workspace_layout(desc->L_r, desc->D_r, desc->n_req, desc->r_tok_ptr[desc->n_req]).total;
+  return HF_OK;
+}
+
+extern "C" hf_status hf_plan_create(const hf_plan_desc* desc, void* d_workspace,
+                                    size_t workspace_bytes, hf_stream_t stream_, hf_plan* out) {
+  if (!out) {
+    set_error("hf_plan_create: null output handle");
+    return HF_ERR_INVALID_ARGUMENT;
+  }
+  *out = nullptr;
+  const hf_status v = validate(desc);
+  if (v != HF_OK) return v;
+  const WorkspaceLayout lay =
+      workspace_layout(desc->L_r, desc->D_r, desc->n_req, desc->r_tok_ptr[desc->n_req]);
+  if (!d_workspace || workspace_bytes < lay.total ||
+      (reinterpret_cast<uintptr_t>(d_workspace) & 255u)) {
+    set_error("hf_plan_create: workspace missing, too small or not 256-byte aligned");
+    return HF_ERR_WORKSPACE;
+  }
+  hf_plan_s* p = new hf_plan_s();
+  p->desc = *desc;
+  p->d_s = desc->H_s * desc->D_s;
+  p->d_r = desc->H_r * desc->D_r;
+  p->n_seg = desc->layer_mode == HF_LAYER_PAPER3 ? 3 : 1;
+  p->K = p->n_seg * p->d_s;
+  p->T_s = desc->s_tok_ptr[desc->n_req];
+  p->T_r = desc->r_tok_ptr[desc->n_req];
+  p->BN = (p->d_r % 256 == 0) ? 256 : 128;
+  p->groups = ((p->BN / 2) % desc->D_r == 0) ? 2 : 1;
+  p->gather = desc->layer_mode == HF_LAYER_PAPER3 && desc->align_mode != HF_ALIGN_OVERLAP_MEAN;
+  p->ws = static_cast<char*>(d_workspace);
+  p->ws_bytes = workspace_bytes;
+  p->lay = lay;
+  // host arrays are not kept
+  p->desc.s_tok_ptr = nullptr;
+  p->desc.r_tok_ptr = nullptr;
+  p->desc.r_pos0 = nullptr;
+  p->desc.h_r = nullptr;
+
+  PlanTables* t = new PlanTables();
+  std::memset(t, 0, sizeof(*t));
+  t->L_r = desc->L_r;
+  t->D_r = desc->D_r;
+  t->n_req = desc->n_req;
+  build_layer_table(*desc, t->segs);
+  for (int i = 0; i < 2 * desc->L_r; ++i) t->inv_r[i] = static_cast<float>(1.0 / desc->h_r[i]);
+  // inv_freq_i = fp32(theta^(-2i/D)) evaluated in double precision
+  for (int i = 0; i < desc->D_r / 2; ++i)
+    t->inv_freq[i] = desc->theta_r > 0.0
+                         ? static_cast<float>(std::pow(desc->theta_r, -(2.0 * i) / desc->D_r))
+                         : 0.0f;
+  for (int q = 0; q <= desc->n_req; ++q) t->r_tok_ptr[q] = desc->r_tok_ptr[q];
+  for (int q = 0; q < desc->n_req; ++q) t->r_pos0[q] = desc->r_pos0 ? desc->r_pos0[q] : 0;
+  const hf_status s = launch_plan_kernels(p, *t, reinterpret_cast<cudaStream_t>(stream_));
+  delete t;
+  if (s != HF_OK) {
+    delete p;
+    return s;
+  }
+  *out = p;
+  return HF_OK;
+}
+
+extern "C" hf_status hf_plan_destroy(hf_plan plan) {
+  delete plan;
+  return HF_OK;
+}
+
+static hf_status read_word(hf_plan plan, hf_stream_t stream_, size_t off, int32_t* outv) {
+  if (!plan || !outv) {
+    set_error("null plan or output");
+    return HF_ERR_INVALID_ARGUMENT;
+  }
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  int32_t v = 0;
+  HF_CUDA_TRY(cudaMemcpyAsync(&v, plan->ws + off, sizeof(v), cudaMemcpyDeviceToHost, stream),
+              "read device word");
+  HF_CUDA_TRY(cudaStreamSynchronize(stream), "stream synchronize");
+  *outv = v;
+  return HF_OK;
+}
+
+extern "C" hf_status hf_plan_device_status(hf_plan plan, hf_stream_t stream, int32_t* flags) {
+  if (!plan) {
+    set_error("null plan");
+    return HF_ERR_INVALID_ARGUMENT;
+  }
+  const hf_status s = read_word(plan, stream, plan->lay.status, flags);
+  if (s != HF_OK) return s;
+  if (*flags != 0) {
+    char buf[96];
+    std::snprintf(buf, sizeof(buf), "device checks failed: status bits 0x%x", *flags);
+    set_error(buf);
+    return HF_ERR_DEVICE_CHECK;
+  }
+  return HF_OK;
+}
+
+extern "C" hf_status hf_plan_distinct_rows(hf_plan plan, hf_stream_t stream, int32_t* n_rows) {
+  if (!plan) {
+    set_error("null plan");
+    return HF_ERR_INVALID_ARGUMENT;
+  }
+  return read_word(plan, stream, plan->lay.n_distinct, n_rows);
+}
+
+extern "C" const char* hf_status_string(hf_status s) {
+  switch (s) {
+    case HF_OK: return "ok";
+    case HF_ERR_INVALID_ARGUMENT: return "invalid argument";
+    case HF_ERR_UNSUPPORTED: return "unsupported";
+    case HF_ERR_CUDA: return "CUDA error";
+    case HF_ERR_DEVICE_CHECK: return "device check failed";
+    case HF_ERR_WORKSPACE: return "bad workspace";
+  }
+  return "unknown status";
+}
+
+extern "C" const char* hf_last_error(void) { return g_last_error.c_str(); }

@@ -1,0 +1,145 @@
+"""Shared machinery of the GPU parity tests: generate a workload's inputs on
+the device, run the transfer through the C ABI, and compare with the fp64
+oracle fed from the same seeded inputs."""
+
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from oracle import heterofold_oracle as O
+from paper_2609_32259_gb300 import pipeline
+from paper_2609_32259_gb300 import workloads as W
+
+# Tolerances of the transfer against the fp64 oracle (bf16 inputs, fp32
+# accumulation): per receiver layer and role.
+REL_FRO_TOL = 5e-3
+MAX_ABS_TOL = 2e-2
+
+
+class RowFetcher:
+    """sender[t][c][rows] -> fp32 numpy rows, fetched from the device on demand."""
+
+    def __init__(self, sender: torch.Tensor):
+        self.s = sender
+
+    class _LC:
+        def __init__(self, t):
+            self.t = t
+
+        def __getitem__(self, idx):
+            ix = torch.as_tensor(np.asarray(idx, dtype=np.int64), device=self.t.device)
+            return self.t.index_select(0, ix).float().cpu().numpy()
+
+    class _L:
+        def __init__(self, t):
+            self.t = t
+
+        def __getitem__(self, c):
+            return RowFetcher._LC(self.t[c])
+
+    def __getitem__(self, t):
+        return RowFetcher._L(self.s[t])
+
+
+class MapFetcher:
+    """A[l][c] = W[l][c]^T as fp64 numpy (the paper's x @ A orientation)."""
+
+    def __init__(self, Wm: torch.Tensor):
+        self.W = Wm
+
+    class _L:
+        def __init__(self, Wl):
+            self.Wl = Wl
+
+        def __getitem__(self, c):
+            return self.Wl[c].float().cpu().numpy().T
+
+    def __getitem__(self, l):
+        return MapFetcher._L(self.W[l])
+
+
+class Case:
+    def __init__(self, w: W.Workload, device="cuda", sentinel=None):
+        self.w = w
+        self.dev = torch.device(device)
+        self.tok = W.tokens(w)
+        self.sender = W.sender_kv(w, self.tok.T_s, self.dev)
+        self.Wm, self.b, self.r = W.maps(w, self.dev)
+        self.paged = W.paged_layout(w, self.tok) if w.paged else None
+        self.knorm_w = W.knorm_weight(w)
+        self.r_pos0 = W.r_pos0(w)
+        self.job = pipeline.job_from_workload(w, self.tok, self.sender, self.Wm, self.b, self.r,
+                                              paged=self.paged, knorm_w=self.knorm_w,
+                                              r_pos0=self.r_pos0, device=self.dev)
+        if sentinel is not None:
+            self.job.receiver.fill_(sentinel)
+        self.csr = O.alignment_csr(w.align_mode, self.tok.s_tok_ptr, self.tok.r_tok_ptr,
+                                   self.tok.s_end, self.tok.r_end)
+        self.segs = O.layer_segments(w.layer_mode, w.L_s, w.L_r)
+        self.pos = O.receiver_positions(self.tok.r_tok_ptr, self.r_pos0)
+
+    def run(self):
+        self.job.step()
+        torch.cuda.synchronize()
+        return self
+
+    # --------------------------------------------------------------- checks
+    def check_csr(self):
+        rp, col, wt = self.job.csr()
+        assert self.job.align_status() == 0, self.job.align_status()
+        assert np.array_equal(rp, self.csr.row_ptr.astype(np.int32))
+        assert np.array_equal(col, self.csr.col.astype(np.int32))
+        assert np.array_equal(wt.view(np.uint32), self.csr.w32.view(np.uint32))
+
+    def dst_rows(self, rows):
+        rows = np.asarray(rows, dtype=np.int64)
+        if self.paged is None:
+            return rows
+        rp = self.tok.r_tok_ptr
+        q = np.searchsorted(rp, rows, side="right") - 1
+        t = rows - rp[q]
+        bs = self.w.block_size
+        return self.paged.block_table[q, t // bs].astype(np.int64) * bs + t % bs
+
+    def gpu_rows(self, l, c, rows):
+        d = torch.as_tensor(self.dst_rows(rows), device=self.dev)
+        y = self.job.receiver[l, c].index_select(0, d).double().cpu().numpy()
+        return y.reshape(len(rows), self.w.H_r, self.w.D_r)
+
+    def oracle(self, layers, rows, roles=(0, 1)):
+        return O.transfer(RowFetcher(self.sender), self.csr, self.segs, MapFetcher(self.Wm),
+                          self.b.cpu().numpy(), self.r, H_r=self.w.H_r, D_r=self.w.D_r,
+                          pos=self.pos, inv_freq_r=O.rope_inv_freq(self.w.theta_r, self.w.D_r),
+                          knorm_g=self.knorm_w, knorm_eps=1e-6, layers=layers, rows=rows,
+                          roles=roles)
+
+    def check_parity(self, layers=None, rows=None, rel_tol=REL_FRO_TOL, abs_tol=MAX_ABS_TOL):
+        layers = list(range(self.w.L_r)) if layers is None else list(layers)
+        rows = np.arange(self.tok.T_r) if rows is None else np.asarray(rows, dtype=np.int64)
+        worst = {"rel_fro": 0.0, "max_abs": 0.0}
+        assert self.job.device_status() == 0
+        for l in layers:
+            ref = self.oracle([l], rows)
+            for (ll, c), y in ref.items():
+                g = self.gpu_rows(ll, c, rows)
+                diff = g - y
+                rel = float(np.linalg.norm(diff) / max(np.linalg.norm(y), 1e-30))
+                mx = float(np.abs(diff).max()) if diff.size else 0.0
+                worst["rel_fro"] = max(worst["rel_fro"], rel)
+                worst["max_abs"] = max(worst["max_abs"], mx)
+                assert rel <= rel_tol, (ll, c, rel)
+                assert mx <= abs_tol, (ll, c, mx)
+        return worst
+
+
+def sampled_rows(tok, n, seed=0):
+    """Seeded rows plus the edges: each request's first and last rows."""
+    rng = np.random.default_rng(seed)
+    T = tok.T_r
+    rows = set(rng.choice(T, size=min(n, T), replace=False).tolist())
+    for q in range(len(tok.r_tok_ptr) - 1):
+        a, b = int(tok.r_tok_ptr[q]), int(tok.r_tok_ptr[q + 1])
+        if b > a:
+            rows.update({a, b - 1, min(a + 1, b - 1)})
+    return np.array(sorted(rows), dtype=np.int64)

@@ -1,0 +1,224 @@
+"""GPU parity: the CUDA path through the C ABI against the fp64 oracle on
+the same seeded inputs.  CSRs must match bit for bit; transferred K/V must
+match within relative Frobenius error 5e-3 and max abs error 2e-2 per
+receiver layer and role."""
+
+import numpy as np
+import pytest
+import torch
+
+from gpu_harness import Case, sampled_rows
+from oracle import heterofold_oracle as O
+from paper_2609_32259_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import __graft_entry__ as g
+
+    g.build()
+
+
+# ---------------------------------------------------------------- the five workloads
+def test_tiny_overlap_interp_f32_full():
+    c = Case(W.tiny()).run()
+    c.check_csr()
+    worst = c.check_parity()
+    assert worst["rel_fro"] < 5e-3
+
+
+def test_llama_to_qwen25_4k_full():
+    c = Case(W.llama_to_qwen25(4096)).run()
+    c.check_csr()
+    c.check_parity()
+
+
+def test_llama_to_ministral_32k_sampled():
+    c = Case(W.llama_to_ministral(32768)).run()
+    c.check_csr()
+    c.check_parity(layers=[0, c.w.L_r - 1])                       # two whole layers
+    c.check_parity(rows=sampled_rows(c.tok, 1024, seed=2))       # every layer, sampled rows
+
+
+def test_qwen25_to_llama_batched_paged():
+    w = W.qwen25_to_llama_batched()
+    c = Case(w, sentinel=1234.0).run()
+    c.check_csr()
+    c.check_parity(rows=sampled_rows(c.tok, 1536, seed=3))
+    c.check_parity(layers=[5], rows=np.arange(int(c.tok.r_tok_ptr[1])))  # a whole request
+    # blocks no request owns keep the sentinel
+    used = set(c.paged.block_table[c.paged.block_table >= 0].tolist())
+    spare = [b for b in range(c.paged.n_blocks) if b not in used]
+    assert spare
+    bs = w.block_size
+    rows = torch.as_tensor(np.concatenate([np.arange(b * bs, (b + 1) * bs) for b in spare]),
+                           device=c.dev)
+    untouched = c.job.receiver[:, :, rows]
+    assert bool((untouched == 1234.0).all())
+
+
+@pytest.mark.parametrize("T_r", [1024, 4096, 131072])
+def test_ministral_to_llama_sweep(T_r):
+    c = Case(W.ministral_to_llama(T_r)).run()
+    c.check_csr()
+    if T_r <= 1024:
+        c.check_parity()
+    else:
+        c.check_parity(layers=[c.w.L_r // 2])
+        c.check_parity(rows=sampled_rows(c.tok, 512, seed=T_r))
+
+
+# ---------------------------------------------------------------- alignment CSR
+@pytest.mark.parametrize("mode", ["ta", "overlap_mean", "same_index"])
+@pytest.mark.parametrize("make", [lambda: W.llama_to_qwen25(4096), W.qwen25_to_llama_batched,
+                                  lambda: W.ministral_to_llama(131072)],
+                         ids=["4k", "batched", "128k"])
+def test_align_csr_bitexact(mode, make):
+    w = make().with_(align_mode=mode, L_s=1, L_r=1, H_s=1, D_s=64, H_r=1, D_r=128)
+    c = Case(w)
+    c.job.align()
+    torch.cuda.synchronize()
+    c.check_csr()
+
+
+def _csr_case(s_ptr, r_ptr, s_end, r_end, mode):
+    from paper_2609_32259_gb300 import binding as B
+    dev = torch.device("cuda")
+    T_s, T_r = int(s_ptr[-1]), int(r_ptr[-1])
+    cap = T_r + T_s + 1
+    row_ptr = torch.full((T_r + 1,), -7, dtype=torch.int32, device=dev)
+    col = torch.zeros(cap, dtype=torch.int32, device=dev)
+    wt = torch.zeros(cap, dtype=torch.float32, device=dev)
+    info = torch.zeros(2, dtype=torch.int32, device=dev)
+    B.align_build(mode, s_ptr, r_ptr, torch.as_tensor(np.asarray(s_end, np.int32), device=dev),
+                  torch.as_tensor(np.asarray(r_end, np.int32), device=dev), row_ptr, col, wt,
+                  cap, info)
+    torch.cuda.synchronize()
+    nnz = int(info[0])
+    return (row_ptr.cpu().numpy(), col[:nnz].cpu().numpy(), wt[:nnz].cpu().numpy(),
+            int(info[1]))
+
+
+@pytest.mark.parametrize("mode", ["ta", "overlap_mean", "same_index"])
+def test_align_adversarial(mode):
+    cases = [
+        ([0, 4], [0, 6], [3, 16, 23, 24], [3, 9, 12, 16, 23, 24]),          # worked example
+        ([0, 6], [0, 4], [3, 9, 12, 16, 23, 24], [3, 16, 23, 24]),          # reverse
+        ([0, 4], [0, 3], [1, 2, 4, 6], [1, 3, 6]),                          # sender-only boundary
+        ([0, 1], [0, 1], [5], [5]),                                         # one token each
+        ([0, 1], [0, 5], [5], [1, 2, 3, 4, 5]),                              # one sender token
+        ([0, 5], [0, 1], [1, 2, 3, 4, 5], [5]),                              # one receiver token
+        ([0, 2, 2, 5, 6], [0, 3, 3, 4, 6], [2, 4, 1, 2, 3, 7], [1, 3, 4, 3, 2, 7]),  # empty request
+    ]
+    rng = np.random.default_rng(5)
+    for n_req in (1, 7, 64):
+        s_ptr, r_ptr, s_end, r_end = [0], [0], [], []
+        for _ in range(n_req):
+            n = int(rng.integers(1, 400))
+            def seg(lo, hi):
+                e, out = 0, []
+                while e < n:
+                    e = min(n, e + int(rng.integers(lo, hi + 1)))
+                    out.append(e)
+                return out
+            s, r = seg(1, 6), seg(1, 5)
+            s_end += s
+            r_end += r
+            s_ptr.append(s_ptr[-1] + len(s))
+            r_ptr.append(r_ptr[-1] + len(r))
+        cases.append((s_ptr, r_ptr, s_end, r_end))
+    for s_ptr, r_ptr, s_end, r_end in cases:
+        ref = O.alignment_csr(mode, s_ptr, r_ptr, s_end, r_end)
+        rp, col, wt, bits = _csr_case(s_ptr, r_ptr, s_end, r_end, mode)
+        assert bits == 0
+        assert np.array_equal(rp, ref.row_ptr)
+        assert np.array_equal(col, ref.col)
+        assert np.array_equal(wt.view(np.uint32), ref.w32.view(np.uint32))
+
+
+def test_align_flags_unsorted_offsets():
+    rp, col, wt, bits = _csr_case([0, 3], [0, 2], [3, 2, 5], [2, 5], "ta")
+    assert bits & 0x01
+    rp, col, wt, bits = _csr_case([0, 2], [0, 2], [2, 5], [2, 6], "overlap_mean")
+    assert bits & 0x01
+
+
+# ---------------------------------------------------------------- edge cases and modes
+EDGE = {
+    "one_token": lambda: W.llama_to_ministral(1).with_(L_s=3, L_r=5),
+    "ragged_129": lambda: W.llama_to_ministral(129).with_(L_s=4, L_r=3),
+    "ragged_300": lambda: W.llama_to_qwen25(300).with_(L_s=5, L_r=4),
+    "knorm_pos0": lambda: W.llama_to_ministral(700).with_(L_s=4, L_r=4, knorm=True,
+                                                           r_pos0=(100000,)),
+    "interp_ta_bf16": lambda: W.llama_to_ministral(600).with_(L_s=5, L_r=7, layer_mode="interp"),
+    "overlap_paper_bf16": lambda: W.llama_to_ministral(600).with_(L_s=5, L_r=4,
+                                                                  align_mode="overlap_mean"),
+    "ta_paper_f32": lambda: W.llama_to_ministral(400).with_(L_s=4, L_r=3, dtype="f32"),
+    "same_index": lambda: W.llama_to_ministral(500).with_(L_s=4, L_r=3, align_mode="same_index"),
+    "d128_one_head": lambda: W.llama_to_ministral(333).with_(L_s=3, L_r=2, H_r=1, D_r=128),
+    "head64": lambda: W.llama_to_ministral(333).with_(L_s=3, L_r=2, H_r=4, D_r=64),
+    "batched_small_paged": lambda: W.qwen25_to_llama_batched(n_req=5, lo=1, hi=300, seed=9)
+    .with_(L_s=3, L_r=3),
+}
+
+
+@pytest.mark.parametrize("name", sorted(EDGE))
+def test_edge_case(name):
+    c = Case(EDGE[name]()).run()
+    c.check_csr()
+    c.check_parity()
+
+
+def test_identity_map_bit_exact():
+    """Same depth and tokenisation, A = [0; I; 0], b = 0, r = 1: V is copied
+    bit for bit; K at position 0 (no rotation) too."""
+    from paper_2609_32259_gb300 import pipeline
+    w = W.llama_to_ministral(500).with_(L_s=4, L_r=4)
+    tok = W.tokens(w)
+    dev = torch.device("cuda")
+    T = tok.T_r
+    sender = W.sender_kv(w, T, dev)
+    d = w.d_r
+    Wm = torch.zeros((w.L_r, 2, d, 3 * d), dtype=torch.bfloat16, device=dev)
+    Wm[:, :, :, d:2 * d] = torch.eye(d, dtype=torch.bfloat16, device=dev)
+    b = torch.zeros((w.L_r, 2, d), dtype=torch.float32, device=dev)
+    r = np.ones((w.L_r, 2), np.float32)
+    job = pipeline.TransferJob(L_s=w.L_s, H_s=w.H_s, D_s=w.D_s, L_r=w.L_r, H_r=w.H_r,
+                               D_r=w.D_r, dtype="bf16", align_mode="ta", layer_mode="paper3",
+                               s_tok_ptr=tok.r_tok_ptr, r_tok_ptr=tok.r_tok_ptr,
+                               s_end=tok.r_end, r_end=tok.r_end, sender=sender, W=Wm, b=b,
+                               r=r, theta_r=w.theta_r, device=dev)
+    job.step()
+    torch.cuda.synchronize()
+    assert job.device_status() == 0
+    assert job.distinct_rows() == T
+    assert torch.equal(job.receiver[:, 1], sender[:, 1])
+    assert torch.equal(job.receiver[:, 0, 0], sender[:, 0, 0])
+
+
+def test_device_flags_bad_block_and_column():
+    w = W.qwen25_to_llama_batched(n_req=2, lo=40, hi=60, seed=4).with_(L_s=3, L_r=2)
+    c = Case(w, sentinel=7.0)
+    c.job.block_table[0, 0] = c.paged.n_blocks + 5  # outside the pool
+    c.job.step()
+    torch.cuda.synchronize()
+    assert c.job.device_status() & 0x08
+    used = set(c.paged.block_table[c.paged.block_table >= 0].tolist())
+    used.discard(int(c.paged.block_table[0, 0]))
+    bs = w.block_size
+    spare = [b for b in range(c.paged.n_blocks) if b not in used]
+    rows = torch.as_tensor(np.concatenate([np.arange(b * bs, (b + 1) * bs) for b in spare]),
+                           device=c.dev)
+    assert bool((c.job.receiver[:, :, rows] == 7.0).all())
+    # a corrupted CSR column is flagged and skipped
+    c2 = Case(W.llama_to_ministral(200).with_(L_s=3, L_r=2, align_mode="overlap_mean"))
+    c2.job.align()
+    c2.job.col[3] = 10 ** 6
+    c2.job.make_plan()
+    c2.job.transfer()
+    torch.cuda.synchronize()
+    assert c2.job.device_status() & 0x02
