@@ -49,9 +49,28 @@ def workload(name):
         "qwen25_to_llama_batched_paged": W.qwen25_to_llama_batched,
         "tiny": W.tiny,
     }
-    if name.startswith("ministral_to_llama_"):
-        return W.ministral_to_llama(int(name.rsplit("_", 1)[1]))
+    for prefix, make in (("ministral_to_llama_", W.ministral_to_llama),
+                         ("llama_to_ministral_", W.llama_to_ministral),
+                         ("llama_to_qwen25_", W.llama_to_qwen25)):
+        if name.startswith(prefix) and name[len(prefix):].isdigit():
+            return make(int(name[len(prefix):]))
     return table[name]()
+
+
+def aggregate(times_ms, T_r_per_rank, world):
+    """Max over ranks of each time (ms); whole-job throughput = all ranks'
+    receiver tokens / the slowest rank's step time."""
+    times = list(times_ms)
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        dev = torch.device("cuda", torch.cuda.current_device()) if (
+            dist.get_backend() == "nccl") else torch.device("cpu")
+        t = torch.tensor(times, dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        times = [float(x) for x in t.cpu()]
+    value = world * T_r_per_rank / (times[0] * 1e-3)
+    return value, times
 
 
 def peaks():
@@ -296,11 +315,7 @@ def run_ours(args):
     clk = clocks.stop()
     step_ms = t_start.elapsed_time(t_end) / args.steps
     kern_ms = statistics.mean(a.elapsed_time(bb) for a, bb in ev)
-    if world > 1:
-        t = torch.tensor([step_ms, kern_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        step_ms, kern_ms = float(t[0]), float(t[1])
-    value = world * tok.T_r / (step_ms * 1e-3)
+    value, (step_ms, kern_ms) = aggregate([step_ms, kern_ms], tok.T_r, world)
 
     # end to end through the API with host buffers
     e2e = None
@@ -325,14 +340,11 @@ def run_ours(args):
         e1.record(stream)
         torch.cuda.synchronize()
         e2e_ms = e0.elapsed_time(e1) / n_e2e
-        if world > 1:
-            t = torch.tensor([e2e_ms], device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            e2e_ms = float(t[0])
+        e2e_value, (e2e_ms,) = aggregate([e2e_ms], tok.T_r, world)
         h2d = (sender.numel() * sender.element_size() + h_s_end.numel() * 4 +
                h_r_end.numel() * 4)
         d2h = job.receiver.numel() * job.receiver.element_size()
-        e2e = {"value": world * tok.T_r / (e2e_ms * 1e-3), "unit": UNIT, "ms_per_step": e2e_ms,
+        e2e = {"value": e2e_value, "unit": UNIT, "ms_per_step": e2e_ms,
                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
         del h_sender, h_recv
 
