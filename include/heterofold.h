@@ -219,6 +219,28 @@ hf_status hf_plan_device_status(hf_plan plan, hf_stream_t stream, int32_t* flags
 /* Synchronises `stream` and returns the number of distinct alignment rows. */
 hf_status hf_plan_distinct_rows(hf_plan plan, hf_stream_t stream, int32_t* n_rows);
 
+/*
+ * hf_transfer_noalloc — hf_plan_create + hf_transfer + hf_plan_destroy in
+ * one call that allocates no memory: the plan metadata goes to a device
+ * array built into the library instead of a caller workspace.  The paper
+ * has no counterpart; this is a convenience for callers that cannot
+ * allocate device memory per call (a host framework or plugin that owns
+ * every device allocation, or a fixed memory budget).
+ *  - The built-in array holds 8 MiB per GPU (about 400K receiver tokens);
+ *    every GPU that loads the library keeps it until the process exits.
+ *    Larger transfers are rejected with HF_ERR_UNSUPPORTED and a message.
+ *  - The first call on a device looks the array's device address up
+ *    (cudaGetSymbolAddress) with that device current; make that first call
+ *    before any stream capture.
+ *  - Every call shares the array: calls that overlap on the GPU (different
+ *    streams, or another thread) race and give wrong results.  Calls on one
+ *    stream are ordered and safe.  The device status bits are not reported.
+ *  - desc, sender_kv and receiver_kv are as for hf_plan_create and
+ *    hf_transfer; the call is asynchronous on `stream`.
+ */
+hf_status hf_transfer_noalloc(const hf_plan_desc* desc, const void* sender_kv,
+                              void* receiver_kv, hf_stream_t stream);
+
 const char* hf_status_string(hf_status status);
 const char* hf_last_error(void);
 

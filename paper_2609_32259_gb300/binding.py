@@ -36,7 +36,7 @@ CHECK_BITS = {
 
 EXPORTED = ("hf_align_build", "hf_plan_workspace_size", "hf_plan_create", "hf_transfer",
             "hf_plan_destroy", "hf_plan_device_status", "hf_plan_distinct_rows",
-            "hf_status_string", "hf_last_error")
+            "hf_status_string", "hf_last_error", "hf_transfer_noalloc")
 
 _p = ctypes.c_void_p
 _i32p = ctypes.POINTER(ctypes.c_int32)
@@ -87,6 +87,8 @@ def lib() -> ctypes.CDLL:
         L.hf_plan_destroy.argtypes = [_p]
         L.hf_plan_device_status.argtypes = [_p, _p, _i32p]
         L.hf_plan_distinct_rows.argtypes = [_p, _p, _i32p]
+        L.hf_transfer_noalloc.argtypes = [ctypes.POINTER(PlanDesc), _p, _p, _p]
+        L.hf_transfer_noalloc.restype = ctypes.c_int
         L.hf_status_string.argtypes = [ctypes.c_int]
         L.hf_status_string.restype = ctypes.c_char_p
         L.hf_last_error.argtypes = []
@@ -201,6 +203,13 @@ def plan_create(desc: Desc, workspace, stream=None) -> Plan:
 def transfer(plan: Plan, sender_kv, receiver_kv, stream=None) -> None:
     _check(lib().hf_transfer(plan.handle, _dptr(sender_kv), _dptr(receiver_kv), _stream(stream)),
            "hf_transfer")
+
+
+def transfer_noalloc(desc: Desc, sender_kv, receiver_kv, stream=None) -> None:
+    """hf_transfer_noalloc: plan + transfer with the library's built-in
+    metadata array (no workspace, no allocation)."""
+    _check(lib().hf_transfer_noalloc(ctypes.byref(desc.c), _dptr(sender_kv), _dptr(receiver_kv),
+                                     _stream(stream)), "hf_transfer_noalloc")
 
 
 def plan_device_status(plan: Plan, stream=None) -> int:

@@ -77,6 +77,8 @@ hf_status cuda_fail(cudaError_t e, const char* what);
 int device_sm_count();
 
 hf_status launch_plan_kernels(hf_plan_s* p, const PlanTables& tables, cudaStream_t stream);
+hf_status plan_build(const hf_plan_desc* desc, void* d_workspace, size_t workspace_bytes,
+                     cudaStream_t stream, hf_plan_s* p, PlanTables* t);
 hf_status launch_transfer(hf_plan_s* p, const void* sender, void* receiver, cudaStream_t stream);
 
 }  // namespace hf

@@ -330,13 +330,12 @@ extern "C" hf_status hf_plan_workspace_size(const hf_plan_desc* desc, size_t* by
   return HF_OK;
 }
 
-extern "C" hf_status hf_plan_create(const hf_plan_desc* desc, void* d_workspace,
-                                    size_t workspace_bytes, hf_stream_t stream_, hf_plan* out) {
-  if (!out) {
-    set_error("hf_plan_create: null output handle");
-    return HF_ERR_INVALID_ARGUMENT;
-  }
-  *out = nullptr;
+namespace hf {
+
+// Validates `desc`, fills `p` and `t`, and launches the plan kernels into
+// the given workspace.  `p` and `t` belong to the caller.
+hf_status plan_build(const hf_plan_desc* desc, void* d_workspace, size_t workspace_bytes,
+                     cudaStream_t stream, hf_plan_s* p, PlanTables* t) {
   const hf_status v = validate(desc);
   if (v != HF_OK) return v;
   const WorkspaceLayout lay =
@@ -346,7 +345,6 @@ extern "C" hf_status hf_plan_create(const hf_plan_desc* desc, void* d_workspace,
     set_error("hf_plan_create: workspace missing, too small or not 256-byte aligned");
     return HF_ERR_WORKSPACE;
   }
-  hf_plan_s* p = new hf_plan_s();
   p->desc = *desc;
   p->d_s = desc->H_s * desc->D_s;
   p->d_r = desc->H_r * desc->D_r;
@@ -366,7 +364,6 @@ extern "C" hf_status hf_plan_create(const hf_plan_desc* desc, void* d_workspace,
   p->desc.r_pos0 = nullptr;
   p->desc.h_r = nullptr;
 
-  PlanTables* t = new PlanTables();
   std::memset(t, 0, sizeof(*t));
   t->L_r = desc->L_r;
   t->D_r = desc->D_r;
@@ -380,7 +377,22 @@ extern "C" hf_status hf_plan_create(const hf_plan_desc* desc, void* d_workspace,
                          : 0.0f;
   for (int q = 0; q <= desc->n_req; ++q) t->r_tok_ptr[q] = desc->r_tok_ptr[q];
   for (int q = 0; q < desc->n_req; ++q) t->r_pos0[q] = desc->r_pos0 ? desc->r_pos0[q] : 0;
-  const hf_status s = launch_plan_kernels(p, *t, reinterpret_cast<cudaStream_t>(stream_));
+  return launch_plan_kernels(p, *t, stream);
+}
+
+}  // namespace hf
+
+extern "C" hf_status hf_plan_create(const hf_plan_desc* desc, void* d_workspace,
+                                    size_t workspace_bytes, hf_stream_t stream_, hf_plan* out) {
+  if (!out) {
+    set_error("hf_plan_create: null output handle");
+    return HF_ERR_INVALID_ARGUMENT;
+  }
+  *out = nullptr;
+  hf_plan_s* p = new hf_plan_s();
+  PlanTables* t = new PlanTables();
+  const hf_status s = plan_build(desc, d_workspace, workspace_bytes,
+                                 reinterpret_cast<cudaStream_t>(stream_), p, t);
   delete t;
   if (s != HF_OK) {
     delete p;
