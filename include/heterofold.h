@@ -99,6 +99,7 @@ typedef enum {
 #define HF_CHECK_BAD_BLOCK     0x08 /* a block-table entry outside the pool */
 #define HF_CHECK_CAPACITY      0x10 /* the CSR did not fit the given capacity */
 #define HF_CHECK_TIMEOUT       0x20 /* a pipeline wait gave up (internal error) */
+#define HF_CHECK_INTERNAL      0x40 /* a launch invariant did not hold (internal error) */
 
 /*
  * hf_align_build — alignment CSR from character-end offsets (Section 3.1,
@@ -226,7 +227,7 @@ hf_status hf_plan_distinct_rows(hf_plan plan, hf_stream_t stream, int32_t* n_row
  * has no counterpart; this is a convenience for callers that cannot
  * allocate device memory per call (a host framework or plugin that owns
  * every device allocation, or a fixed memory budget).
- *  - The built-in array holds 8 MiB per GPU (about 400K receiver tokens);
+ *  - The built-in array holds 8 MiB per GPU (about 340K receiver tokens);
  *    every GPU that loads the library keeps it until the process exits.
  *    Larger transfers are rejected with HF_ERR_UNSUPPORTED and a message.
  *  - The first call on a device looks the array's device address up

@@ -32,6 +32,7 @@ DTYPES = {"bf16": 0, "f32": 1}
 CHECK_BITS = {
     0x01: "HF_CHECK_BAD_OFFSETS", 0x02: "HF_CHECK_BAD_COLUMN", 0x04: "HF_CHECK_BAD_ROW",
     0x08: "HF_CHECK_BAD_BLOCK", 0x10: "HF_CHECK_CAPACITY", 0x20: "HF_CHECK_TIMEOUT",
+    0x40: "HF_CHECK_INTERNAL",
 }
 
 EXPORTED = ("hf_align_build", "hf_plan_workspace_size", "hf_plan_create", "hf_transfer",

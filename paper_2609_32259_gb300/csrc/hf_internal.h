@@ -37,6 +37,7 @@ struct WorkspaceLayout {
   size_t r_pos0;     // int32[n_req]
   size_t run_ptr;    // int32[T_r + 1]: first receiver row of each distinct row
   size_t ucol;       // int32[T_r]: sender column of each distinct row (one-entry rows)
+  size_t upos;       // int32[T_r]: RoPE position of each distinct row's first receiver row
   size_t pos;        // int32[T_r]: RoPE position of each receiver row
   size_t dst_row;    // int32[T_r]: destination row of each receiver row
   size_t new_flag;   // int32[T_r]: 1 where a receiver row starts a new distinct row

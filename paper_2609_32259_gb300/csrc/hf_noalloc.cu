@@ -20,7 +20,7 @@
 namespace hf {
 namespace {
 
-constexpr size_t kNoAllocScratchBytes = 8u << 20;  // 8 MiB: ~400K receiver tokens
+constexpr size_t kNoAllocScratchBytes = 8u << 20;  // 8 MiB: ~340K receiver tokens
 constexpr int kMaxDevices = 64;
 
 __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
@@ -60,7 +60,7 @@ extern "C" hf_status hf_transfer_noalloc(const hf_plan_desc* desc, const void* s
     set_error("hf_transfer_noalloc: this transfer needs " + std::to_string(need) +
               " bytes of metadata but the built-in scratch holds " +
               std::to_string(kNoAllocScratchBytes) +
-              " bytes (about 400K receiver tokens); use hf_plan_create with a workspace");
+              " bytes (about 340K receiver tokens); use hf_plan_create with a workspace");
     return HF_ERR_UNSUPPORTED;
   }
   void* ws = nullptr;

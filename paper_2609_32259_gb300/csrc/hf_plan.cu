@@ -54,6 +54,7 @@ WorkspaceLayout workspace_layout(int L_r, int D_r, int n_req, int64_t T_r) {
   w.r_pos0 = take(sizeof(int32_t) * (size_t)n_req);
   w.run_ptr = take(sizeof(int32_t) * (size_t)(T_r + 1));
   w.ucol = take(sizeof(int32_t) * (size_t)(T_r > 0 ? T_r : 1));
+  w.upos = take(sizeof(int32_t) * (size_t)(T_r > 0 ? T_r : 1));
   w.pos = take(sizeof(int32_t) * (size_t)(T_r > 0 ? T_r : 1));
   w.dst_row = take(sizeof(int32_t) * (size_t)(T_r > 0 ? T_r : 1));
   w.new_flag = take(sizeof(int32_t) * (size_t)(T_r > 0 ? T_r : 1));
@@ -73,6 +74,7 @@ struct PlanDev {
   int32_t* r_pos0;
   int32_t* run_ptr;
   int32_t* ucol;
+  int32_t* upos;
   int32_t* pos;
   int32_t* dst_row;
   int32_t* new_flag;
@@ -90,6 +92,7 @@ PlanDev plan_dev(const hf_plan_s* p) {
   d.r_pos0 = reinterpret_cast<int32_t*>(at(p->lay.r_pos0));
   d.run_ptr = reinterpret_cast<int32_t*>(at(p->lay.run_ptr));
   d.ucol = reinterpret_cast<int32_t*>(at(p->lay.ucol));
+  d.upos = reinterpret_cast<int32_t*>(at(p->lay.upos));
   d.pos = reinterpret_cast<int32_t*>(at(p->lay.pos));
   d.dst_row = reinterpret_cast<int32_t*>(at(p->lay.dst_row));
   d.new_flag = reinterpret_cast<int32_t*>(at(p->lay.new_flag));
@@ -186,6 +189,7 @@ __global__ void plan_runs_kernel(RowArgs a) {
       int32_t k = a.col[a.row_ptr[j]];
       if (k < 0 || k >= a.T_s) k = 0;  // flagged by plan_rows_kernel
       d.ucol[u] = k;
+      d.upos[u] = d.pos[j];
     }
     if (j == a.T_r - 1) {
       d.run_ptr[incl] = static_cast<int32_t>(a.T_r);

@@ -9,28 +9,31 @@
 // Receiver tokens whose alignment rows are identical have identical y
 // before RoPE, so the contraction runs over the U distinct rows only; each
 // distinct row covers a run of consecutive receiver rows [run_ptr[u],
-// run_ptr[u+1]), and the epilogue writes y (rotated per position for K) to
-// every row of its run.
+// run_ptr[u+1]) at consecutive positions from upos[u], and the epilogue
+// writes y (rotated per position for K) to every row of its run.
 //
 // One persistent CTA per SM walks tiles (l, c, 128 distinct rows, BN
 // receiver columns) with warp-specialised roles:
-//   warp 0      TMA producer: map tile W[l][c][n0:n0+BN][k0:k0+BK] and, when
-//               every map input row is a single sender row (Token Alignment
-//               + the three-layer neighbourhood), the 128 sender rows of the
-//               A tile via tile::gather4, into 128-byte-swizzled smem stages;
+//   warp 0      TMA producer of the map tile W[l][c][n0:n0+BN][k0:k0+BK]
+//               (2-D tiled load, 128-byte swizzle);
 //   warp 1      TMEM allocator and the single thread issuing tcgen05.mma
 //               (M = 128, N = BN, K = 16 bf16 / 8 tf32 per instruction) into
 //               one of two TMEM accumulators;
 //   warps 2-9   epilogue, two groups of four warps (one per TMEM lane
 //               quarter), each group owning half of the tile's columns;
-//   warps 10-13 (pooled / blended inputs only) build the A tile in fp32
-//               registers from weighted CSR entries and sender layers.
+//   warps 10-13 A tile builders.  When every map input row is one sender row
+//               (Token Alignment with the three-layer neighbourhood) they copy
+//               the 128 sender rows with cp.async, eight lanes per 128-byte
+//               row; for pooled or blended rows they sum weighted sender rows
+//               in fp32 registers and round once.  Both write the 128-byte
+//               swizzled layout and fence it to the async proxy before
+//               arriving on the stage barrier.
 // Pipeline hand-offs use mbarriers with bounded waits; nothing traps.
 #include <algorithm>
 #include <climits>
 #include <cstring>
-#include <string>
 #include <mutex>
+#include <string>
 
 #include "hf_device.cuh"
 #include "hf_internal.h"
@@ -39,10 +42,12 @@ namespace hf {
 namespace {
 
 constexpr int kBM = 128;                 // distinct rows per tile (UMMA M)
+constexpr int kThreads = 448;            // 14 warps
 constexpr int kStageABytes = kBM * 128;  // 128 rows x 128 bytes
 constexpr int kStgFloats = kBM * 32;     // epilogue staging per group
-constexpr int kRunStride = 136;          // run pointers per group (129 used)
+constexpr int kRunStride = 132;          // run starts / positions per group (129 used)
 constexpr int kMaxStages = 8;
+constexpr int kLag = 3;                  // cp.async groups in flight per loader thread
 constexpr int kTmemCols = 512;           // two accumulators of up to 256 columns
 
 struct XferParams {
@@ -58,7 +63,7 @@ struct XferParams {
   const float* w;
   const int32_t* run_ptr;
   const int32_t* ucol;
-  const int32_t* pos;
+  const int32_t* upos;
   const int32_t* dst_row;
   const int32_t* n_distinct;
   int32_t* status;
@@ -134,22 +139,86 @@ __device__ __forceinline__ uint4 pack16(const float* a, const float*) {
                     __float_as_uint(a[3]));
 }
 
+// One chain of the epilogue's position walk: a lane's two rotation pairs at
+// receiver row j (row u of the tile), with RoPE state carried from the
+// chain's previous position four rows back.
+struct Chain {
+  int u;          // tile row holding the current position
+  int expect;     // position this chain expects next (angle-addition valid)
+  float cs0, sn0, cs1, sn1;
+};
+
+template <typename T>
+__device__ __forceinline__ void walk_step(Chain& ch, int j, int it, const int32_t* srun,
+                                          const int32_t* supos, const float* stg, int pl, int p0,
+                                          bool do_rope, float f0, float f1, float C0, float S0,
+                                          float C1, float S1, const XferParams& P, T* out_lc,
+                                          int ocol, int q, int half) {
+  const int drow = P.paged ? __ldg(P.dst_row + j) : j;
+  while (srun[ch.u + 1] <= j) ++ch.u;
+  const int u = ch.u;
+  const float* urow = stg + u * 32;
+  const int sw = u & 7;
+  const float2 lo = *reinterpret_cast<const float2*>(urow + (((pl >> 1) ^ sw) << 2) + (p0 & 3));
+  const float2 hi =
+      *reinterpret_cast<const float2*>(urow + (((4 + (pl >> 1)) ^ sw) << 2) + (p0 & 3));
+  float a0 = lo.x, a1 = lo.y, b0 = hi.x, b1 = hi.y;
+  if (do_rope) {
+    const int p = supos[u] + (j - srun[u]);
+    if (p != ch.expect || (it & 15) == 0) {
+      rope_sincos(p, f0, &ch.sn0, &ch.cs0);
+      rope_sincos(p, f1, &ch.sn1, &ch.cs1);
+    } else {  // advance the angle by four positions
+      const float t0 = ch.cs0 * C0 - ch.sn0 * S0;
+      ch.sn0 = ch.sn0 * C0 + ch.cs0 * S0;
+      ch.cs0 = t0;
+      const float t1 = ch.cs1 * C1 - ch.sn1 * S1;
+      ch.sn1 = ch.sn1 * C1 + ch.cs1 * S1;
+      ch.cs1 = t1;
+    }
+    ch.expect = p + 4;
+    const float oa0 = a0 * ch.cs0 - b0 * ch.sn0, ob0 = b0 * ch.cs0 + a0 * ch.sn0;
+    const float oa1 = a1 * ch.cs1 - b1 * ch.sn1, ob1 = b1 * ch.cs1 + a1 * ch.sn1;
+    a0 = oa0;
+    b0 = ob0;
+    a1 = oa1;
+    b1 = ob1;
+  }
+  if (drow >= 0) {
+    T* o = out_lc + static_cast<int64_t>(drow) * P.d_r + ocol;
+    store_pair(o + q + p0, a0, a1);
+    store_pair(o + half + q + p0, b0, b1);
+  }
+}
+
+// Last u in [0, nrows) with srun[u] <= j.
+__device__ __forceinline__ int find_row(const int32_t* srun, int nrows, int j) {
+  int lo = 0, hi = nrows - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (srun[mid] <= j) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
+
 template <typename T, bool kGather>
-__global__ void __launch_bounds__(kGather ? 320 : 448, 1)
-    transfer_kernel(const __grid_constant__ CUtensorMap tmap_s,
-                    const __grid_constant__ CUtensorMap tmap_w, const XferParams P) {
+__global__ void __launch_bounds__(kThreads, 1)
+    transfer_kernel(const __grid_constant__ CUtensorMap tmap_w, const XferParams P) {
   constexpr int kBK = Elem<T>::kBK;
   constexpr int kPerChunk = 16 / sizeof(T);  // elements per 16-byte chunk
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>(
-      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  extern __shared__ __align__(1024) uint8_t smem[];
+  if (smem_addr(smem) & 1023u) {  // the swizzled stages need 1024-byte alignment
+    if (threadIdx.x == 0) atomicOr(P.status, HF_CHECK_INTERNAL);
+    return;
+  }
   const int stages = P.stages;
   const int stage_b_bytes = P.BN * 128;
   uint8_t* sA = smem;
   uint8_t* sB = sA + stages * kStageABytes;
   float* sStg = reinterpret_cast<float*>(sB + stages * stage_b_bytes);
   int32_t* sRun = reinterpret_cast<int32_t*>(sStg + 2 * kStgFloats);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sRun + 2 * kRunStride);
+  int32_t* sUpos = sRun + 2 * kRunStride;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sUpos + 2 * kRunStride);
   uint64_t* full = bars;
   uint64_t* empty = bars + kMaxStages;
   uint64_t* tfull = bars + 2 * kMaxStages;
@@ -162,7 +231,7 @@ __global__ void __launch_bounds__(kGather ? 320 : 448, 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < stages; ++s) {
-      mbar_init(smem_addr(&full[s]), kGather ? 1 : 1 + kBM);
+      mbar_init(smem_addr(&full[s]), 1 + kBM);  // TMA expect_tx + 128 A builders
       mbar_init(smem_addr(&empty[s]), 1);
     }
     for (int a = 0; a < 2; ++a) {
@@ -173,10 +242,7 @@ __global__ void __launch_bounds__(kGather ? 320 : 448, 1)
     *sAbort = 0;
     fence_barrier_init();
   }
-  if (warp == 0 && lane == 0) {
-    tma_prefetch_map(&tmap_w);
-    if (kGather) tma_prefetch_map(&tmap_s);
-  }
+  if (warp == 0 && lane == 0) tma_prefetch_map(&tmap_w);
   if (warp == 1) {
     tmem_alloc(smem_addr(sTmem), kTmemCols);
     tmem_relinquish();
@@ -191,52 +257,32 @@ __global__ void __launch_bounds__(kGather ? 320 : 448, 1)
   const int total_tiles = 2 * P.L_r * tiles_per_lc;
 
   if (warp == 0) {
-    // ------------------------------------------------------------ producer
-    int stage = 0;
-    uint32_t phase = 0;
-    const uint32_t tx_bytes = stage_b_bytes + (kGather ? kStageABytes : 0);
-    bool ok = true;
-    for (int tile = blockIdx.x; tile < total_tiles && ok; tile += gridDim.x) {
-      int lc, m, n;
-      decode_tile(tile, tiles_per_lc, P.n_tiles_n, &lc, &m, &n);
-      const int l = lc >> 1, c = lc & 1;
-      const LayerSegs* segs = P.segs + l;
-      int r0 = 0, r1 = 0, r2 = 0, r3 = 0;
-      if (kGather) {
-        const int ub = m * kBM + lane * 4;
-        r0 = P.ucol[min(ub + 0, U - 1)];
-        r1 = P.ucol[min(ub + 1, U - 1)];
-        r2 = P.ucol[min(ub + 2, U - 1)];
-        r3 = P.ucol[min(ub + 3, U - 1)];
-      }
-      for (int kb = 0; kb < P.n_kb; ++kb) {
-        const int seg = kb / P.kb_per_seg;
-        const int kin = kb - seg * P.kb_per_seg;
-        if (!mbar_wait(smem_addr(&empty[stage]), phase ^ 1)) {
-          raise_timeout(P, sAbort);
-          ok = false;
-          break;
-        }
-        const uint32_t fb = smem_addr(&full[stage]);
-        if (lane == 0) {
-          mbar_arrive_expect_tx(fb, tx_bytes);
+    // ------------------------------------------------------------ map tiles
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < total_tiles && ok; tile += gridDim.x) {
+        int lc, m, n;
+        decode_tile(tile, tiles_per_lc, P.n_tiles_n, &lc, &m, &n);
+        for (int kb = 0; kb < P.n_kb; ++kb) {
+          if (!mbar_wait(smem_addr(&empty[stage]), phase ^ 1)) {
+            raise_timeout(P, sAbort);
+            ok = false;
+            break;
+          }
+          const uint32_t fb = smem_addr(&full[stage]);
+          mbar_arrive_expect_tx(fb, stage_b_bytes);
           tma_load_2d(smem_addr(sB + stage * stage_b_bytes), &tmap_w, kb * kBK,
                       lc * P.d_r + n * P.BN, fb);
-        }
-        if (kGather) {
-          __syncwarp();
-          const int t = segs->layer[seg][0];
-          const int rb = (t * 2 + c) * static_cast<int>(P.T_s);
-          tma_gather4(smem_addr(sA + stage * kStageABytes + lane * 512), &tmap_s, kin * kBK,
-                      rb + r0, rb + r1, rb + r2, rb + r3, fb);
-        }
-        if (++stage == stages) {
-          stage = 0;
-          phase ^= 1;
+          if (++stage == stages) {
+            stage = 0;
+            phase ^= 1;
+          }
         }
       }
-      __syncwarp();
     }
+    __syncwarp();
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issue
     if (lane == 0) {
@@ -293,6 +339,7 @@ __global__ void __launch_bounds__(kGather ? 320 : 448, 1)
     const int row = sp * 32 + lane;
     float* stg = sStg + g * kStgFloats;
     int32_t* srun = sRun + g * kRunStride;
+    int32_t* supos = sUpos + g * kRunStride;
     const bool active = P.groups == 2 || g == 0;
     const int gcols = P.groups == 2 ? P.BN / 2 : P.BN;
     const int gcol0 = P.groups == 2 ? g * (P.BN / 2) : 0;
@@ -312,23 +359,21 @@ __global__ void __launch_bounds__(kGather ? 320 : 448, 1)
       if (active) {
         const int u0 = m * kBM;
         const int nrows = min(kBM, U - u0);
-        for (int i = row; i <= nrows; i += kBM) srun[i] = P.run_ptr[u0 + i];
+        for (int i = row; i <= nrows; i += kBM) {
+          srun[i] = P.run_ptr[u0 + i];
+          supos[i] = i < nrows ? P.upos[u0 + i] : 0;
+        }
         named_barrier_sync(1 + g, 128);
+        // this warp's receiver rows [wjb, wje), walked as two chains
         const int jb = srun[0], je = srun[nrows];
         const int per = (je - jb + 3) >> 2;
         const int wjb = min(je, jb + sp * per), wje = min(je, wjb + per);
-        const int n_it = (wje - wjb + 3) >> 2;
-        const int jstart = wjb + pg;
-        // distinct row holding position jstart: last u with srun[u] <= jstart
-        int ustart = 0;
-        if (jstart < wje) {
-          int lo = 0, hi = nrows - 1;
-          while (lo < hi) {
-            const int mid = (lo + hi + 1) >> 1;
-            if (srun[mid] <= jstart) lo = mid; else hi = mid - 1;
-          }
-          ustart = lo;
-        }
+        const int hlen = (((wje - wjb + 1) >> 1) + 3) & ~3;  // chain A length, multiple of 4
+        const int amid = min(wje, wjb + hlen);
+        const int n_it = (hlen + 3) >> 2;
+        const int ja0 = wjb + pg, jb0 = amid + pg;
+        const int ua0 = ja0 < amid ? find_row(srun, nrows, ja0) : 0;
+        const int ub0 = jb0 < wje ? find_row(srun, nrows, jb0) : 0;
         const float inv_r = P.inv_r[lc];
         const float* bias = P.bias + static_cast<int64_t>(lc) * P.d_r;
         const bool do_rope = P.rope && c == 0;
@@ -338,8 +383,8 @@ __global__ void __launch_bounds__(kGather ? 320 : 448, 1)
         T* const out_lc = reinterpret_cast<T*>(P.receiver) +
                           (static_cast<int64_t>(lc) * P.recv_rows) * P.d_r;
         for (int h0 = 0; h0 < gcols; h0 += D) {
-          const int tcol = gcol0 + h0;           // accumulator column of the head
-          const int ocol = n * P.BN + tcol;      // receiver feature index of the head
+          const int tcol = gcol0 + h0;       // accumulator column of the head
+          const int ocol = n * P.BN + tcol;  // receiver feature index of the head
           float rn = 1.0f;
           if (do_knorm) {
             float ss = 0.0f;
@@ -358,11 +403,19 @@ __global__ void __launch_bounds__(kGather ? 320 : 448, 1)
             // step 1: 16 rotation pairs (columns q.., half+q..) of every row -> smem
             uint32_t v[32];
             tmem_load_2x16(ta + tcol + q, ta + tcol + half + q, v);
+            float bl[16], bh[16];
+#pragma unroll
+            for (int i = 0; i < 16; i += 4) {
+              const float4 x = __ldg(reinterpret_cast<const float4*>(bias + ocol + q + i));
+              const float4 z = __ldg(reinterpret_cast<const float4*>(bias + ocol + half + q + i));
+              bl[i] = x.x; bl[i + 1] = x.y; bl[i + 2] = x.z; bl[i + 3] = x.w;
+              bh[i] = z.x; bh[i + 1] = z.y; bh[i + 2] = z.z; bh[i + 3] = z.w;
+            }
             float y[32];
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
-              y[i] = fmaf(__uint_as_float(v[i]), inv_r, __ldg(bias + ocol + q + i));
-              y[16 + i] = fmaf(__uint_as_float(v[16 + i]), inv_r, __ldg(bias + ocol + half + q + i));
+              y[i] = fmaf(__uint_as_float(v[i]), inv_r, bl[i]);
+              y[16 + i] = fmaf(__uint_as_float(v[16 + i]), inv_r, bh[i]);
             }
             if (do_knorm) {
 #pragma unroll
@@ -373,61 +426,29 @@ __global__ void __launch_bounds__(kGather ? 320 : 448, 1)
             }
             float* srow = stg + row * 32;
 #pragma unroll
-            for (int ch = 0; ch < 8; ++ch)
-              *reinterpret_cast<float4*>(srow + ((ch ^ (row & 7)) << 2)) =
-                  make_float4(y[4 * ch], y[4 * ch + 1], y[4 * ch + 2], y[4 * ch + 3]);
+            for (int k = 0; k < 8; ++k)
+              *reinterpret_cast<float4*>(srow + ((k ^ (row & 7)) << 2)) =
+                  make_float4(y[4 * k], y[4 * k + 1], y[4 * k + 2], y[4 * k + 3]);
             named_barrier_sync(1 + g, 128);
-            // step 2: this warp's receiver positions, 4 per iteration, lanes
-            // 8*pg .. 8*pg+7 own position wjb + pg + 4*it, two pairs each
+            // step 2: lanes 8*pg .. 8*pg+7 own rows j = chain start + pg + 4*it
+            // (two pairs each); a step advances the RoPE angle by four rows.
             float f0 = 0.f, f1 = 0.f, C0 = 1.f, S0 = 0.f, C1 = 1.f, S1 = 0.f;
             if (do_rope) {
               f0 = __ldg(P.inv_freq + q + p0);
               f1 = __ldg(P.inv_freq + q + p0 + 1);
-              rope_sincos(4, f0, &S0, &C0);  // one step = four positions
+              rope_sincos(4, f0, &S0, &C0);
               rope_sincos(4, f1, &S1, &C1);
             }
-            int ucur = ustart;
-            int expect = INT_MIN;
-            float cs0 = 1.f, sn0 = 0.f, cs1 = 1.f, sn1 = 0.f;
+            Chain ca{ua0, INT_MIN, 1.f, 0.f, 1.f, 0.f};
+            Chain cb{ub0, INT_MIN, 1.f, 0.f, 1.f, 0.f};
             for (int it = 0; it < n_it; ++it) {
-              const int j = jstart + 4 * it;
-              if (j < wje) {
-                while (srun[ucur + 1] <= j) ++ucur;
-                const float* urow = stg + ucur * 32;
-                const int sw = ucur & 7;
-                const float2 lo =
-                    *reinterpret_cast<const float2*>(urow + (((pl >> 1) ^ sw) << 2) + (p0 & 3));
-                const float2 hi = *reinterpret_cast<const float2*>(
-                    urow + (((4 + (pl >> 1)) ^ sw) << 2) + (p0 & 3));
-                float a0 = lo.x, a1 = lo.y, b0 = hi.x, b1 = hi.y;
-                if (do_rope) {
-                  const int p = P.pos[j];
-                  if (p != expect || (it & 15) == 0) {
-                    rope_sincos(p, f0, &sn0, &cs0);
-                    rope_sincos(p, f1, &sn1, &cs1);
-                  } else {
-                    const float t0 = cs0 * C0 - sn0 * S0;
-                    sn0 = sn0 * C0 + cs0 * S0;
-                    cs0 = t0;
-                    const float t1 = cs1 * C1 - sn1 * S1;
-                    sn1 = sn1 * C1 + cs1 * S1;
-                    cs1 = t1;
-                  }
-                  expect = p + 4;
-                  const float oa0 = a0 * cs0 - b0 * sn0, ob0 = b0 * cs0 + a0 * sn0;
-                  const float oa1 = a1 * cs1 - b1 * sn1, ob1 = b1 * cs1 + a1 * sn1;
-                  a0 = oa0;
-                  b0 = ob0;
-                  a1 = oa1;
-                  b1 = ob1;
-                }
-                const int drow = P.paged ? P.dst_row[j] : j;
-                if (drow >= 0) {
-                  T* o = out_lc + static_cast<int64_t>(drow) * P.d_r + ocol;
-                  store_pair(o + q + p0, a0, a1);
-                  store_pair(o + half + q + p0, b0, b1);
-                }
-              }
+              const int ja = ja0 + 4 * it, jbb = jb0 + 4 * it;
+              if (ja < amid)
+                walk_step<T>(ca, ja, it, srun, supos, stg, pl, p0, do_rope, f0, f1, C0, S0, C1,
+                             S1, P, out_lc, ocol, q, half);
+              if (jbb < wje)
+                walk_step<T>(cb, jbb, it, srun, supos, stg, pl, p0, do_rope, f0, f1, C0, S0, C1,
+                             S1, P, out_lc, ocol, q, half);
             }
             named_barrier_sync(1 + g, 128);
           }
@@ -439,59 +460,113 @@ __global__ void __launch_bounds__(kGather ? 320 : 448, 1)
       acc ^= 1;
       if (acc == 0) acc_phase ^= 1;
     }
-  } else if (!kGather) {
-    // ------------------------------------------------------------ A builder
-    // (pooled CSR rows and/or blended sender layers): thread r owns tile row r.
-    const int r = threadIdx.x - 320;
+  } else {
+    // ------------------------------------------------------------ A builders
+    const int t = threadIdx.x - 320;  // 0..127
     const T* sender = reinterpret_cast<const T*>(P.sender);
     int stage = 0;
     uint32_t phase = 0;
     bool ok = true;
-    for (int tile = blockIdx.x; tile < total_tiles && ok; tile += gridDim.x) {
-      int lc, m, n;
-      decode_tile(tile, tiles_per_lc, P.n_tiles_n, &lc, &m, &n);
-      const int l = lc >> 1, c = lc & 1;
-      const LayerSegs segs = P.segs[l];
-      const int u = min(m * kBM + r, U - 1);
-      const int j0 = P.run_ptr[u];
-      const int e0 = P.row_ptr[j0], e1 = P.row_ptr[j0 + 1];
-      for (int kb = 0; kb < P.n_kb; ++kb) {
-        const int seg = kb / P.kb_per_seg;
-        const int kin = kb - seg * P.kb_per_seg;
-        if (!mbar_wait(smem_addr(&empty[stage]), phase ^ 1)) {
-          raise_timeout(P, sAbort);
-          ok = false;
-          break;
+    if (kGather) {
+      // eight lanes per 128-byte row: lane -> (row 32*slab + 4*i + lane/8, chunk lane%8)
+      const int slab = t >> 5, rsub = lane >> 3, ch = lane & 7;
+      int pending = 0;  // committed groups whose stage arrival is still owed
+      for (int tile = blockIdx.x; tile < total_tiles && ok; tile += gridDim.x) {
+        int lc, m, n;
+        decode_tile(tile, tiles_per_lc, P.n_tiles_n, &lc, &m, &n);
+        const int l = lc >> 1, c = lc & 1;
+        const LayerSegs* segs = P.segs + l;
+        int64_t roff[8];
+        uint32_t doff[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const int r = slab * 32 + 4 * i + rsub;
+          const int u = min(m * kBM + r, U - 1);
+          roff[i] = static_cast<int64_t>(P.ucol[u]) * P.d_s + ch * kPerChunk;
+          doff[i] = static_cast<uint32_t>(r * 128 + ((ch ^ (r & 7)) << 4));
         }
-        float acc[kBK];
+        for (int kb = 0; kb < P.n_kb; ++kb) {
+          const int seg = kb / P.kb_per_seg;
+          const int kin = kb - seg * P.kb_per_seg;
+          if (!mbar_wait(smem_addr(&empty[stage]), phase ^ 1)) {
+            raise_timeout(P, sAbort);
+            ok = false;
+            break;
+          }
+          const int tl = segs->layer[seg][0];
+          const T* base = sender + (static_cast<int64_t>(tl * 2 + c) * P.T_s) * P.d_s + kin * kBK;
+          const uint32_t sa = smem_addr(sA + stage * kStageABytes);
 #pragma unroll
-        for (int i = 0; i < kBK; ++i) acc[i] = 0.f;
-        for (int ti = 0; ti < segs.n_terms[seg]; ++ti) {
-          const int t = segs.layer[seg][ti];
-          const float om = segs.w[seg][ti];
-          const T* base = sender + (static_cast<int64_t>(t * 2 + c) * P.T_s) * P.d_s + kin * kBK;
-          for (int e = e0; e < e1; ++e) {
-            const int k = P.col[e];
-            if (k < 0 || k >= P.T_s) continue;  // flagged at plan creation
-            const float wt = om * P.w[e];
-            const uint4* src = reinterpret_cast<const uint4*>(base + static_cast<int64_t>(k) * P.d_s);
-            uint4 x[8];
-#pragma unroll
-            for (int ch = 0; ch < 8; ++ch) x[ch] = __ldg(src + ch);
-#pragma unroll
-            for (int ch = 0; ch < 8; ++ch) accum16(x[ch], wt, acc + ch * kPerChunk, (const T*)nullptr);
+          for (int i = 0; i < 8; ++i) cp_async_16(sa + doff[i], base + roff[i]);
+          cp_async_commit();
+          if (pending == kLag) {
+            // the group kLag k-blocks back has landed: publish its stage
+            cp_async_wait<kLag>();
+            fence_proxy_async_smem();
+            const int s_old = (stage + stages - kLag) % stages;
+            mbar_arrive(smem_addr(&full[s_old]));
+          } else {
+            ++pending;
+          }
+          if (++stage == stages) {
+            stage = 0;
+            phase ^= 1;
           }
         }
-        uint8_t* dst = sA + stage * kStageABytes + r * 128;
+      }
+      cp_async_wait<0>();
+      fence_proxy_async_smem();
+      for (int k = pending; k >= 1; --k) mbar_arrive(smem_addr(&full[(stage + stages - k) % stages]));
+    } else {
+      // pooled CSR rows and/or blended sender layers: thread t owns tile row t
+      for (int tile = blockIdx.x; tile < total_tiles && ok; tile += gridDim.x) {
+        int lc, m, n;
+        decode_tile(tile, tiles_per_lc, P.n_tiles_n, &lc, &m, &n);
+        const int l = lc >> 1, c = lc & 1;
+        const LayerSegs segs = P.segs[l];
+        const int u = min(m * kBM + t, U - 1);
+        const int j0 = P.run_ptr[u];
+        const int e0 = P.row_ptr[j0], e1 = P.row_ptr[j0 + 1];
+        for (int kb = 0; kb < P.n_kb; ++kb) {
+          const int seg = kb / P.kb_per_seg;
+          const int kin = kb - seg * P.kb_per_seg;
+          if (!mbar_wait(smem_addr(&empty[stage]), phase ^ 1)) {
+            raise_timeout(P, sAbort);
+            ok = false;
+            break;
+          }
+          float acc[kBK];
 #pragma unroll
-        for (int ch = 0; ch < 8; ++ch)
-          *reinterpret_cast<uint4*>(dst + ((ch ^ (r & 7)) << 4)) =
-              pack16(acc + ch * kPerChunk, (const T*)nullptr);
-        fence_proxy_async_smem();
-        mbar_arrive(smem_addr(&full[stage]));
-        if (++stage == stages) {
-          stage = 0;
-          phase ^= 1;
+          for (int i = 0; i < kBK; ++i) acc[i] = 0.f;
+          for (int ti = 0; ti < segs.n_terms[seg]; ++ti) {
+            const int tl = segs.layer[seg][ti];
+            const float om = segs.w[seg][ti];
+            const T* base = sender + (static_cast<int64_t>(tl * 2 + c) * P.T_s) * P.d_s + kin * kBK;
+            for (int e = e0; e < e1; ++e) {
+              const int k = P.col[e];
+              if (k < 0 || k >= P.T_s) continue;  // flagged at plan creation
+              const float wt = om * P.w[e];
+              const uint4* src =
+                  reinterpret_cast<const uint4*>(base + static_cast<int64_t>(k) * P.d_s);
+              uint4 x[8];
+#pragma unroll
+              for (int k2 = 0; k2 < 8; ++k2) x[k2] = __ldg(src + k2);
+#pragma unroll
+              for (int k2 = 0; k2 < 8; ++k2)
+                accum16(x[k2], wt, acc + k2 * kPerChunk, (const T*)nullptr);
+            }
+          }
+          uint8_t* dst = sA + stage * kStageABytes + t * 128;
+#pragma unroll
+          for (int k2 = 0; k2 < 8; ++k2)
+            *reinterpret_cast<uint4*>(dst + ((k2 ^ (t & 7)) << 4)) =
+                pack16(acc + k2 * kPerChunk, (const T*)nullptr);
+          fence_proxy_async_smem();
+          mbar_arrive(smem_addr(&full[stage]));
+          if (++stage == stages) {
+            stage = 0;
+            phase ^= 1;
+          }
         }
       }
     }
@@ -556,9 +631,9 @@ hf_status make_map(CUtensorMap* map, const void* base, bool f32, uint64_t rows, 
 }
 
 size_t smem_bytes(int BN, int stages) {
-  return 1024 + static_cast<size_t>(stages) * (kStageABytes + BN * 128) +
-         2 * kStgFloats * sizeof(float) + 2 * kRunStride * sizeof(int32_t) +
-         (2 * kMaxStages + 5) * sizeof(uint64_t) + 16;
+  return static_cast<size_t>(stages) * (kStageABytes + BN * 128) +
+         2 * kStgFloats * sizeof(float) + 4 * kRunStride * sizeof(int32_t) +
+         (2 * kMaxStages + 5) * sizeof(uint64_t) + 8;
 }
 
 int pick_stages(int BN) {
@@ -566,18 +641,18 @@ int pick_stages(int BN) {
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
   int s = 6;
-  while (s > 2 && smem_bytes(BN, s) > static_cast<size_t>(optin)) --s;
+  while (s > kLag + 1 && smem_bytes(BN, s) > static_cast<size_t>(optin)) --s;
   return s;
 }
 
 template <typename T, bool kGather>
-hf_status launch_typed(const CUtensorMap& ms, const CUtensorMap& mw, const XferParams& P, int grid,
-                       size_t smem, cudaStream_t stream) {
+hf_status launch_typed(const CUtensorMap& mw, const XferParams& P, int grid, size_t smem,
+                       cudaStream_t stream) {
   auto kern = transfer_kernel<T, kGather>;
   HF_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                    static_cast<int>(smem)),
               "set shared memory size");
-  kern<<<grid, kGather ? 320 : 448, smem, stream>>>(ms, mw, P);
+  kern<<<grid, kThreads, smem, stream>>>(mw, P);
   HF_CUDA_TRY(cudaGetLastError(), "transfer kernel launch");
   return HF_OK;
 }
@@ -590,18 +665,11 @@ hf_status launch_transfer(hf_plan_s* p, const void* sender, void* receiver, cuda
   const bool f32 = d.dtype == HF_F32;
   const int esize = f32 ? 4 : 2;
   const int bk = 128 / esize;
-  CUtensorMap ms, mw;
-  std::memset(&ms, 0, sizeof(ms));
+  CUtensorMap mw;
   hf_status s = make_map(&mw, d.d_W, f32, static_cast<uint64_t>(d.L_r) * 2 * p->d_r,
                          static_cast<uint64_t>(p->K), static_cast<uint32_t>(p->BN),
                          static_cast<uint32_t>(bk), CU_TENSOR_MAP_L2_PROMOTION_L2_256B);
   if (s != HF_OK) return s;
-  if (p->gather) {
-    s = make_map(&ms, sender, f32, static_cast<uint64_t>(d.L_s) * 2 * p->T_s,
-                 static_cast<uint64_t>(p->d_s), 1, static_cast<uint32_t>(bk),
-                 CU_TENSOR_MAP_L2_PROMOTION_L2_128B);
-    if (s != HF_OK) return s;
-  }
   XferParams P;
   std::memset(&P, 0, sizeof(P));
   char* ws = p->ws;
@@ -617,7 +685,7 @@ hf_status launch_transfer(hf_plan_s* p, const void* sender, void* receiver, cuda
   P.w = d.d_w;
   P.run_ptr = reinterpret_cast<const int32_t*>(ws + p->lay.run_ptr);
   P.ucol = reinterpret_cast<const int32_t*>(ws + p->lay.ucol);
-  P.pos = reinterpret_cast<const int32_t*>(ws + p->lay.pos);
+  P.upos = reinterpret_cast<const int32_t*>(ws + p->lay.upos);
   P.dst_row = reinterpret_cast<const int32_t*>(ws + p->lay.dst_row);
   P.n_distinct = reinterpret_cast<const int32_t*>(ws + p->lay.n_distinct);
   P.status = reinterpret_cast<int32_t*>(ws + p->lay.status);
@@ -643,10 +711,10 @@ hf_status launch_transfer(hf_plan_s* p, const void* sender, void* receiver, cuda
       2LL * d.L_r * ((p->T_r + kBM - 1) / kBM) * static_cast<int64_t>(P.n_tiles_n);
   const int grid = static_cast<int>(std::min<int64_t>(device_sm_count(), max_tiles));
   if (f32)
-    return p->gather ? launch_typed<float, true>(ms, mw, P, grid, smem, stream)
-                     : launch_typed<float, false>(ms, mw, P, grid, smem, stream);
-  return p->gather ? launch_typed<__nv_bfloat16, true>(ms, mw, P, grid, smem, stream)
-                   : launch_typed<__nv_bfloat16, false>(ms, mw, P, grid, smem, stream);
+    return p->gather ? launch_typed<float, true>(mw, P, grid, smem, stream)
+                     : launch_typed<float, false>(mw, P, grid, smem, stream);
+  return p->gather ? launch_typed<__nv_bfloat16, true>(mw, P, grid, smem, stream)
+                   : launch_typed<__nv_bfloat16, false>(mw, P, grid, smem, stream);
 }
 
 }  // namespace hf
