@@ -44,10 +44,9 @@ namespace {
 constexpr int kBM = 128;                 // distinct rows per tile (UMMA M)
 constexpr int kThreads = 448;            // 14 warps
 constexpr int kStageABytes = kBM * 128;  // 128 rows x 128 bytes
-constexpr int kStgFloats = kBM * 32;     // epilogue staging per group
-constexpr int kRunStride = 132;          // run starts / positions per group (129 used)
+constexpr int kStgFloats = kBM * 64;     // epilogue staging: 128 rows x 2 heads x 32
+constexpr int kRunStride = 132;          // run starts / positions of a tile (129 used)
 constexpr int kMaxStages = 8;
-constexpr int kLag = 3;                  // cp.async groups in flight per loader thread
 constexpr int kTmemCols = 512;           // two accumulators of up to 256 columns
 
 struct XferParams {
@@ -70,7 +69,8 @@ struct XferParams {
   int64_t T_s;        // sender rows per (layer, role)
   int64_t recv_rows;  // receiver rows per (layer, role) in receiver_kv
   int L_r, d_s, d_r, D_r;
-  int n_kb, kb_per_seg, BN, n_tiles_n, groups, stages;
+  int n_kb, kb_per_seg, BN, n_tiles_n, groups;
+  int stages_a, stages_b, lag;  // A ring, B ring, cp.async groups in flight per loader
   int rope, paged, knorm;
   float knorm_eps;
   uint32_t idesc;
@@ -139,55 +139,78 @@ __device__ __forceinline__ uint4 pack16(const float* a, const float*) {
                     __float_as_uint(a[3]));
 }
 
-// One chain of the epilogue's position walk: a lane's two rotation pairs at
-// receiver row j (row u of the tile), with RoPE state carried from the
-// chain's previous position four rows back.
-struct Chain {
-  int u;          // tile row holding the current position
-  int expect;     // position this chain expects next (angle-addition valid)
-  float cs0, sn0, cs1, sn1;
+__device__ __forceinline__ void store4(__nv_bfloat16* p, const float4& v) {
+  const __nv_bfloat162 x = __floats2bfloat162_rn(v.x, v.y), y = __floats2bfloat162_rn(v.z, v.w);
+  *reinterpret_cast<uint2*>(p) =
+      make_uint2(*reinterpret_cast<const uint32_t*>(&x), *reinterpret_cast<const uint32_t*>(&y));
+}
+__device__ __forceinline__ void store4(float* p, const float4& v) {
+  *reinterpret_cast<float4*>(p) = v;
+}
+
+// Rotates the pairs (x[k], y[k]) by the angles with cosines c[k], sines s[k].
+__device__ __forceinline__ void rotate4(float4& x, float4& y, const float* c, const float* s) {
+  const float x0 = x.x * c[0] - y.x * s[0], y0 = y.x * c[0] + x.x * s[0];
+  const float x1 = x.y * c[1] - y.y * s[1], y1 = y.y * c[1] + x.y * s[1];
+  const float x2 = x.z * c[2] - y.z * s[2], y2 = y.z * c[2] + x.z * s[2];
+  const float x3 = x.w * c[3] - y.w * s[3], y3 = y.w * c[3] + x.w * s[3];
+  x = make_float4(x0, x1, x2, x3);
+  y = make_float4(y0, y1, y2, y3);
+}
+
+// The epilogue's position walk: a lane owns four rotation pairs (columns
+// q+4*qq .. +3 of the first half of each head and their partners half
+// further on) of one receiver row j at a time, for up to two heads, and
+// carries the RoPE angles of its four frequencies from row j - 8.
+struct Walk {
+  int u;       // tile row holding the current receiver row
+  int expect;  // position for which the carried angles are valid
+  float cs[4], sn[4];
 };
 
 template <typename T>
-__device__ __forceinline__ void walk_step(Chain& ch, int j, int it, const int32_t* srun,
-                                          const int32_t* supos, const float* stg, int pl, int p0,
-                                          bool do_rope, float f0, float f1, float C0, float S0,
-                                          float C1, float S1, const XferParams& P, T* out_lc,
-                                          int ocol, int q, int half) {
+__device__ __forceinline__ void walk_step(Walk& w, int j, int it, const int32_t* srun,
+                                          const int32_t* supos, const float* stg, int qq,
+                                          bool two_heads, bool do_rope, const float* f,
+                                          const float* C8, const float* S8, const XferParams& P,
+                                          T* out_lc, int ocol, int q, int half) {
   const int drow = P.paged ? __ldg(P.dst_row + j) : j;
-  while (srun[ch.u + 1] <= j) ++ch.u;
-  const int u = ch.u;
-  const float* urow = stg + u * 32;
+  while (srun[w.u + 1] <= j) ++w.u;
+  const int u = w.u;
+  const float* urow = stg + u * 64;
   const int sw = u & 7;
-  const float2 lo = *reinterpret_cast<const float2*>(urow + (((pl >> 1) ^ sw) << 2) + (p0 & 3));
-  const float2 hi =
-      *reinterpret_cast<const float2*>(urow + (((4 + (pl >> 1)) ^ sw) << 2) + (p0 & 3));
-  float a0 = lo.x, a1 = lo.y, b0 = hi.x, b1 = hi.y;
+  float4 a0 = *reinterpret_cast<const float4*>(urow + ((qq ^ sw) << 2));
+  float4 b0 = *reinterpret_cast<const float4*>(urow + (((4 + qq) ^ sw) << 2));
+  float4 a1 = make_float4(0.f, 0.f, 0.f, 0.f), b1 = a1;
+  if (two_heads) {
+    a1 = *reinterpret_cast<const float4*>(urow + 32 + ((qq ^ sw) << 2));
+    b1 = *reinterpret_cast<const float4*>(urow + 32 + (((4 + qq) ^ sw) << 2));
+  }
   if (do_rope) {
     const int p = supos[u] + (j - srun[u]);
-    if (p != ch.expect || (it & 15) == 0) {
-      rope_sincos(p, f0, &ch.sn0, &ch.cs0);
-      rope_sincos(p, f1, &ch.sn1, &ch.cs1);
-    } else {  // advance the angle by four positions
-      const float t0 = ch.cs0 * C0 - ch.sn0 * S0;
-      ch.sn0 = ch.sn0 * C0 + ch.cs0 * S0;
-      ch.cs0 = t0;
-      const float t1 = ch.cs1 * C1 - ch.sn1 * S1;
-      ch.sn1 = ch.sn1 * C1 + ch.cs1 * S1;
-      ch.cs1 = t1;
+    if (p != w.expect || (it & 15) == 0) {
+#pragma unroll
+      for (int k = 0; k < 4; ++k) rope_sincos(p, f[k], &w.sn[k], &w.cs[k]);
+    } else {  // advance every angle by eight positions
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const float t = w.cs[k] * C8[k] - w.sn[k] * S8[k];
+        w.sn[k] = w.sn[k] * C8[k] + w.cs[k] * S8[k];
+        w.cs[k] = t;
+      }
     }
-    ch.expect = p + 4;
-    const float oa0 = a0 * ch.cs0 - b0 * ch.sn0, ob0 = b0 * ch.cs0 + a0 * ch.sn0;
-    const float oa1 = a1 * ch.cs1 - b1 * ch.sn1, ob1 = b1 * ch.cs1 + a1 * ch.sn1;
-    a0 = oa0;
-    b0 = ob0;
-    a1 = oa1;
-    b1 = ob1;
+    w.expect = p + 8;
+    rotate4(a0, b0, w.cs, w.sn);
+    if (two_heads) rotate4(a1, b1, w.cs, w.sn);
   }
   if (drow >= 0) {
-    T* o = out_lc + static_cast<int64_t>(drow) * P.d_r + ocol;
-    store_pair(o + q + p0, a0, a1);
-    store_pair(o + half + q + p0, b0, b1);
+    T* o = out_lc + static_cast<int64_t>(drow) * P.d_r + ocol + q + 4 * qq;
+    store4(o, a0);
+    store4(o + half, b0);
+    if (two_heads) {
+      store4(o + 2 * half, a1);
+      store4(o + 3 * half, b1);
+    }
   }
 }
 
@@ -201,6 +224,71 @@ __device__ __forceinline__ int find_row(const int32_t* srun, int nrows, int j) {
   return lo;
 }
 
+// A tile rows for one-entry alignment rows: the 128 sender rows of a tile
+// are copied with cp.async, eight lanes per 128-byte row (lane -> row
+// 32*slab + 4*i + lane/8, 16-byte chunk lane%8), into the 128-byte swizzled
+// layout.  A thread keeps LAG groups in flight: after committing k-block i
+// it waits for k-block i-LAG, fences it to the async proxy and arrives on
+// that stage's barrier.
+template <typename T, int LAG>
+__device__ __forceinline__ void gather_rows(const XferParams& P, uint8_t* sA, uint64_t* full_a,
+                                            uint64_t* empty_a, volatile int* sAbort, int t,
+                                            int lane, int U, int total_tiles, int tiles_per_lc) {
+  constexpr int kBK = Elem<T>::kBK;
+  constexpr int kPerChunk = 16 / sizeof(T);
+  const T* sender = reinterpret_cast<const T*>(P.sender);
+  const int stages = P.stages_a;
+  const int slab = t >> 5, rsub = lane >> 3, ch = lane & 7;
+  int stage = 0;
+  uint32_t phase = 0;
+  int pending = 0;  // committed groups whose stage arrival is still owed
+  bool ok = true;
+  for (int tile = blockIdx.x; tile < total_tiles && ok; tile += gridDim.x) {
+    int lc, m, n;
+    decode_tile(tile, tiles_per_lc, P.n_tiles_n, &lc, &m, &n);
+    const int l = lc >> 1, c = lc & 1;
+    const LayerSegs* segs = P.segs + l;
+    int64_t roff[8];
+    uint32_t doff[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int r = slab * 32 + 4 * i + rsub;
+      const int u = min(m * kBM + r, U - 1);
+      roff[i] = static_cast<int64_t>(P.ucol[u]) * P.d_s + ch * kPerChunk;
+      doff[i] = static_cast<uint32_t>(r * 128 + ((ch ^ (r & 7)) << 4));
+    }
+    for (int kb = 0; kb < P.n_kb; ++kb) {
+      const int seg = kb / P.kb_per_seg;
+      const int kin = kb - seg * P.kb_per_seg;
+      if (!mbar_wait(smem_addr(&empty_a[stage]), phase ^ 1)) {
+        raise_timeout(P, sAbort);
+        ok = false;
+        break;
+      }
+      const int tl = segs->layer[seg][0];
+      const T* base = sender + (static_cast<int64_t>(tl * 2 + c) * P.T_s) * P.d_s + kin * kBK;
+      const uint32_t sa = smem_addr(sA + stage * kStageABytes);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) cp_async_16(sa + doff[i], base + roff[i]);
+      cp_async_commit();
+      if (pending == LAG) {
+        cp_async_wait<LAG>();
+        fence_proxy_async_smem();
+        mbar_arrive(smem_addr(&full_a[(stage + stages - LAG) % stages]));
+      } else {
+        ++pending;
+      }
+      if (++stage == stages) {
+        stage = 0;
+        phase ^= 1;
+      }
+    }
+  }
+  cp_async_wait<0>();
+  fence_proxy_async_smem();
+  for (int k = pending; k >= 1; --k) mbar_arrive(smem_addr(&full_a[(stage + stages - k) % stages]));
+}
+
 template <typename T, bool kGather>
 __global__ void __launch_bounds__(kThreads, 1)
     transfer_kernel(const __grid_constant__ CUtensorMap tmap_w, const XferParams P) {
@@ -211,17 +299,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) atomicOr(P.status, HF_CHECK_INTERNAL);
     return;
   }
-  const int stages = P.stages;
+  const int stages_a = P.stages_a, stages_b = P.stages_b;
   const int stage_b_bytes = P.BN * 128;
   uint8_t* sA = smem;
-  uint8_t* sB = sA + stages * kStageABytes;
-  float* sStg = reinterpret_cast<float*>(sB + stages * stage_b_bytes);
-  int32_t* sRun = reinterpret_cast<int32_t*>(sStg + 2 * kStgFloats);
-  int32_t* sUpos = sRun + 2 * kRunStride;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sUpos + 2 * kRunStride);
-  uint64_t* full = bars;
-  uint64_t* empty = bars + kMaxStages;
-  uint64_t* tfull = bars + 2 * kMaxStages;
+  uint8_t* sB = sA + stages_a * kStageABytes;
+  float* sStg = reinterpret_cast<float*>(sB + stages_b * stage_b_bytes);
+  int32_t* sRun = reinterpret_cast<int32_t*>(sStg + kStgFloats);
+  int32_t* sUpos = sRun + kRunStride;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sUpos + kRunStride);
+  uint64_t* full_a = bars;
+  uint64_t* empty_a = bars + kMaxStages;
+  uint64_t* full_b = bars + 2 * kMaxStages;
+  uint64_t* empty_b = bars + 3 * kMaxStages;
+  uint64_t* tfull = bars + 4 * kMaxStages;
   uint64_t* tempty = tfull + 2;
   uint64_t* drain = tempty + 2;
   uint32_t* sTmem = reinterpret_cast<uint32_t*>(drain + 1);
@@ -230,9 +320,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < stages; ++s) {
-      mbar_init(smem_addr(&full[s]), 1 + kBM);  // TMA expect_tx + 128 A builders
-      mbar_init(smem_addr(&empty[s]), 1);
+    for (int s = 0; s < stages_a; ++s) {
+      mbar_init(smem_addr(&full_a[s]), kBM);  // one arrival per A builder thread
+      mbar_init(smem_addr(&empty_a[s]), 1);
+    }
+    for (int s = 0; s < stages_b; ++s) {
+      mbar_init(smem_addr(&full_b[s]), 1);  // expect_tx + the TMA bytes
+      mbar_init(smem_addr(&empty_b[s]), 1);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(smem_addr(&tfull[a]), 1);
@@ -266,16 +360,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         int lc, m, n;
         decode_tile(tile, tiles_per_lc, P.n_tiles_n, &lc, &m, &n);
         for (int kb = 0; kb < P.n_kb; ++kb) {
-          if (!mbar_wait(smem_addr(&empty[stage]), phase ^ 1)) {
+          if (!mbar_wait(smem_addr(&empty_b[stage]), phase ^ 1)) {
             raise_timeout(P, sAbort);
             ok = false;
             break;
           }
-          const uint32_t fb = smem_addr(&full[stage]);
+          const uint32_t fb = smem_addr(&full_b[stage]);
           mbar_arrive_expect_tx(fb, stage_b_bytes);
           tma_load_2d(smem_addr(sB + stage * stage_b_bytes), &tmap_w, kb * kBK,
                       lc * P.d_r + n * P.BN, fb);
-          if (++stage == stages) {
+          if (++stage == stages_b) {
             stage = 0;
             phase ^= 1;
           }
@@ -286,8 +380,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issue
     if (lane == 0) {
-      int stage = 0;
-      uint32_t phase = 0;
+      int sa = 0, sb = 0;
+      uint32_t pa = 0, pb = 0;
       int acc = 0;
       uint32_t acc_phase = 0;
       bool ok = true;
@@ -299,14 +393,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_after_sync();
         const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * 256);
         for (int kb = 0; kb < P.n_kb; ++kb) {
-          if (!mbar_wait(smem_addr(&full[stage]), phase)) {
+          if (!mbar_wait(smem_addr(&full_a[sa]), pa) || !mbar_wait(smem_addr(&full_b[sb]), pb)) {
             raise_timeout(P, sAbort);
             ok = false;
             break;
           }
           tc_fence_after_sync();
-          const uint32_t a0 = smem_addr(sA + stage * kStageABytes);
-          const uint32_t b0 = smem_addr(sB + stage * stage_b_bytes);
+          const uint32_t a0 = smem_addr(sA + sa * kStageABytes);
+          const uint32_t b0 = smem_addr(sB + sb * stage_b_bytes);
 #pragma unroll
           for (int k = 0; k < 4; ++k) {  // four 32-byte K steps per 128-byte k-block
             const uint64_t ad = sw128_kmajor_desc(a0 + 32 * k);
@@ -316,10 +410,15 @@ __global__ void __launch_bounds__(kThreads, 1)
             else
               mma_tf32(d_tmem, ad, bd, P.idesc, (kb | k) != 0);
           }
-          tc_commit(smem_addr(&empty[stage]));
-          if (++stage == stages) {
-            stage = 0;
-            phase ^= 1;
+          tc_commit(smem_addr(&empty_a[sa]));
+          tc_commit(smem_addr(&empty_b[sb]));
+          if (++sa == stages_a) {
+            sa = 0;
+            pa ^= 1;
+          }
+          if (++sb == stages_b) {
+            sb = 0;
+            pb ^= 1;
           }
         }
         if (!ok) break;
@@ -334,17 +433,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
   } else if (warp < 10) {
     // ------------------------------------------------------------ epilogue
-    const int g = (warp - 2) >> 2;
+    // Eight warps.  Step 1 (per 16 rotation pairs of a head pair): warp
+    // (g, sp) reads TMEM lane quarter sp of head 2*hp+g, applies 1/r, bias
+    // and key norm, and stages fp32 rows in smem.  Step 2: the eight warps
+    // split the tile's receiver rows and write both heads, rotated.
+    const int e = warp - 2;   // 0..7: slice of the tile's receiver rows
+    const int g = e >> 2;     // head of the pair this warp stages
     const int sp = warp & 3;  // TMEM lane quarter this warp may access
     const int row = sp * 32 + lane;
-    float* stg = sStg + g * kStgFloats;
-    int32_t* srun = sRun + g * kRunStride;
-    int32_t* supos = sUpos + g * kRunStride;
-    const bool active = P.groups == 2 || g == 0;
-    const int gcols = P.groups == 2 ? P.BN / 2 : P.BN;
-    const int gcol0 = P.groups == 2 ? g * (P.BN / 2) : 0;
+    const int tid_e = threadIdx.x - 64;
     const int D = P.D_r, half = P.D_r / 2;
-    const int pg = lane >> 3, pl = lane & 7, p0 = 2 * pl;
+    const int n_heads = P.BN / D;
+    const bool two_heads = n_heads >= 2;
+    const int n_pairs = two_heads ? n_heads / 2 : 1;
+    const int ps = lane >> 2, qq = lane & 3;  // row slot 0..7, pair quad 0..3
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int tile = blockIdx.x; tile < total_tiles; tile += gridDim.x) {
@@ -356,66 +458,66 @@ __global__ void __launch_bounds__(kThreads, 1)
         break;
       }
       tc_fence_after_sync();
-      if (active) {
-        const int u0 = m * kBM;
-        const int nrows = min(kBM, U - u0);
-        for (int i = row; i <= nrows; i += kBM) {
-          srun[i] = P.run_ptr[u0 + i];
-          supos[i] = i < nrows ? P.upos[u0 + i] : 0;
-        }
-        named_barrier_sync(1 + g, 128);
-        // this warp's receiver rows [wjb, wje), walked as two chains
-        const int jb = srun[0], je = srun[nrows];
-        const int per = (je - jb + 3) >> 2;
-        const int wjb = min(je, jb + sp * per), wje = min(je, wjb + per);
-        const int hlen = (((wje - wjb + 1) >> 1) + 3) & ~3;  // chain A length, multiple of 4
-        const int amid = min(wje, wjb + hlen);
-        const int n_it = (hlen + 3) >> 2;
-        const int ja0 = wjb + pg, jb0 = amid + pg;
-        const int ua0 = ja0 < amid ? find_row(srun, nrows, ja0) : 0;
-        const int ub0 = jb0 < wje ? find_row(srun, nrows, jb0) : 0;
-        const float inv_r = P.inv_r[lc];
-        const float* bias = P.bias + static_cast<int64_t>(lc) * P.d_r;
-        const bool do_rope = P.rope && c == 0;
-        const bool do_knorm = P.knorm && c == 0;
-        const uint32_t ta = tmem_base + static_cast<uint32_t>(acc * 256) +
-                            (static_cast<uint32_t>(sp * 32) << 16);
-        T* const out_lc = reinterpret_cast<T*>(P.receiver) +
-                          (static_cast<int64_t>(lc) * P.recv_rows) * P.d_r;
-        for (int h0 = 0; h0 < gcols; h0 += D) {
-          const int tcol = gcol0 + h0;       // accumulator column of the head
-          const int ocol = n * P.BN + tcol;  // receiver feature index of the head
-          float rn = 1.0f;
-          if (do_knorm) {
-            float ss = 0.0f;
-            for (int q2 = 0; q2 < D; q2 += 16) {
-              uint32_t v[16];
-              tmem_load_16(ta + tcol + q2, v);
-#pragma unroll
-              for (int i = 0; i < 16; ++i) {
-                const float y = fmaf(__uint_as_float(v[i]), inv_r, __ldg(bias + ocol + q2 + i));
-                ss = fmaf(y, y, ss);
-              }
-            }
-            rn = rsqrtf(ss / static_cast<float>(D) + P.knorm_eps);
-          }
-          for (int q = 0; q < half; q += 16) {
-            // step 1: 16 rotation pairs (columns q.., half+q..) of every row -> smem
-            uint32_t v[32];
-            tmem_load_2x16(ta + tcol + q, ta + tcol + half + q, v);
-            float bl[16], bh[16];
-#pragma unroll
-            for (int i = 0; i < 16; i += 4) {
-              const float4 x = __ldg(reinterpret_cast<const float4*>(bias + ocol + q + i));
-              const float4 z = __ldg(reinterpret_cast<const float4*>(bias + ocol + half + q + i));
-              bl[i] = x.x; bl[i + 1] = x.y; bl[i + 2] = x.z; bl[i + 3] = x.w;
-              bh[i] = z.x; bh[i + 1] = z.y; bh[i + 2] = z.z; bh[i + 3] = z.w;
-            }
-            float y[32];
+      const int u0 = m * kBM;
+      const int nrows = min(kBM, U - u0);
+      for (int i = tid_e; i <= nrows; i += 256) {
+        sRun[i] = P.run_ptr[u0 + i];
+        sUpos[i] = i < nrows ? P.upos[u0 + i] : 0;
+      }
+      named_barrier_sync(1, 256);
+      // this warp's receiver rows [wjb, wje); lane slot ps takes rows wjb+ps, +8, ...
+      const int jb = sRun[0], je = sRun[nrows];
+      const int per = (je - jb + 7) >> 3;
+      const int wjb = min(je, jb + e * per), wje = min(je, wjb + per);
+      const int n_it = (wje - wjb + 7) >> 3;
+      const int j0 = wjb + ps;
+      const int ustart = j0 < wje ? find_row(sRun, nrows, j0) : 0;
+      const float inv_r = P.inv_r[lc];
+      const float* bias = P.bias + static_cast<int64_t>(lc) * P.d_r;
+      const bool do_rope = P.rope && c == 0;
+      const bool do_knorm = P.knorm && c == 0;
+      const uint32_t ta = tmem_base + static_cast<uint32_t>(acc * 256) +
+                          (static_cast<uint32_t>(sp * 32) << 16);
+      T* const out_lc = reinterpret_cast<T*>(P.receiver) +
+                        (static_cast<int64_t>(lc) * P.recv_rows) * P.d_r;
+      for (int hp = 0; hp < n_pairs; ++hp) {
+        const bool stages_head = g == 0 || two_heads;
+        const int tcol = (2 * hp + g) * D;           // accumulator column of this warp's head
+        const int ocol_pair = n * P.BN + 2 * hp * D;  // receiver feature of the pair's first head
+        float rn = 1.0f;
+        if (do_knorm && stages_head) {
+          float ss = 0.0f;
+          for (int q2 = 0; q2 < D; q2 += 16) {
+            uint32_t v[16];
+            tmem_load_16(ta + tcol + q2, v);
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
-              y[i] = fmaf(__uint_as_float(v[i]), inv_r, bl[i]);
-              y[16 + i] = fmaf(__uint_as_float(v[16 + i]), inv_r, bh[i]);
+              const float y = fmaf(__uint_as_float(v[i]), inv_r,
+                                   __ldg(bias + n * P.BN + tcol + q2 + i));
+              ss = fmaf(y, y, ss);
+            }
+          }
+          rn = rsqrtf(ss / static_cast<float>(D) + P.knorm_eps);
+        }
+        for (int q = 0; q < half; q += 16) {
+          if (stages_head) {
+            // step 1: pairs q..q+15 of head 2*hp+g for this warp's 32 rows
+            uint32_t v[32];
+            tmem_load_2x16(ta + tcol + q, ta + tcol + half + q, v);
+            const float* bcol = bias + n * P.BN + tcol;
+            float y[32];
+#pragma unroll
+            for (int i = 0; i < 16; i += 4) {
+              const float4 x = __ldg(reinterpret_cast<const float4*>(bcol + q + i));
+              const float4 z = __ldg(reinterpret_cast<const float4*>(bcol + half + q + i));
+              y[i] = fmaf(__uint_as_float(v[i]), inv_r, x.x);
+              y[i + 1] = fmaf(__uint_as_float(v[i + 1]), inv_r, x.y);
+              y[i + 2] = fmaf(__uint_as_float(v[i + 2]), inv_r, x.z);
+              y[i + 3] = fmaf(__uint_as_float(v[i + 3]), inv_r, x.w);
+              y[16 + i] = fmaf(__uint_as_float(v[16 + i]), inv_r, z.x);
+              y[16 + i + 1] = fmaf(__uint_as_float(v[16 + i + 1]), inv_r, z.y);
+              y[16 + i + 2] = fmaf(__uint_as_float(v[16 + i + 2]), inv_r, z.z);
+              y[16 + i + 3] = fmaf(__uint_as_float(v[16 + i + 3]), inv_r, z.w);
             }
             if (do_knorm) {
 #pragma unroll
@@ -424,34 +526,37 @@ __global__ void __launch_bounds__(kThreads, 1)
                 y[16 + i] *= rn * __ldg(P.knorm_w + half + q + i);
               }
             }
-            float* srow = stg + row * 32;
+            float* srow = sStg + row * 64 + g * 32;
 #pragma unroll
             for (int k = 0; k < 8; ++k)
               *reinterpret_cast<float4*>(srow + ((k ^ (row & 7)) << 2)) =
                   make_float4(y[4 * k], y[4 * k + 1], y[4 * k + 2], y[4 * k + 3]);
-            named_barrier_sync(1 + g, 128);
-            // step 2: lanes 8*pg .. 8*pg+7 own rows j = chain start + pg + 4*it
-            // (two pairs each); a step advances the RoPE angle by four rows.
-            float f0 = 0.f, f1 = 0.f, C0 = 1.f, S0 = 0.f, C1 = 1.f, S1 = 0.f;
-            if (do_rope) {
-              f0 = __ldg(P.inv_freq + q + p0);
-              f1 = __ldg(P.inv_freq + q + p0 + 1);
-              rope_sincos(4, f0, &S0, &C0);
-              rope_sincos(4, f1, &S1, &C1);
-            }
-            Chain ca{ua0, INT_MIN, 1.f, 0.f, 1.f, 0.f};
-            Chain cb{ub0, INT_MIN, 1.f, 0.f, 1.f, 0.f};
-            for (int it = 0; it < n_it; ++it) {
-              const int ja = ja0 + 4 * it, jbb = jb0 + 4 * it;
-              if (ja < amid)
-                walk_step<T>(ca, ja, it, srun, supos, stg, pl, p0, do_rope, f0, f1, C0, S0, C1,
-                             S1, P, out_lc, ocol, q, half);
-              if (jbb < wje)
-                walk_step<T>(cb, jbb, it, srun, supos, stg, pl, p0, do_rope, f0, f1, C0, S0, C1,
-                             S1, P, out_lc, ocol, q, half);
-            }
-            named_barrier_sync(1 + g, 128);
           }
+          named_barrier_sync(1, 256);
+          // step 2: rows of this warp's slice, both heads of the pair
+          float f[4], C8[4], S8[4];
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            f[k] = do_rope ? __ldg(P.inv_freq + q + 4 * qq + k) : 0.f;
+            C8[k] = 1.f;
+            S8[k] = 0.f;
+            if (do_rope) rope_sincos(8, f[k], &S8[k], &C8[k]);  // one step = eight rows
+          }
+          Walk wk;
+          wk.u = ustart;
+          wk.expect = INT_MIN;
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            wk.cs[k] = 1.f;
+            wk.sn[k] = 0.f;
+          }
+          for (int it = 0; it < n_it; ++it) {
+            const int j = j0 + 8 * it;
+            if (j < wje)
+              walk_step<T>(wk, j, it, sRun, sUpos, sStg, qq, two_heads, do_rope, f, C8, S8, P,
+                           out_lc, ocol_pair, q, half);
+          }
+          named_barrier_sync(1, 256);
         }
       }
       tc_fence_before_sync();
@@ -468,55 +573,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t phase = 0;
     bool ok = true;
     if (kGather) {
-      // eight lanes per 128-byte row: lane -> (row 32*slab + 4*i + lane/8, chunk lane%8)
-      const int slab = t >> 5, rsub = lane >> 3, ch = lane & 7;
-      int pending = 0;  // committed groups whose stage arrival is still owed
-      for (int tile = blockIdx.x; tile < total_tiles && ok; tile += gridDim.x) {
-        int lc, m, n;
-        decode_tile(tile, tiles_per_lc, P.n_tiles_n, &lc, &m, &n);
-        const int l = lc >> 1, c = lc & 1;
-        const LayerSegs* segs = P.segs + l;
-        int64_t roff[8];
-        uint32_t doff[8];
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          const int r = slab * 32 + 4 * i + rsub;
-          const int u = min(m * kBM + r, U - 1);
-          roff[i] = static_cast<int64_t>(P.ucol[u]) * P.d_s + ch * kPerChunk;
-          doff[i] = static_cast<uint32_t>(r * 128 + ((ch ^ (r & 7)) << 4));
-        }
-        for (int kb = 0; kb < P.n_kb; ++kb) {
-          const int seg = kb / P.kb_per_seg;
-          const int kin = kb - seg * P.kb_per_seg;
-          if (!mbar_wait(smem_addr(&empty[stage]), phase ^ 1)) {
-            raise_timeout(P, sAbort);
-            ok = false;
-            break;
-          }
-          const int tl = segs->layer[seg][0];
-          const T* base = sender + (static_cast<int64_t>(tl * 2 + c) * P.T_s) * P.d_s + kin * kBK;
-          const uint32_t sa = smem_addr(sA + stage * kStageABytes);
-#pragma unroll
-          for (int i = 0; i < 8; ++i) cp_async_16(sa + doff[i], base + roff[i]);
-          cp_async_commit();
-          if (pending == kLag) {
-            // the group kLag k-blocks back has landed: publish its stage
-            cp_async_wait<kLag>();
-            fence_proxy_async_smem();
-            const int s_old = (stage + stages - kLag) % stages;
-            mbar_arrive(smem_addr(&full[s_old]));
-          } else {
-            ++pending;
-          }
-          if (++stage == stages) {
-            stage = 0;
-            phase ^= 1;
-          }
-        }
+      switch (P.lag) {
+        case 2: gather_rows<T, 2>(P, sA, full_a, empty_a, sAbort, t, lane, U, total_tiles, tiles_per_lc); break;
+        case 3: gather_rows<T, 3>(P, sA, full_a, empty_a, sAbort, t, lane, U, total_tiles, tiles_per_lc); break;
+        case 4: gather_rows<T, 4>(P, sA, full_a, empty_a, sAbort, t, lane, U, total_tiles, tiles_per_lc); break;
+        default: gather_rows<T, 5>(P, sA, full_a, empty_a, sAbort, t, lane, U, total_tiles, tiles_per_lc); break;
       }
-      cp_async_wait<0>();
-      fence_proxy_async_smem();
-      for (int k = pending; k >= 1; --k) mbar_arrive(smem_addr(&full[(stage + stages - k) % stages]));
     } else {
       // pooled CSR rows and/or blended sender layers: thread t owns tile row t
       for (int tile = blockIdx.x; tile < total_tiles && ok; tile += gridDim.x) {
@@ -530,7 +592,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int kb = 0; kb < P.n_kb; ++kb) {
           const int seg = kb / P.kb_per_seg;
           const int kin = kb - seg * P.kb_per_seg;
-          if (!mbar_wait(smem_addr(&empty[stage]), phase ^ 1)) {
+          if (!mbar_wait(smem_addr(&empty_a[stage]), phase ^ 1)) {
             raise_timeout(P, sAbort);
             ok = false;
             break;
@@ -562,8 +624,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             *reinterpret_cast<uint4*>(dst + ((k2 ^ (t & 7)) << 4)) =
                 pack16(acc + k2 * kPerChunk, (const T*)nullptr);
           fence_proxy_async_smem();
-          mbar_arrive(smem_addr(&full[stage]));
-          if (++stage == stages) {
+          mbar_arrive(smem_addr(&full_a[stage]));
+          if (++stage == stages_a) {
             stage = 0;
             phase ^= 1;
           }
@@ -630,19 +692,25 @@ hf_status make_map(CUtensorMap* map, const void* base, bool f32, uint64_t rows, 
   return HF_OK;
 }
 
-size_t smem_bytes(int BN, int stages) {
-  return static_cast<size_t>(stages) * (kStageABytes + BN * 128) +
-         2 * kStgFloats * sizeof(float) + 4 * kRunStride * sizeof(int32_t) +
-         (2 * kMaxStages + 5) * sizeof(uint64_t) + 8;
+size_t smem_bytes(int BN, int stages_a, int stages_b) {
+  return static_cast<size_t>(stages_a) * kStageABytes + static_cast<size_t>(stages_b) * BN * 128 +
+         kStgFloats * sizeof(float) + 2 * kRunStride * sizeof(int32_t) +
+         (4 * kMaxStages + 5) * sizeof(uint64_t) + 8;
 }
 
-int pick_stages(int BN) {
+// Ring depths: as many A stages as fit next to `stages_b` B stages, with
+// the loaders keeping all but two A stages in flight (so the tensor core
+// always has two k-blocks queued).
+void pick_rings(int BN, int* stages_a, int* stages_b, int* lag) {
   int dev = 0, optin = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
-  int s = 6;
-  while (s > kLag + 1 && smem_bytes(BN, s) > static_cast<size_t>(optin)) --s;
-  return s;
+  int sb = BN == 256 ? 3 : 4;
+  int sa = kMaxStages;
+  while (sa > 4 && smem_bytes(BN, sa, sb) > static_cast<size_t>(optin)) --sa;
+  *stages_a = sa;
+  *stages_b = sb;
+  *lag = std::min(5, std::max(2, sa - 3));
 }
 
 template <typename T, bool kGather>
@@ -700,13 +768,13 @@ hf_status launch_transfer(hf_plan_s* p, const void* sender, void* receiver, cuda
   P.BN = p->BN;
   P.n_tiles_n = p->d_r / p->BN;
   P.groups = p->groups;
-  P.stages = pick_stages(p->BN);
+  pick_rings(p->BN, &P.stages_a, &P.stages_b, &P.lag);
   P.rope = d.theta_r > 0.0 ? 1 : 0;
   P.paged = d.paged ? 1 : 0;
   P.knorm = d.d_knorm_w ? 1 : 0;
   P.knorm_eps = d.knorm_eps;
   P.idesc = make_idesc(f32 ? 2u : 1u, kBM, p->BN);
-  const size_t smem = smem_bytes(p->BN, P.stages);
+  const size_t smem = smem_bytes(p->BN, P.stages_a, P.stages_b);
   const int64_t max_tiles =
       2LL * d.L_r * ((p->T_r + kBM - 1) / kBM) * static_cast<int64_t>(P.n_tiles_n);
   const int grid = static_cast<int>(std::min<int64_t>(device_sm_count(), max_tiles));
