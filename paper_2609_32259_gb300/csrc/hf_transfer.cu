@@ -94,10 +94,16 @@ __device__ __forceinline__ void store_pair(float* p, float a, float b) {
   *reinterpret_cast<float2*>(p) = make_float2(a, b);
 }
 
-__device__ __forceinline__ void decode_tile(int tile, int tiles_per_lc, int n_tiles_n, int* lc,
-                                            int* m, int* n) {
-  *lc = tile / tiles_per_lc;
-  const int rem = tile - *lc * tiles_per_lc;
+// Tile order: role-major, then receiver layer, then 128-row block, then
+// column block.  Consecutive receiver layers of one role share most of their
+// Eq. 1 sender layers, so their A rows are still in L2.  lc = 2 * l + c
+// indexes the maps, biases and receiver cache.
+__device__ __forceinline__ void decode_tile(int tile, int tiles_per_lc, int n_tiles_n, int L_r,
+                                            int* lc, int* m, int* n) {
+  const int ord = tile / tiles_per_lc;
+  const int rem = tile - ord * tiles_per_lc;
+  const int c = ord >= L_r ? 1 : 0;
+  *lc = 2 * (ord - c * L_r) + c;
   *m = rem / n_tiles_n;
   *n = rem - *m * n_tiles_n;
 }
@@ -245,7 +251,7 @@ __device__ __forceinline__ void gather_rows(const XferParams& P, uint8_t* sA, ui
   bool ok = true;
   for (int tile = blockIdx.x; tile < total_tiles && ok; tile += gridDim.x) {
     int lc, m, n;
-    decode_tile(tile, tiles_per_lc, P.n_tiles_n, &lc, &m, &n);
+    decode_tile(tile, tiles_per_lc, P.n_tiles_n, P.L_r, &lc, &m, &n);
     const int l = lc >> 1, c = lc & 1;
     const LayerSegs* segs = P.segs + l;
     int64_t roff[8];
@@ -358,7 +364,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       for (int tile = blockIdx.x; tile < total_tiles && ok; tile += gridDim.x) {
         int lc, m, n;
-        decode_tile(tile, tiles_per_lc, P.n_tiles_n, &lc, &m, &n);
+        decode_tile(tile, tiles_per_lc, P.n_tiles_n, P.L_r, &lc, &m, &n);
         for (int kb = 0; kb < P.n_kb; ++kb) {
           if (!mbar_wait(smem_addr(&empty_b[stage]), phase ^ 1)) {
             raise_timeout(P, sAbort);
@@ -451,7 +457,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t acc_phase = 0;
     for (int tile = blockIdx.x; tile < total_tiles; tile += gridDim.x) {
       int lc, m, n;
-      decode_tile(tile, tiles_per_lc, P.n_tiles_n, &lc, &m, &n);
+      decode_tile(tile, tiles_per_lc, P.n_tiles_n, P.L_r, &lc, &m, &n);
       const int c = lc & 1;
       if (!mbar_wait(smem_addr(&tfull[acc]), acc_phase)) {
         raise_timeout(P, sAbort);
@@ -583,7 +589,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // pooled CSR rows and/or blended sender layers: thread t owns tile row t
       for (int tile = blockIdx.x; tile < total_tiles && ok; tile += gridDim.x) {
         int lc, m, n;
-        decode_tile(tile, tiles_per_lc, P.n_tiles_n, &lc, &m, &n);
+        decode_tile(tile, tiles_per_lc, P.n_tiles_n, P.L_r, &lc, &m, &n);
         const int l = lc >> 1, c = lc & 1;
         const LayerSegs segs = P.segs[l];
         const int u = min(m * kBM + t, U - 1);
