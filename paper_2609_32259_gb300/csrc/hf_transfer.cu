@@ -41,8 +41,10 @@
 namespace hf {
 namespace {
 
-constexpr int kBM = 128;                 // distinct rows per tile (UMMA M)
+constexpr int kBM = 128;                 // distinct rows per CTA of a pair tile
+constexpr int kPairRows = 2 * kBM;       // distinct rows per pair tile (UMMA M = 256)
 constexpr int kThreads = 448;            // 14 warps
+constexpr int kBuilderWarps = 4;         // A tile builders: warps 10-13
 constexpr int kStageABytes = kBM * 128;  // 128 rows x 128 bytes
 constexpr int kStgFloats = kBM * 64;     // epilogue staging: 128 rows x 2 heads x 32
 constexpr int kRunStride = 132;          // run starts / positions of a tile (129 used)
@@ -86,13 +88,6 @@ template <>
 struct Elem<float> {
   static constexpr int kBK = 32;
 };
-
-__device__ __forceinline__ void store_pair(__nv_bfloat16* p, float a, float b) {
-  *reinterpret_cast<__nv_bfloat162*>(p) = __floats2bfloat162_rn(a, b);
-}
-__device__ __forceinline__ void store_pair(float* p, float a, float b) {
-  *reinterpret_cast<float2*>(p) = make_float2(a, b);
-}
 
 // Tile order: role-major, then receiver layer, then 128-row block, then
 // column block.  Consecutive receiver layers of one role share most of their
@@ -230,16 +225,27 @@ __device__ __forceinline__ int find_row(const int32_t* srun, int nrows, int j) {
   return lo;
 }
 
-// A tile rows for one-entry alignment rows: the 128 sender rows of a tile
-// are copied with cp.async, eight lanes per 128-byte row (lane -> row
+// Arrival on the leader CTA's copy of a pair barrier (`bar` is the local
+// offset): a local arrive in the leader, a relaxed remote arrive in the
+// follower.  What is announced is complete and visible before the call.
+__device__ __forceinline__ void arrive_leader(uint32_t bar, int row0) {
+  if (row0 == 0)
+    mbar_arrive_relaxed(bar);
+  else
+    mbar_arrive_cluster(mapa_shared(bar, 0));
+}
+
+// A tile rows for one-entry alignment rows: this CTA's 128 sender rows of a
+// tile are copied with cp.async, eight lanes per 128-byte row (lane -> row
 // 32*slab + 4*i + lane/8, 16-byte chunk lane%8), into the 128-byte swizzled
 // layout.  A thread keeps LAG groups in flight: after committing k-block i
-// it waits for k-block i-LAG, fences it to the async proxy and arrives on
-// that stage's barrier.
+// it waits for k-block i-LAG and fences it to the async proxy; then one lane
+// per warp arrives on that stage's barrier in the leader CTA of the pair.
 template <typename T, int LAG>
 __device__ __forceinline__ void gather_rows(const XferParams& P, uint8_t* sA, uint64_t* full_a,
                                             uint64_t* empty_a, volatile int* sAbort, int t,
-                                            int lane, int U, int total_tiles, int tiles_per_lc) {
+                                            int lane, int U, int row0, int total_tiles,
+                                            int tiles_per_lc, int first_tile, int tile_step) {
   constexpr int kBK = Elem<T>::kBK;
   constexpr int kPerChunk = 16 / sizeof(T);
   const T* sender = reinterpret_cast<const T*>(P.sender);
@@ -249,17 +255,21 @@ __device__ __forceinline__ void gather_rows(const XferParams& P, uint8_t* sA, ui
   uint32_t phase = 0;
   int pending = 0;  // committed groups whose stage arrival is still owed
   bool ok = true;
-  for (int tile = blockIdx.x; tile < total_tiles && ok; tile += gridDim.x) {
+  for (int tile = first_tile; tile < total_tiles && ok; tile += tile_step) {
     int lc, m, n;
     decode_tile(tile, tiles_per_lc, P.n_tiles_n, P.L_r, &lc, &m, &n);
     const int l = lc >> 1, c = lc & 1;
-    const LayerSegs* segs = P.segs + l;
+    // element offset of each segment's sender layer/role block, for the whole tile
+    int64_t seg_base[kMaxSeg];
+#pragma unroll
+    for (int s2 = 0; s2 < kMaxSeg; ++s2)
+      seg_base[s2] = (static_cast<int64_t>(P.segs[l].layer[s2][0] * 2 + c) * P.T_s) * P.d_s;
     int64_t roff[8];
     uint32_t doff[8];
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
       const int r = slab * 32 + 4 * i + rsub;
-      const int u = min(m * kBM + r, U - 1);
+      const int u = min(m * kPairRows + row0 + r, U - 1);
       roff[i] = static_cast<int64_t>(P.ucol[u]) * P.d_s + ch * kPerChunk;
       doff[i] = static_cast<uint32_t>(r * 128 + ((ch ^ (r & 7)) << 4));
     }
@@ -271,8 +281,8 @@ __device__ __forceinline__ void gather_rows(const XferParams& P, uint8_t* sA, ui
         ok = false;
         break;
       }
-      const int tl = segs->layer[seg][0];
-      const T* base = sender + (static_cast<int64_t>(tl * 2 + c) * P.T_s) * P.d_s + kin * kBK;
+      const int64_t sbase = seg == 0 ? seg_base[0] : (seg == 1 ? seg_base[1] : seg_base[2]);
+      const T* base = sender + sbase + kin * kBK;
       const uint32_t sa = smem_addr(sA + stage * kStageABytes);
 #pragma unroll
       for (int i = 0; i < 8; ++i) cp_async_16(sa + doff[i], base + roff[i]);
@@ -280,7 +290,8 @@ __device__ __forceinline__ void gather_rows(const XferParams& P, uint8_t* sA, ui
       if (pending == LAG) {
         cp_async_wait<LAG>();
         fence_proxy_async_smem();
-        mbar_arrive(smem_addr(&full_a[(stage + stages - LAG) % stages]));
+        __syncwarp();  // the warp's copies of that stage have landed
+        if (lane == 0) arrive_leader(smem_addr(&full_a[(stage + stages - LAG) % stages]), row0);
       } else {
         ++pending;
       }
@@ -292,7 +303,10 @@ __device__ __forceinline__ void gather_rows(const XferParams& P, uint8_t* sA, ui
   }
   cp_async_wait<0>();
   fence_proxy_async_smem();
-  for (int k = pending; k >= 1; --k) mbar_arrive(smem_addr(&full_a[(stage + stages - k) % stages]));
+  __syncwarp();
+  if (lane == 0)
+    for (int k = pending; k >= 1; --k)
+      arrive_leader(smem_addr(&full_a[(stage + stages - k) % stages]), row0);
 }
 
 template <typename T, bool kGather>
@@ -305,8 +319,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) atomicOr(P.status, HF_CHECK_INTERNAL);
     return;
   }
+  const uint32_t rank = cluster_ctarank();  // 0: leader of the pair (issues the MMAs)
+  const bool leader = rank == 0;
+  const int first_tile = static_cast<int>(cluster_id_x());
+  const int tile_step = static_cast<int>(nclusters_x());
+  const int row0 = static_cast<int>(rank) * kBM;  // this CTA's rows within a pair tile
   const int stages_a = P.stages_a, stages_b = P.stages_b;
-  const int stage_b_bytes = P.BN * 128;
+  const int half_bn = P.BN / 2;                    // B rows (receiver columns) per CTA
+  const int stage_b_bytes = half_bn * 128;
   uint8_t* sA = smem;
   uint8_t* sB = sA + stages_a * kStageABytes;
   float* sStg = reinterpret_cast<float*>(sB + stages_b * stage_b_bytes);
@@ -326,17 +346,20 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
+    // full_a / full_b / tempty of the leader collect both CTAs' arrivals;
+    // the follower's copies are unused.  empty_* / tfull / drain receive the
+    // leader's multicast commits in both CTAs.
     for (int s = 0; s < stages_a; ++s) {
-      mbar_init(smem_addr(&full_a[s]), kBM);  // one arrival per A builder thread
+      mbar_init(smem_addr(&full_a[s]), 2 * kBuilderWarps);  // every A builder warp of the pair
       mbar_init(smem_addr(&empty_a[s]), 1);
     }
     for (int s = 0; s < stages_b; ++s) {
-      mbar_init(smem_addr(&full_b[s]), 1);  // expect_tx + the TMA bytes
+      mbar_init(smem_addr(&full_b[s]), 2);  // one expect_tx per CTA + the TMA bytes
       mbar_init(smem_addr(&empty_b[s]), 1);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(smem_addr(&tfull[a]), 1);
-      mbar_init(smem_addr(&tempty[a]), 8);  // one arrival per epilogue warp
+      mbar_init(smem_addr(&tempty[a]), 16);  // every epilogue warp of the pair
     }
     mbar_init(smem_addr(drain), 1);
     *sAbort = 0;
@@ -344,25 +367,27 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   if (warp == 0 && lane == 0) tma_prefetch_map(&tmap_w);
   if (warp == 1) {
-    tmem_alloc(smem_addr(sTmem), kTmemCols);
-    tmem_relinquish();
+    tmem_alloc_pair(smem_addr(sTmem), kTmemCols);
+    tmem_relinquish_pair();
   }
   __syncthreads();
+  cluster_sync();  // the leader's barriers exist before any remote arrival
   tc_fence_after_sync();
   const uint32_t tmem_base = *sTmem;
 
   const int U = *P.n_distinct;
-  const int m_tiles = (U + kBM - 1) / kBM;
+  const int m_tiles = (U + kPairRows - 1) / kPairRows;
   const int tiles_per_lc = m_tiles * P.n_tiles_n;
   const int total_tiles = 2 * P.L_r * tiles_per_lc;
 
   if (warp == 0) {
     // ------------------------------------------------------------ map tiles
+    // this CTA's half of the B tile: receiver columns n0 + rank*BN/2 .. +BN/2
     if (lane == 0) {
       int stage = 0;
       uint32_t phase = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; tile < total_tiles && ok; tile += gridDim.x) {
+      for (int tile = first_tile; tile < total_tiles && ok; tile += tile_step) {
         int lc, m, n;
         decode_tile(tile, tiles_per_lc, P.n_tiles_n, P.L_r, &lc, &m, &n);
         for (int kb = 0; kb < P.n_kb; ++kb) {
@@ -371,10 +396,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             ok = false;
             break;
           }
-          const uint32_t fb = smem_addr(&full_b[stage]);
-          mbar_arrive_expect_tx(fb, stage_b_bytes);
-          tma_load_2d(smem_addr(sB + stage * stage_b_bytes), &tmap_w, kb * kBK,
-                      lc * P.d_r + n * P.BN, fb);
+          const uint32_t fb = mapa_shared(smem_addr(&full_b[stage]), 0);
+          mbar_arrive_expect_tx_cluster(fb, stage_b_bytes);
+          tma_load_2d_pair(smem_addr(sB + stage * stage_b_bytes), &tmap_w, kb * kBK,
+                           lc * P.d_r + n * P.BN + static_cast<int>(rank) * half_bn, fb);
           if (++stage == stages_b) {
             stage = 0;
             phase ^= 1;
@@ -385,13 +410,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issue
-    if (lane == 0) {
+    if (lane == 0 && leader) {
       int sa = 0, sb = 0;
       uint32_t pa = 0, pb = 0;
       int acc = 0;
       uint32_t acc_phase = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; tile < total_tiles && ok; tile += gridDim.x) {
+      for (int tile = first_tile; tile < total_tiles && ok; tile += tile_step) {
         if (!mbar_wait(smem_addr(&tempty[acc]), acc_phase ^ 1)) {
           raise_timeout(P, sAbort);
           break;
@@ -412,12 +437,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint64_t ad = sw128_kmajor_desc(a0 + 32 * k);
             const uint64_t bd = sw128_kmajor_desc(b0 + 32 * k);
             if (sizeof(T) == 2)
-              mma_bf16(d_tmem, ad, bd, P.idesc, (kb | k) != 0);
+              mma_bf16_pair(d_tmem, ad, bd, P.idesc, (kb | k) != 0);
             else
-              mma_tf32(d_tmem, ad, bd, P.idesc, (kb | k) != 0);
+              mma_tf32_pair(d_tmem, ad, bd, P.idesc, (kb | k) != 0);
           }
-          tc_commit(smem_addr(&empty_a[sa]));
-          tc_commit(smem_addr(&empty_b[sb]));
+          tc_commit_pair(smem_addr(&empty_a[sa]), 0x3);
+          tc_commit_pair(smem_addr(&empty_b[sb]), 0x3);
           if (++sa == stages_a) {
             sa = 0;
             pa ^= 1;
@@ -428,21 +453,24 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
         if (!ok) break;
-        tc_commit(smem_addr(&tfull[acc]));
+        tc_commit_pair(smem_addr(&tfull[acc]), 0x3);
         acc ^= 1;
         if (acc == 0) acc_phase ^= 1;
       }
       // every issued MMA has completed before TMEM is released
-      tc_commit(smem_addr(drain));
+      tc_commit_pair(smem_addr(drain), 0x3);
+    }
+    if (lane == 0) {
       if (!mbar_wait(smem_addr(drain), 0)) raise_timeout(P, sAbort);
     }
     __syncwarp();
   } else if (warp < 10) {
     // ------------------------------------------------------------ epilogue
-    // Eight warps.  Step 1 (per 16 rotation pairs of a head pair): warp
-    // (g, sp) reads TMEM lane quarter sp of head 2*hp+g, applies 1/r, bias
-    // and key norm, and stages fp32 rows in smem.  Step 2: the eight warps
-    // split the tile's receiver rows and write both heads, rotated.
+    // Eight warps per CTA, for the CTA's 128 rows of the pair tile.  Step 1
+    // (per 16 rotation pairs of a head pair): warp (g, sp) reads TMEM lane
+    // quarter sp of head 2*hp+g, applies 1/r, bias and key norm, and stages
+    // fp32 rows in smem.  Step 2: the eight warps split the rows' receiver
+    // positions and write both heads, rotated.
     const int e = warp - 2;   // 0..7: slice of the tile's receiver rows
     const int g = e >> 2;     // head of the pair this warp stages
     const int sp = warp & 3;  // TMEM lane quarter this warp may access
@@ -455,7 +483,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int ps = lane >> 2, qq = lane & 3;  // row slot 0..7, pair quad 0..3
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int tile = blockIdx.x; tile < total_tiles; tile += gridDim.x) {
+    for (int tile = first_tile; tile < total_tiles; tile += tile_step) {
       int lc, m, n;
       decode_tile(tile, tiles_per_lc, P.n_tiles_n, P.L_r, &lc, &m, &n);
       const int c = lc & 1;
@@ -464,135 +492,137 @@ __global__ void __launch_bounds__(kThreads, 1)
         break;
       }
       tc_fence_after_sync();
-      const int u0 = m * kBM;
-      const int nrows = min(kBM, U - u0);
-      for (int i = tid_e; i <= nrows; i += 256) {
-        sRun[i] = P.run_ptr[u0 + i];
-        sUpos[i] = i < nrows ? P.upos[u0 + i] : 0;
-      }
-      named_barrier_sync(1, 256);
-      // this warp's receiver rows [wjb, wje); lane slot ps takes rows wjb+ps, +8, ...
-      const int jb = sRun[0], je = sRun[nrows];
-      const int per = (je - jb + 7) >> 3;
-      const int wjb = min(je, jb + e * per), wje = min(je, wjb + per);
-      const int n_it = (wje - wjb + 7) >> 3;
-      const int j0 = wjb + ps;
-      const int ustart = j0 < wje ? find_row(sRun, nrows, j0) : 0;
-      const float inv_r = P.inv_r[lc];
-      const float* bias = P.bias + static_cast<int64_t>(lc) * P.d_r;
-      const bool do_rope = P.rope && c == 0;
-      const bool do_knorm = P.knorm && c == 0;
-      const uint32_t ta = tmem_base + static_cast<uint32_t>(acc * 256) +
-                          (static_cast<uint32_t>(sp * 32) << 16);
-      T* const out_lc = reinterpret_cast<T*>(P.receiver) +
-                        (static_cast<int64_t>(lc) * P.recv_rows) * P.d_r;
-      for (int hp = 0; hp < n_pairs; ++hp) {
-        const bool stages_head = g == 0 || two_heads;
-        const int tcol = (2 * hp + g) * D;           // accumulator column of this warp's head
-        const int ocol_pair = n * P.BN + 2 * hp * D;  // receiver feature of the pair's first head
-        float rn = 1.0f;
-        if (do_knorm && stages_head) {
-          float ss = 0.0f;
-          for (int q2 = 0; q2 < D; q2 += 16) {
-            uint32_t v[16];
-            tmem_load_16(ta + tcol + q2, v);
-#pragma unroll
-            for (int i = 0; i < 16; ++i) {
-              const float y = fmaf(__uint_as_float(v[i]), inv_r,
-                                   __ldg(bias + n * P.BN + tcol + q2 + i));
-              ss = fmaf(y, y, ss);
-            }
-          }
-          rn = rsqrtf(ss / static_cast<float>(D) + P.knorm_eps);
+      const int u0 = m * kPairRows + row0;
+      const int nrows = min(kBM, U - u0);  // <= 0: this CTA has no rows in the tile
+      if (nrows > 0) {
+        for (int i = tid_e; i <= nrows; i += 256) {
+          sRun[i] = P.run_ptr[u0 + i];
+          sUpos[i] = i < nrows ? P.upos[u0 + i] : 0;
         }
-        for (int q = 0; q < half; q += 16) {
-          if (stages_head) {
-            // step 1: pairs q..q+15 of head 2*hp+g for this warp's 32 rows
-            uint32_t v[32];
-            tmem_load_2x16(ta + tcol + q, ta + tcol + half + q, v);
-            const float* bcol = bias + n * P.BN + tcol;
-            float y[32];
-#pragma unroll
-            for (int i = 0; i < 16; i += 4) {
-              const float4 x = __ldg(reinterpret_cast<const float4*>(bcol + q + i));
-              const float4 z = __ldg(reinterpret_cast<const float4*>(bcol + half + q + i));
-              y[i] = fmaf(__uint_as_float(v[i]), inv_r, x.x);
-              y[i + 1] = fmaf(__uint_as_float(v[i + 1]), inv_r, x.y);
-              y[i + 2] = fmaf(__uint_as_float(v[i + 2]), inv_r, x.z);
-              y[i + 3] = fmaf(__uint_as_float(v[i + 3]), inv_r, x.w);
-              y[16 + i] = fmaf(__uint_as_float(v[16 + i]), inv_r, z.x);
-              y[16 + i + 1] = fmaf(__uint_as_float(v[16 + i + 1]), inv_r, z.y);
-              y[16 + i + 2] = fmaf(__uint_as_float(v[16 + i + 2]), inv_r, z.z);
-              y[16 + i + 3] = fmaf(__uint_as_float(v[16 + i + 3]), inv_r, z.w);
-            }
-            if (do_knorm) {
+        named_barrier_sync(1, 256);
+        // this warp's receiver rows [wjb, wje); lane slot ps takes rows wjb+ps, +8, ...
+        const int jb = sRun[0], je = sRun[nrows];
+        const int per = (je - jb + 7) >> 3;
+        const int wjb = min(je, jb + e * per), wje = min(je, wjb + per);
+        const int n_it = (wje - wjb + 7) >> 3;
+        const int j0 = wjb + ps;
+        const int ustart = j0 < wje ? find_row(sRun, nrows, j0) : 0;
+        const float inv_r = P.inv_r[lc];
+        const float* bias = P.bias + static_cast<int64_t>(lc) * P.d_r;
+        const bool do_rope = P.rope && c == 0;
+        const bool do_knorm = P.knorm && c == 0;
+        const uint32_t ta = tmem_base + static_cast<uint32_t>(acc * 256) +
+                            (static_cast<uint32_t>(sp * 32) << 16);
+        T* const out_lc = reinterpret_cast<T*>(P.receiver) +
+                          (static_cast<int64_t>(lc) * P.recv_rows) * P.d_r;
+        for (int hp = 0; hp < n_pairs; ++hp) {
+          const bool stages_head = g == 0 || two_heads;
+          const int tcol = (2 * hp + g) * D;            // accumulator column of this warp's head
+          const int ocol_pair = n * P.BN + 2 * hp * D;  // receiver feature of the pair's first head
+          float rn = 1.0f;
+          if (do_knorm && stages_head) {
+            float ss = 0.0f;
+            for (int q2 = 0; q2 < D; q2 += 16) {
+              uint32_t v[16];
+              tmem_load_16(ta + tcol + q2, v);
 #pragma unroll
               for (int i = 0; i < 16; ++i) {
-                y[i] *= rn * __ldg(P.knorm_w + q + i);
-                y[16 + i] *= rn * __ldg(P.knorm_w + half + q + i);
+                const float y = fmaf(__uint_as_float(v[i]), inv_r,
+                                     __ldg(bias + n * P.BN + tcol + q2 + i));
+                ss = fmaf(y, y, ss);
               }
             }
-            float* srow = sStg + row * 64 + g * 32;
+            rn = rsqrtf(ss / static_cast<float>(D) + P.knorm_eps);
+          }
+          for (int q = 0; q < half; q += 16) {
+            if (stages_head) {
+              // step 1: pairs q..q+15 of head 2*hp+g for this warp's 32 rows
+              uint32_t v[32];
+              tmem_load_2x16(ta + tcol + q, ta + tcol + half + q, v);
+              const float* bcol = bias + n * P.BN + tcol;
+              float y[32];
 #pragma unroll
-            for (int k = 0; k < 8; ++k)
-              *reinterpret_cast<float4*>(srow + ((k ^ (row & 7)) << 2)) =
-                  make_float4(y[4 * k], y[4 * k + 1], y[4 * k + 2], y[4 * k + 3]);
-          }
-          named_barrier_sync(1, 256);
-          // step 2: rows of this warp's slice, both heads of the pair
-          float f[4], C8[4], S8[4];
+              for (int i = 0; i < 16; i += 4) {
+                const float4 x = __ldg(reinterpret_cast<const float4*>(bcol + q + i));
+                const float4 z = __ldg(reinterpret_cast<const float4*>(bcol + half + q + i));
+                y[i] = fmaf(__uint_as_float(v[i]), inv_r, x.x);
+                y[i + 1] = fmaf(__uint_as_float(v[i + 1]), inv_r, x.y);
+                y[i + 2] = fmaf(__uint_as_float(v[i + 2]), inv_r, x.z);
+                y[i + 3] = fmaf(__uint_as_float(v[i + 3]), inv_r, x.w);
+                y[16 + i] = fmaf(__uint_as_float(v[16 + i]), inv_r, z.x);
+                y[16 + i + 1] = fmaf(__uint_as_float(v[16 + i + 1]), inv_r, z.y);
+                y[16 + i + 2] = fmaf(__uint_as_float(v[16 + i + 2]), inv_r, z.z);
+                y[16 + i + 3] = fmaf(__uint_as_float(v[16 + i + 3]), inv_r, z.w);
+              }
+              if (do_knorm) {
 #pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            f[k] = do_rope ? __ldg(P.inv_freq + q + 4 * qq + k) : 0.f;
-            C8[k] = 1.f;
-            S8[k] = 0.f;
-            if (do_rope) rope_sincos(8, f[k], &S8[k], &C8[k]);  // one step = eight rows
-          }
-          Walk wk;
-          wk.u = ustart;
-          wk.expect = INT_MIN;
+                for (int i = 0; i < 16; ++i) {
+                  y[i] *= rn * __ldg(P.knorm_w + q + i);
+                  y[16 + i] *= rn * __ldg(P.knorm_w + half + q + i);
+                }
+              }
+              float* srow = sStg + row * 64 + g * 32;
 #pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            wk.cs[k] = 1.f;
-            wk.sn[k] = 0.f;
+              for (int k = 0; k < 8; ++k)
+                *reinterpret_cast<float4*>(srow + ((k ^ (row & 7)) << 2)) =
+                    make_float4(y[4 * k], y[4 * k + 1], y[4 * k + 2], y[4 * k + 3]);
+            }
+            named_barrier_sync(1, 256);
+            // step 2: rows of this warp's slice, both heads of the pair
+            float f[4], C8[4], S8[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              f[k] = do_rope ? __ldg(P.inv_freq + q + 4 * qq + k) : 0.f;
+              C8[k] = 1.f;
+              S8[k] = 0.f;
+              if (do_rope) rope_sincos(8, f[k], &S8[k], &C8[k]);  // one step = eight rows
+            }
+            Walk wk;
+            wk.u = ustart;
+            wk.expect = INT_MIN;
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              wk.cs[k] = 1.f;
+              wk.sn[k] = 0.f;
+            }
+            for (int it = 0; it < n_it; ++it) {
+              const int j = j0 + 8 * it;
+              if (j < wje)
+                walk_step<T>(wk, j, it, sRun, sUpos, sStg, qq, two_heads, do_rope, f, C8, S8, P,
+                             out_lc, ocol_pair, q, half);
+            }
+            named_barrier_sync(1, 256);
           }
-          for (int it = 0; it < n_it; ++it) {
-            const int j = j0 + 8 * it;
-            if (j < wje)
-              walk_step<T>(wk, j, it, sRun, sUpos, sStg, qq, two_heads, do_rope, f, C8, S8, P,
-                           out_lc, ocol_pair, q, half);
-          }
-          named_barrier_sync(1, 256);
         }
       }
       tc_fence_before_sync();
       __syncwarp();
-      if (lane == 0) mbar_arrive(smem_addr(&tempty[acc]));
+      if (lane == 0) arrive_leader(smem_addr(&tempty[acc]), row0);
       acc ^= 1;
       if (acc == 0) acc_phase ^= 1;
     }
   } else {
     // ------------------------------------------------------------ A builders
     const int t = threadIdx.x - 320;  // 0..127
-    const T* sender = reinterpret_cast<const T*>(P.sender);
-    int stage = 0;
-    uint32_t phase = 0;
-    bool ok = true;
     if (kGather) {
       switch (P.lag) {
-        case 2: gather_rows<T, 2>(P, sA, full_a, empty_a, sAbort, t, lane, U, total_tiles, tiles_per_lc); break;
-        case 3: gather_rows<T, 3>(P, sA, full_a, empty_a, sAbort, t, lane, U, total_tiles, tiles_per_lc); break;
-        case 4: gather_rows<T, 4>(P, sA, full_a, empty_a, sAbort, t, lane, U, total_tiles, tiles_per_lc); break;
-        default: gather_rows<T, 5>(P, sA, full_a, empty_a, sAbort, t, lane, U, total_tiles, tiles_per_lc); break;
+        case 2: gather_rows<T, 2>(P, sA, full_a, empty_a, sAbort, t, lane, U, row0, total_tiles, tiles_per_lc, first_tile, tile_step); break;
+        case 3: gather_rows<T, 3>(P, sA, full_a, empty_a, sAbort, t, lane, U, row0, total_tiles, tiles_per_lc, first_tile, tile_step); break;
+        case 4: gather_rows<T, 4>(P, sA, full_a, empty_a, sAbort, t, lane, U, row0, total_tiles, tiles_per_lc, first_tile, tile_step); break;
+        default: gather_rows<T, 5>(P, sA, full_a, empty_a, sAbort, t, lane, U, row0, total_tiles, tiles_per_lc, first_tile, tile_step); break;
       }
     } else {
       // pooled CSR rows and/or blended sender layers: thread t owns tile row t
-      for (int tile = blockIdx.x; tile < total_tiles && ok; tile += gridDim.x) {
+      const T* sender = reinterpret_cast<const T*>(P.sender);
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      for (int tile = first_tile; tile < total_tiles && ok; tile += tile_step) {
         int lc, m, n;
         decode_tile(tile, tiles_per_lc, P.n_tiles_n, P.L_r, &lc, &m, &n);
         const int l = lc >> 1, c = lc & 1;
         const LayerSegs segs = P.segs[l];
-        const int u = min(m * kBM + t, U - 1);
+        const int u = min(m * kPairRows + row0 + t, U - 1);
         const int j0 = P.run_ptr[u];
         const int e0 = P.row_ptr[j0], e1 = P.row_ptr[j0 + 1];
         for (int kb = 0; kb < P.n_kb; ++kb) {
@@ -630,7 +660,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             *reinterpret_cast<uint4*>(dst + ((k2 ^ (t & 7)) << 4)) =
                 pack16(acc + k2 * kPerChunk, (const T*)nullptr);
           fence_proxy_async_smem();
-          mbar_arrive(smem_addr(&full_a[stage]));
+          __syncwarp();
+          if (lane == 0) arrive_leader(smem_addr(&full_a[stage]), row0);
           if (++stage == stages_a) {
             stage = 0;
             phase ^= 1;
@@ -647,9 +678,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     while (global_timer_ns() - t0 < 200000ull) {
     }
   }
+  cluster_sync();  // neither CTA leaves while the pair's MMAs or arrivals may touch it
   if (warp == 1) {
     tc_fence_after_sync();
-    tmem_dealloc(tmem_base, kTmemCols);
+    tmem_dealloc_pair(tmem_base, kTmemCols);
   }
 }
 
@@ -699,19 +731,19 @@ hf_status make_map(CUtensorMap* map, const void* base, bool f32, uint64_t rows, 
 }
 
 size_t smem_bytes(int BN, int stages_a, int stages_b) {
-  return static_cast<size_t>(stages_a) * kStageABytes + static_cast<size_t>(stages_b) * BN * 128 +
-         kStgFloats * sizeof(float) + 2 * kRunStride * sizeof(int32_t) +
-         (4 * kMaxStages + 5) * sizeof(uint64_t) + 8;
+  return static_cast<size_t>(stages_a) * kStageABytes +
+         static_cast<size_t>(stages_b) * (BN / 2) * 128 + kStgFloats * sizeof(float) +
+         2 * kRunStride * sizeof(int32_t) + (4 * kMaxStages + 5) * sizeof(uint64_t) + 8;
 }
 
-// Ring depths: as many A stages as fit next to `stages_b` B stages, with
-// the loaders keeping all but two A stages in flight (so the tensor core
-// always has two k-blocks queued).
+// Ring depths: as many A stages as fit next to four B stages, with the
+// loaders keeping all but two A stages in flight (so the tensor core always
+// has two k-blocks queued).
 void pick_rings(int BN, int* stages_a, int* stages_b, int* lag) {
   int dev = 0, optin = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
-  int sb = BN == 256 ? 3 : 4;
+  const int sb = 4;
   int sa = kMaxStages;
   while (sa > 4 && smem_bytes(BN, sa, sb) > static_cast<size_t>(optin)) --sa;
   *stages_a = sa;
@@ -720,14 +752,32 @@ void pick_rings(int BN, int* stages_a, int* stages_b, int* lag) {
 }
 
 template <typename T, bool kGather>
-hf_status launch_typed(const CUtensorMap& mw, const XferParams& P, int grid, size_t smem,
-                       cudaStream_t stream) {
+hf_status launch_typed(const CUtensorMap& mw, const XferParams& P, int64_t max_pair_tiles,
+                       size_t smem, cudaStream_t stream) {
   auto kern = transfer_kernel<T, kGather>;
   HF_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                    static_cast<int>(smem)),
               "set shared memory size");
-  kern<<<grid, kThreads, smem, stream>>>(mw, P);
-  HF_CUDA_TRY(cudaGetLastError(), "transfer kernel launch");
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  // one CTA pair per co-resident cluster slot, at most one per pair tile
+  int clusters = device_sm_count() / 2;
+  cfg.gridDim = dim3(2 * clusters, 1, 1);
+  int active = 0;
+  if (cudaOccupancyMaxActiveClusters(&active, kern, &cfg) == cudaSuccess && active > 0)
+    clusters = std::min(clusters, active);
+  clusters = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(clusters, max_pair_tiles)));
+  cfg.gridDim = dim3(2 * clusters, 1, 1);
+  HF_CUDA_TRY(cudaLaunchKernelEx(&cfg, kern, mw, P), "transfer kernel launch");
   return HF_OK;
 }
 
@@ -741,7 +791,7 @@ hf_status launch_transfer(hf_plan_s* p, const void* sender, void* receiver, cuda
   const int bk = 128 / esize;
   CUtensorMap mw;
   hf_status s = make_map(&mw, d.d_W, f32, static_cast<uint64_t>(d.L_r) * 2 * p->d_r,
-                         static_cast<uint64_t>(p->K), static_cast<uint32_t>(p->BN),
+                         static_cast<uint64_t>(p->K), static_cast<uint32_t>(p->BN / 2),
                          static_cast<uint32_t>(bk), CU_TENSOR_MAP_L2_PROMOTION_L2_256B);
   if (s != HF_OK) return s;
   XferParams P;
@@ -773,22 +823,20 @@ hf_status launch_transfer(hf_plan_s* p, const void* sender, void* receiver, cuda
   P.kb_per_seg = p->d_s / bk;
   P.BN = p->BN;
   P.n_tiles_n = p->d_r / p->BN;
-  P.groups = p->groups;
   pick_rings(p->BN, &P.stages_a, &P.stages_b, &P.lag);
   P.rope = d.theta_r > 0.0 ? 1 : 0;
   P.paged = d.paged ? 1 : 0;
   P.knorm = d.d_knorm_w ? 1 : 0;
   P.knorm_eps = d.knorm_eps;
-  P.idesc = make_idesc(f32 ? 2u : 1u, kBM, p->BN);
+  P.idesc = make_idesc(f32 ? 2u : 1u, kPairRows, p->BN);
   const size_t smem = smem_bytes(p->BN, P.stages_a, P.stages_b);
-  const int64_t max_tiles =
-      2LL * d.L_r * ((p->T_r + kBM - 1) / kBM) * static_cast<int64_t>(P.n_tiles_n);
-  const int grid = static_cast<int>(std::min<int64_t>(device_sm_count(), max_tiles));
+  const int64_t max_pair_tiles =
+      2LL * d.L_r * ((p->T_r + kPairRows - 1) / kPairRows) * static_cast<int64_t>(P.n_tiles_n);
   if (f32)
-    return p->gather ? launch_typed<float, true>(mw, P, grid, smem, stream)
-                     : launch_typed<float, false>(mw, P, grid, smem, stream);
-  return p->gather ? launch_typed<__nv_bfloat16, true>(mw, P, grid, smem, stream)
-                   : launch_typed<__nv_bfloat16, false>(mw, P, grid, smem, stream);
+    return p->gather ? launch_typed<float, true>(mw, P, max_pair_tiles, smem, stream)
+                     : launch_typed<float, false>(mw, P, max_pair_tiles, smem, stream);
+  return p->gather ? launch_typed<__nv_bfloat16, true>(mw, P, max_pair_tiles, smem, stream)
+                   : launch_typed<__nv_bfloat16, false>(mw, P, max_pair_tiles, smem, stream);
 }
 
 }  // namespace hf
