@@ -411,6 +411,17 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issue
     if (lane == 0 && leader) {
+      // This single thread shares its scheduler with busy epilogue and
+      // builder warps, so the loop keeps its instruction count low: barrier
+      // addresses and descriptors advance by adds (a descriptor's start
+      // address field is the smem byte address >> 4; it cannot carry out for
+      // addresses below 256 KB).
+      const uint32_t full_a0 = smem_addr(full_a), empty_a0 = smem_addr(empty_a);
+      const uint32_t full_b0 = smem_addr(full_b), empty_b0 = smem_addr(empty_b);
+      const uint64_t desc_a0 = sw128_kmajor_desc(smem_addr(sA));
+      const uint64_t desc_b0 = sw128_kmajor_desc(smem_addr(sB));
+      const uint32_t step_a = kStageABytes >> 4, step_b = static_cast<uint32_t>(stage_b_bytes) >> 4;
+      const uint32_t idesc = P.idesc;
       int sa = 0, sb = 0;
       uint32_t pa = 0, pb = 0;
       int acc = 0;
@@ -423,26 +434,31 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tc_fence_after_sync();
         const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * 256);
+        uint32_t accumulate = 0;
         for (int kb = 0; kb < P.n_kb; ++kb) {
-          if (!mbar_wait(smem_addr(&full_a[sa]), pa) || !mbar_wait(smem_addr(&full_b[sb]), pb)) {
+          if (!mbar_wait(full_a0 + 8 * sa, pa) || !mbar_wait(full_b0 + 8 * sb, pb)) {
             raise_timeout(P, sAbort);
             ok = false;
             break;
           }
           tc_fence_after_sync();
-          const uint32_t a0 = smem_addr(sA + sa * kStageABytes);
-          const uint32_t b0 = smem_addr(sB + sb * stage_b_bytes);
-#pragma unroll
-          for (int k = 0; k < 4; ++k) {  // four 32-byte K steps per 128-byte k-block
-            const uint64_t ad = sw128_kmajor_desc(a0 + 32 * k);
-            const uint64_t bd = sw128_kmajor_desc(b0 + 32 * k);
-            if (sizeof(T) == 2)
-              mma_bf16_pair(d_tmem, ad, bd, P.idesc, (kb | k) != 0);
-            else
-              mma_tf32_pair(d_tmem, ad, bd, P.idesc, (kb | k) != 0);
+          const uint64_t ad = desc_a0 + sa * step_a;
+          const uint64_t bd = desc_b0 + sb * step_b;
+          // four 32-byte K steps per 128-byte k-block (descriptor units of 16 bytes)
+          if (sizeof(T) == 2) {
+            mma_bf16_pair(d_tmem, ad, bd, idesc, accumulate);
+            mma_bf16_pair(d_tmem, ad + 2, bd + 2, idesc, 1);
+            mma_bf16_pair(d_tmem, ad + 4, bd + 4, idesc, 1);
+            mma_bf16_pair(d_tmem, ad + 6, bd + 6, idesc, 1);
+          } else {
+            mma_tf32_pair(d_tmem, ad, bd, idesc, accumulate);
+            mma_tf32_pair(d_tmem, ad + 2, bd + 2, idesc, 1);
+            mma_tf32_pair(d_tmem, ad + 4, bd + 4, idesc, 1);
+            mma_tf32_pair(d_tmem, ad + 6, bd + 6, idesc, 1);
           }
-          tc_commit_pair(smem_addr(&empty_a[sa]), 0x3);
-          tc_commit_pair(smem_addr(&empty_b[sb]), 0x3);
+          accumulate = 1;
+          tc_commit_pair(empty_a0 + 8 * sa, 0x3);
+          tc_commit_pair(empty_b0 + 8 * sb, 0x3);
           if (++sa == stages_a) {
             sa = 0;
             pa ^= 1;
