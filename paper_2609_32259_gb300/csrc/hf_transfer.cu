@@ -45,7 +45,9 @@ constexpr int kBM = 128;                 // distinct rows per CTA of a pair tile
 constexpr int kPairRows = 2 * kBM;       // distinct rows per pair tile (UMMA M = 256)
 constexpr int kThreads = 448;            // 14 warps
 constexpr int kBuilderWarps = 4;         // A tile builders: warps 10-13
-constexpr int kStageABytes = kBM * 128;  // 128 rows x 128 bytes
+constexpr int kAtoms = 2;                // 128-byte swizzle atoms (k-blocks) per pipeline stage
+constexpr int kAtomABytes = kBM * 128;   // 128 rows x 128 bytes
+constexpr int kStageABytes = kAtoms * kAtomABytes;
 constexpr int kStgFloats = kBM * 64;     // epilogue staging: 128 rows x 2 heads x 32
 constexpr int kRunStride = 132;          // run starts / positions of a tile (129 used)
 constexpr int kMaxStages = 8;
@@ -71,7 +73,7 @@ struct XferParams {
   int64_t T_s;        // sender rows per (layer, role)
   int64_t recv_rows;  // receiver rows per (layer, role) in receiver_kv
   int L_r, d_s, d_r, D_r;
-  int n_kb, kb_per_seg, BN, n_tiles_n, groups;
+  int n_kb, atoms_per_seg, last_atoms, BN, n_tiles_n, groups;  // n_kb: stages per tile
   int stages_a, stages_b, lag;  // A ring, B ring, cp.async groups in flight per loader
   int rope, paged, knorm;
   float knorm_eps;
@@ -273,19 +275,28 @@ __device__ __forceinline__ void gather_rows(const XferParams& P, uint8_t* sA, ui
       roff[i] = static_cast<int64_t>(P.ucol[u]) * P.d_s + ch * kPerChunk;
       doff[i] = static_cast<uint32_t>(r * 128 + ((ch ^ (r & 7)) << 4));
     }
+    int seg = 0, kin = 0;  // segment of the next atom, and the atom within it
     for (int kb = 0; kb < P.n_kb; ++kb) {
-      const int seg = kb / P.kb_per_seg;
-      const int kin = kb - seg * P.kb_per_seg;
       if (!mbar_wait(smem_addr(&empty_a[stage]), phase ^ 1)) {
         raise_timeout(P, sAbort);
         ok = false;
         break;
       }
-      const int64_t sbase = seg == 0 ? seg_base[0] : (seg == 1 ? seg_base[1] : seg_base[2]);
-      const T* base = sender + sbase + kin * kBK;
       const uint32_t sa = smem_addr(sA + stage * kStageABytes);
+      const int na = kb == P.n_kb - 1 ? P.last_atoms : kAtoms;
 #pragma unroll
-      for (int i = 0; i < 8; ++i) cp_async_16(sa + doff[i], base + roff[i]);
+      for (int a = 0; a < kAtoms; ++a) {
+        if (a < na) {
+          const int64_t sbase = seg == 0 ? seg_base[0] : (seg == 1 ? seg_base[1] : seg_base[2]);
+          const T* base = sender + sbase + kin * kBK;
+#pragma unroll
+          for (int i = 0; i < 8; ++i) cp_async_16(sa + a * kAtomABytes + doff[i], base + roff[i]);
+          if (++kin == P.atoms_per_seg) {
+            kin = 0;
+            ++seg;
+          }
+        }
+      }
       cp_async_commit();
       if (pending == LAG) {
         cp_async_wait<LAG>();
@@ -326,7 +337,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int row0 = static_cast<int>(rank) * kBM;  // this CTA's rows within a pair tile
   const int stages_a = P.stages_a, stages_b = P.stages_b;
   const int half_bn = P.BN / 2;                    // B rows (receiver columns) per CTA
-  const int stage_b_bytes = half_bn * 128;
+  const int atom_b_bytes = half_bn * 128;
+  const int stage_b_bytes = kAtoms * atom_b_bytes;
   uint8_t* sA = smem;
   uint8_t* sB = sA + stages_a * kStageABytes;
   float* sStg = reinterpret_cast<float*>(sB + stages_b * stage_b_bytes);
@@ -397,9 +409,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             break;
           }
           const uint32_t fb = mapa_shared(smem_addr(&full_b[stage]), 0);
-          mbar_arrive_expect_tx_cluster(fb, stage_b_bytes);
-          tma_load_2d_pair(smem_addr(sB + stage * stage_b_bytes), &tmap_w, kb * kBK,
-                           lc * P.d_r + n * P.BN + static_cast<int>(rank) * half_bn, fb);
+          const int na = kb == P.n_kb - 1 ? P.last_atoms : kAtoms;
+          mbar_arrive_expect_tx_cluster(fb, na * atom_b_bytes);
+#pragma unroll
+          for (int a = 0; a < kAtoms; ++a)
+            if (a < na)
+              tma_load_2d_pair(smem_addr(sB + stage * stage_b_bytes + a * atom_b_bytes), &tmap_w,
+                               (kb * kAtoms + a) * kBK,
+                               lc * P.d_r + n * P.BN + static_cast<int>(rank) * half_bn, fb);
           if (++stage == stages_b) {
             stage = 0;
             phase ^= 1;
@@ -421,7 +438,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint64_t desc_a0 = sw128_kmajor_desc(smem_addr(sA));
       const uint64_t desc_b0 = sw128_kmajor_desc(smem_addr(sB));
       const uint32_t step_a = kStageABytes >> 4, step_b = static_cast<uint32_t>(stage_b_bytes) >> 4;
+      const uint32_t atom_a = kAtomABytes >> 4, atom_b = static_cast<uint32_t>(atom_b_bytes) >> 4;
       const uint32_t idesc = P.idesc;
+      const int n_kb = P.n_kb, last_atoms = P.last_atoms;
       int sa = 0, sb = 0;
       uint32_t pa = 0, pb = 0;
       int acc = 0;
@@ -435,28 +454,33 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_after_sync();
         const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * 256);
         uint32_t accumulate = 0;
-        for (int kb = 0; kb < P.n_kb; ++kb) {
+        for (int kb = 0; kb < n_kb; ++kb) {
           if (!mbar_wait(full_a0 + 8 * sa, pa) || !mbar_wait(full_b0 + 8 * sb, pb)) {
             raise_timeout(P, sAbort);
             ok = false;
             break;
           }
           tc_fence_after_sync();
-          const uint64_t ad = desc_a0 + sa * step_a;
-          const uint64_t bd = desc_b0 + sb * step_b;
-          // four 32-byte K steps per 128-byte k-block (descriptor units of 16 bytes)
-          if (sizeof(T) == 2) {
-            mma_bf16_pair(d_tmem, ad, bd, idesc, accumulate);
-            mma_bf16_pair(d_tmem, ad + 2, bd + 2, idesc, 1);
-            mma_bf16_pair(d_tmem, ad + 4, bd + 4, idesc, 1);
-            mma_bf16_pair(d_tmem, ad + 6, bd + 6, idesc, 1);
-          } else {
-            mma_tf32_pair(d_tmem, ad, bd, idesc, accumulate);
-            mma_tf32_pair(d_tmem, ad + 2, bd + 2, idesc, 1);
-            mma_tf32_pair(d_tmem, ad + 4, bd + 4, idesc, 1);
-            mma_tf32_pair(d_tmem, ad + 6, bd + 6, idesc, 1);
+          const int na = kb == n_kb - 1 ? last_atoms : kAtoms;
+#pragma unroll
+          for (int a = 0; a < kAtoms; ++a) {
+            if (a >= na) break;
+            const uint64_t ad = desc_a0 + sa * step_a + a * atom_a;
+            const uint64_t bd = desc_b0 + sb * step_b + a * atom_b;
+            // four 32-byte K steps per 128-byte atom (descriptor units of 16 bytes)
+            if (sizeof(T) == 2) {
+              mma_bf16_pair(d_tmem, ad, bd, idesc, accumulate);
+              mma_bf16_pair(d_tmem, ad + 2, bd + 2, idesc, 1);
+              mma_bf16_pair(d_tmem, ad + 4, bd + 4, idesc, 1);
+              mma_bf16_pair(d_tmem, ad + 6, bd + 6, idesc, 1);
+            } else {
+              mma_tf32_pair(d_tmem, ad, bd, idesc, accumulate);
+              mma_tf32_pair(d_tmem, ad + 2, bd + 2, idesc, 1);
+              mma_tf32_pair(d_tmem, ad + 4, bd + 4, idesc, 1);
+              mma_tf32_pair(d_tmem, ad + 6, bd + 6, idesc, 1);
+            }
+            accumulate = 1;
           }
-          accumulate = 1;
           tc_commit_pair(empty_a0 + 8 * sa, 0x3);
           tc_commit_pair(empty_b0 + 8 * sb, 0x3);
           if (++sa == stages_a) {
@@ -622,6 +646,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int t = threadIdx.x - 320;  // 0..127
     if (kGather) {
       switch (P.lag) {
+        case 1: gather_rows<T, 1>(P, sA, full_a, empty_a, sAbort, t, lane, U, row0, total_tiles, tiles_per_lc, first_tile, tile_step); break;
         case 2: gather_rows<T, 2>(P, sA, full_a, empty_a, sAbort, t, lane, U, row0, total_tiles, tiles_per_lc, first_tile, tile_step); break;
         case 3: gather_rows<T, 3>(P, sA, full_a, empty_a, sAbort, t, lane, U, row0, total_tiles, tiles_per_lc, first_tile, tile_step); break;
         case 4: gather_rows<T, 4>(P, sA, full_a, empty_a, sAbort, t, lane, U, row0, total_tiles, tiles_per_lc, first_tile, tile_step); break;
@@ -641,21 +666,23 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int u = min(m * kPairRows + row0 + t, U - 1);
         const int j0 = P.run_ptr[u];
         const int e0 = P.row_ptr[j0], e1 = P.row_ptr[j0 + 1];
+        int seg = 0, kin = 0;  // segment of the next atom, and the atom within it
         for (int kb = 0; kb < P.n_kb; ++kb) {
-          const int seg = kb / P.kb_per_seg;
-          const int kin = kb - seg * P.kb_per_seg;
           if (!mbar_wait(smem_addr(&empty_a[stage]), phase ^ 1)) {
             raise_timeout(P, sAbort);
             ok = false;
             break;
           }
+          const int na = kb == P.n_kb - 1 ? P.last_atoms : kAtoms;
+          for (int a = 0; a < na; ++a) {
           float acc[kBK];
 #pragma unroll
           for (int i = 0; i < kBK; ++i) acc[i] = 0.f;
           for (int ti = 0; ti < segs.n_terms[seg]; ++ti) {
             const int tl = segs.layer[seg][ti];
             const float om = segs.w[seg][ti];
-            const T* base = sender + (static_cast<int64_t>(tl * 2 + c) * P.T_s) * P.d_s + kin * kBK;
+            const T* base =
+                sender + (static_cast<int64_t>(tl * 2 + c) * P.T_s) * P.d_s + kin * kBK;
             for (int e = e0; e < e1; ++e) {
               const int k = P.col[e];
               if (k < 0 || k >= P.T_s) continue;  // flagged at plan creation
@@ -670,11 +697,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                 accum16(x[k2], wt, acc + k2 * kPerChunk, (const T*)nullptr);
             }
           }
-          uint8_t* dst = sA + stage * kStageABytes + t * 128;
+          uint8_t* dst = sA + stage * kStageABytes + a * kAtomABytes + t * 128;
 #pragma unroll
           for (int k2 = 0; k2 < 8; ++k2)
             *reinterpret_cast<uint4*>(dst + ((k2 ^ (t & 7)) << 4)) =
                 pack16(acc + k2 * kPerChunk, (const T*)nullptr);
+          if (++kin == P.atoms_per_seg) {
+            kin = 0;
+            ++seg;
+          }
+          }
           fence_proxy_async_smem();
           __syncwarp();
           if (lane == 0) arrive_leader(smem_addr(&full_a[stage]), row0);
@@ -748,23 +780,25 @@ hf_status make_map(CUtensorMap* map, const void* base, bool f32, uint64_t rows, 
 
 size_t smem_bytes(int BN, int stages_a, int stages_b) {
   return static_cast<size_t>(stages_a) * kStageABytes +
-         static_cast<size_t>(stages_b) * (BN / 2) * 128 + kStgFloats * sizeof(float) +
+         static_cast<size_t>(stages_b) * kAtoms * (BN / 2) * 128 + kStgFloats * sizeof(float) +
          2 * kRunStride * sizeof(int32_t) + (4 * kMaxStages + 5) * sizeof(uint64_t) + 8;
 }
 
-// Ring depths: as many A stages as fit next to four B stages, with the
-// loaders keeping all but two A stages in flight (so the tensor core always
-// has two k-blocks queued).
+// Ring depths (stages of kAtoms k-blocks): three or four B stages, as many
+// A stages as fit next to them.  Each loader keeps two stages of copies in
+// flight (it waits for stage i-1 after issuing stage i), which at 32 KB per
+// stage covers the L2/HBM latency; deeper loader lag only takes stages away
+// from the tensor core.
 void pick_rings(int BN, int* stages_a, int* stages_b, int* lag) {
   int dev = 0, optin = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
-  const int sb = 4;
+  const int sb = BN == 256 ? 3 : 4;
   int sa = kMaxStages;
-  while (sa > 4 && smem_bytes(BN, sa, sb) > static_cast<size_t>(optin)) --sa;
+  while (sa > 2 && smem_bytes(BN, sa, sb) > static_cast<size_t>(optin)) --sa;
   *stages_a = sa;
   *stages_b = sb;
-  *lag = std::min(5, std::max(2, sa - 3));
+  *lag = 1;
 }
 
 template <typename T, bool kGather>
@@ -835,8 +869,10 @@ hf_status launch_transfer(hf_plan_s* p, const void* sender, void* receiver, cuda
   P.d_s = p->d_s;
   P.d_r = p->d_r;
   P.D_r = d.D_r;
-  P.n_kb = p->K / bk;
-  P.kb_per_seg = p->d_s / bk;
+  const int n_atoms = p->K / bk;  // 128-byte k-blocks per output row
+  P.n_kb = (n_atoms + kAtoms - 1) / kAtoms;
+  P.last_atoms = n_atoms - kAtoms * (P.n_kb - 1);
+  P.atoms_per_seg = p->d_s / bk;
   P.BN = p->BN;
   P.n_tiles_n = p->d_r / p->BN;
   pick_rings(p->BN, &P.stages_a, &P.stages_b, &P.lag);
