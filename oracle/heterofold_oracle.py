@@ -41,6 +41,11 @@ Conventions (readings of passages the paper leaves open):
   fp32 rounding of theta ** (-2 i / D) evaluated in double precision, and the
   angle p * inv_freq_i is formed exactly in fp64.
 * Key normalisation, when enabled, is a per-head RMS norm with a weight g[D].
+* Sender keys are normally captured before RoPE (Section 3 opening
+  paragraph).  For a sender cache whose keys already carry RoPE at the sender
+  positions, the keys are first rotated back (the inverse rotation, by the
+  negative angle, at each sender token's own position) and only then pooled
+  and blended; values are never rotated.
 
 Every routine here is a direct restatement of the definitions above in
 numpy float64; nothing is blocked, fused or reordered beyond them.
@@ -267,6 +272,17 @@ def layer_interpolation(L_s: int, L_r: int) -> List[List[Tuple[int, float]]]:
     return out
 
 
+def explicit_segments(seg_layer, seg_w) -> List[List[List[Tuple[int, float]]]]:
+    """A caller-given layer table: seg_layer[l][s][t] (zero-based sender
+    layer) and seg_w[l][s][t] give term t of segment s of receiver layer l.
+    Segment s is the weighted sum of its terms (the same structure as Eq. 2's
+    concatenation, with any layers and weights)."""
+    out = []
+    for layers_l, w_l in zip(seg_layer, seg_w):
+        out.append([[(int(t), float(w)) for t, w in zip(ts, ws)] for ts, ws in zip(layers_l, w_l)])
+    return out
+
+
 def layer_segments(mode: str, L_s: int, L_r: int) -> List[List[List[Tuple[int, float]]]]:
     """Per receiver layer: the K-segments of the map input, each a weighted
     sum of sender layers.  Paper mode: three one-layer segments (Eq. 2);
@@ -314,6 +330,19 @@ def rope(x: np.ndarray, pos: np.ndarray, inv_freq: np.ndarray) -> np.ndarray:
     return np.concatenate([x1 * c - x2 * s, x2 * c + x1 * s], axis=-1)
 
 
+def rope_inverse(x: np.ndarray, pos: np.ndarray, inv_freq: np.ndarray) -> np.ndarray:
+    """The inverse of rope() at the same positions: pair (i, i + D/2) is
+    rotated by the negative angle -pos * inv_freq_i.  x: [n, H, D]."""
+    D = x.shape[-1]
+    half = D // 2
+    ang = np.asarray(pos, dtype=np.float64)[:, None] * inv_freq[None, :]
+    c = np.cos(ang)[:, None, :]
+    s = np.sin(ang)[:, None, :]
+    x1 = x[..., :half]
+    x2 = x[..., half:]
+    return np.concatenate([x1 * c + x2 * s, x2 * c - x1 * s], axis=-1)
+
+
 def key_norm(x: np.ndarray, g: np.ndarray, eps: float) -> np.ndarray:
     """Per-head RMS normalisation of receiver keys with weight g[D]."""
     ms = np.mean(x * x, axis=-1, keepdims=True)
@@ -324,32 +353,45 @@ def key_norm(x: np.ndarray, g: np.ndarray, eps: float) -> np.ndarray:
 # The transfer (Eq. 2 + Eq. 9)
 # ---------------------------------------------------------------------------
 
-def pooled_features(sender_lc, csr: CSR, rows: np.ndarray) -> np.ndarray:
+def pooled_features(sender_lc, csr: CSR, rows: np.ndarray, unrotate=None) -> np.ndarray:
     """Pool one sender layer/role over the alignment rows: for receiver row j,
-    sum_k w_k * c_k over the row's entries (a single copy for TA)."""
+    sum_k w_k * c_k over the row's entries (a single copy for TA).
+
+    unrotate: None, or (s_pos, inv_freq_s, H_s) for sender keys stored with
+    RoPE: each sender row k is first rotated back at its position s_pos[k]
+    (rope_inverse), then weighted and summed."""
     starts = csr.row_ptr[rows]
     ends = csr.row_ptr[rows + 1]
     if np.any(ends <= starts):
         raise ValueError("every alignment row needs at least one sender token")
     lengths = ends - starts
     entry = np.concatenate([np.arange(a, b) for a, b in zip(starts, ends)])
-    feats = np.asarray(sender_lc[csr.col[entry]], dtype=np.float64)
+    cols = csr.col[entry]
+    feats = np.asarray(sender_lc[cols], dtype=np.float64)
+    if unrotate is not None:
+        s_pos, inv_freq_s, H_s = unrotate
+        n, d_s = feats.shape
+        feats = rope_inverse(feats.reshape(n, H_s, d_s // H_s), np.asarray(s_pos)[cols],
+                             inv_freq_s).reshape(n, d_s)
     feats = feats * csr.w[entry][:, None]
     seg_start = np.concatenate([[0], np.cumsum(lengths)[:-1]])
     return np.add.reduceat(feats, seg_start, axis=0)
 
 
-def map_input(sender, csr: CSR, segments_l, role: int, rows: np.ndarray) -> np.ndarray:
+def map_input(sender, csr: CSR, segments_l, role: int, rows: np.ndarray,
+              sender_rope=None) -> np.ndarray:
     """Eq. 2: the concatenated map input x for receiver layer l and role c.
 
     Segment s is the weighted sum of its sender layers' pooled features;
-    the segments are concatenated along the feature axis.
+    the segments are concatenated along the feature axis.  sender_rope
+    (keys only): see pooled_features' unrotate.
     """
+    unrot = sender_rope if role == ROLE_K else None
     parts = []
     for seg in segments_l:
         acc = None
         for (t, omega) in seg:
-            term = omega * pooled_features(sender[t][role], csr, rows)
+            term = omega * pooled_features(sender[t][role], csr, rows, unrot)
             acc = term if acc is None else acc + term
         parts.append(acc)
     return np.concatenate(parts, axis=1)
@@ -360,7 +402,8 @@ def transfer(sender, csr: CSR, segments, A, b, r, *, H_r: int, D_r: int,
              knorm_g: Optional[np.ndarray] = None, knorm_eps: float = 1e-6,
              layers: Optional[Iterable[int]] = None,
              rows: Optional[np.ndarray] = None,
-             roles: Iterable[int] = (ROLE_K, ROLE_V)) -> Dict[Tuple[int, int], np.ndarray]:
+             roles: Iterable[int] = (ROLE_K, ROLE_V),
+             sender_rope=None) -> Dict[Tuple[int, int], np.ndarray]:
     """The receiver cache entries for the requested layers, roles and rows.
 
     sender:  indexable as sender[t][c] -> [T_s, d_S] array (any float dtype)
@@ -369,6 +412,9 @@ def transfer(sender, csr: CSR, segments, A, b, r, *, H_r: int, D_r: int,
     A:       indexable as A[l][c] -> [K, d_R] (paper orientation, x @ A)
     b:       [L_R][2][d_R];  r: [L_R][2] positive scalars (Eq. 3's r)
     pos:     receiver position of every receiver row (RoPE position)
+    sender_rope: None (sender keys captured before RoPE, the paper's case) or
+             (s_pos, inv_freq_s, H_s) when the sender keys carry RoPE at
+             sender positions s_pos: they are rotated back before pooling.
 
     Returns {(l, c): [n_rows, H_r, D_r] float64}.  Eq. 9:
     Phi(x) = (x / r) A + b, reshaped to receiver heads; keys then get the
@@ -380,7 +426,7 @@ def transfer(sender, csr: CSR, segments, A, b, r, *, H_r: int, D_r: int,
     out: Dict[Tuple[int, int], np.ndarray] = {}
     for l in layers:
         for c in roles:
-            x = map_input(sender, csr, segments[l], c, rows)
+            x = map_input(sender, csr, segments[l], c, rows, sender_rope)
             A_lc = np.asarray(A[l][c], dtype=np.float64)
             if A_lc.shape != (x.shape[1], H_r * D_r):
                 raise ValueError(f"map shape {A_lc.shape} does not match input "
@@ -395,13 +441,23 @@ def transfer(sender, csr: CSR, segments, A, b, r, *, H_r: int, D_r: int,
     return out
 
 
-def receiver_positions(r_tok_ptr: Sequence[int], r_pos0: Optional[Sequence[int]] = None) -> np.ndarray:
-    """RoPE position of every concatenated receiver token: the request's
+def token_positions(tok_ptr: Sequence[int], pos0: Optional[Sequence[int]] = None) -> np.ndarray:
+    """RoPE position of every concatenated token of one model: the request's
     origin (default 0) plus the token's index within its request."""
-    n_req = len(r_tok_ptr) - 1
+    n_req = len(tok_ptr) - 1
     pos = []
     for q in range(n_req):
-        base = 0 if r_pos0 is None else int(r_pos0[q])
-        for t in range(int(r_tok_ptr[q + 1]) - int(r_tok_ptr[q])):
+        base = 0 if pos0 is None else int(pos0[q])
+        for t in range(int(tok_ptr[q + 1]) - int(tok_ptr[q])):
             pos.append(base + t)
     return np.asarray(pos, dtype=np.int64)
+
+
+def receiver_positions(r_tok_ptr: Sequence[int], r_pos0: Optional[Sequence[int]] = None) -> np.ndarray:
+    """Receiver RoPE positions (token_positions of the receiver side)."""
+    return token_positions(r_tok_ptr, r_pos0)
+
+
+def sender_positions(s_tok_ptr: Sequence[int], s_pos0: Optional[Sequence[int]] = None) -> np.ndarray:
+    """Sender RoPE positions (token_positions of the sender side)."""
+    return token_positions(s_tok_ptr, s_pos0)

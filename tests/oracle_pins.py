@@ -261,6 +261,23 @@ def check_rope_relative_position():
         assert abs(lhs - rhs) < 1e-8
 
 
+def check_rope_inverse():
+    """rope_inverse is the rotation by the negative angle: the complex form
+    z * exp(-1j p f); it undoes rope at the same position, both ways round."""
+    rng = np.random.default_rng(3)
+    D = 16
+    inv = O.rope_inv_freq(1e6, D)
+    x = rng.normal(size=(5, 2, D))
+    pos = np.array([0, 1, 29, 8191, 131071])
+    y = O.rope_inverse(x, pos, inv)
+    z = x[..., : D // 2] + 1j * x[..., D // 2:]
+    zr = z * np.exp(-1j * pos[:, None, None] * inv[None, None, :])
+    assert np.allclose(y[..., : D // 2], zr.real, atol=1e-9)
+    assert np.allclose(y[..., D // 2:], zr.imag, atol=1e-9)
+    assert np.allclose(O.rope(y, pos, inv), x, atol=1e-9)
+    assert np.allclose(O.rope_inverse(O.rope(x, pos, inv), pos, inv), x, atol=1e-9)
+
+
 def check_inv_freq():
     inv = O.rope_inv_freq(10000.0, 128)
     assert inv[0] == 1.0
@@ -304,10 +321,27 @@ def _tiny_problem(seed, align_mode, layer_mode, L_s=3, L_r=4, H_s=2, D_s=4, H_r=
                 H_r=H_r, D_r=D_r, d_s=d_s, s_end=s_end, r_end=r_end)
 
 
-def _transfer_brute(P, knorm_g=None, eps=1e-6):
-    """Every output element from the definitions, with Python loops."""
+def _transfer_brute(P, knorm_g=None, eps=1e-6, srope=None):
+    """Every output element from the definitions, with Python loops.
+    srope = (s_pos, inv_freq_s, H_s): sender keys carry RoPE and each sender
+    feature is rotated back at its token's position before it is used."""
     sender, segs, A, b, r, csr = P["sender"], P["segs"], P["A"], P["b"], P["r"], P["csr"]
     H_r, D_r, d_s, inv, pos = P["H_r"], P["D_r"], P["d_s"], P["inv"], P["pos"]
+
+    def feature(t, c, k, d):
+        v = sender[t, c, k, d]
+        if srope is None or c != 0:
+            return v
+        s_pos, inv_s, H_s = srope
+        D_s = d_s // H_s
+        h, i = divmod(d, D_s)
+        hs = D_s // 2
+        f = inv_s[i % hs]
+        ang = s_pos[k] * f
+        if i < hs:  # x' = x cos + y sin
+            return v * math.cos(ang) + sender[t, c, k, h * D_s + i + hs] * math.sin(ang)
+        return v * math.cos(ang) - sender[t, c, k, h * D_s + i - hs] * math.sin(ang)
+
     out = {}
     for l in range(len(segs)):
         for c in (0, 1):
@@ -321,7 +355,7 @@ def _transfer_brute(P, knorm_g=None, eps=1e-6):
                             for e in range(csr.row_ptr[j], csr.row_ptr[j + 1]):
                                 k, wk = csr.col[e], csr.w[e]
                                 for d in range(d_s):
-                                    acc += omega * wk * sender[t, c, k, d] * A[l, c, s * d_s + d, n]
+                                    acc += omega * wk * feature(t, c, k, d) * A[l, c, s * d_s + d, n]
                     y.append(acc / r[l, c] + b[l, c, n])
                 for h in range(H_r):
                     v = y[h * D_r:(h + 1) * D_r]
@@ -365,6 +399,48 @@ def check_transfer_brute_force():
         assert np.allclose(got[key], ref[key], rtol=1e-10, atol=1e-10)
 
 
+def check_transfer_brute_force_rotated_sender():
+    """Sender keys stored with RoPE: the brute force rotates each sender
+    feature back at its own sender position; pooled and blended modes."""
+    for seed, am, lm in [(10, O.ALIGN_TA, O.LAYER_PAPER3),
+                         (11, O.ALIGN_OVERLAP_MEAN, O.LAYER_INTERP)]:
+        P = _tiny_problem(seed, am, lm)
+        n_s = len(P["s_end"])
+        s_pos = O.sender_positions([0, n_s], [3])
+        assert s_pos.tolist() == list(range(3, 3 + n_s))
+        inv_s = O.rope_inv_freq(500000.0, 4)
+        got = _run_oracle(P, sender_rope=(s_pos, inv_s, 2))
+        ref = _transfer_brute(P, srope=(s_pos, inv_s, 2))
+        for key in ref:
+            assert np.allclose(got[key], ref[key], rtol=1e-10, atol=1e-10), (seed, key)
+
+
+def check_explicit_segments():
+    """A caller-given layer table: the Eq. 1 triples given explicitly give
+    the paper-mode table, and a hand-made two-term table maps as written."""
+    L_s, L_r = 32, 40
+    trip = O.layer_alignment(L_s, L_r)
+    ex = O.explicit_segments([[[t] for t in tr] for tr in trip], [[[1.0]] * 3 for _ in trip])
+    assert ex == O.layer_segments(O.LAYER_PAPER3, L_s, L_r)
+    ex2 = O.explicit_segments([[[0, 2], [1, 1]]], [[[0.25, 0.75], [1.0, -2.0]]])
+    assert ex2 == [[[(0, 0.25), (2, 0.75)], [(1, 1.0), (1, -2.0)]]]
+    P = _tiny_problem(12, O.ALIGN_OVERLAP_MEAN, O.LAYER_PAPER3, L_s=3, L_r=1)
+    P["segs"] = ex2
+    P["A"] = P["A"][:, :, : 2 * P["d_s"], :]
+    got = _run_oracle(P)
+    ref = _transfer_brute(P)
+    for key in ref:
+        assert np.allclose(got[key], ref[key], rtol=1e-10, atol=1e-10), key
+    # segment 1 is (1 - 2) * layer 1 = -layer 1
+    A1 = np.zeros_like(P["A"])
+    A1[:, :, P["d_s"]:, :] = P["A"][:, :, P["d_s"]:, :]
+    y = _run_oracle(dict(P, A=A1), roles=(1,))[(0, 1)]
+    rows = np.arange(P["csr"].n_rows)
+    x = O.pooled_features(P["sender"][1, 1], P["csr"], rows)
+    ref1 = -x @ P["A"][0, 1, P["d_s"]:, :] / P["r"][0, 1] + P["b"][0, 1]
+    assert np.allclose(y.reshape(len(rows), -1), ref1)
+
+
 def check_identity_map_reproduces_input():
     """Same depth, same tokenisation, A = [0; I; 0] (the middle block reads
     sender layer pi(l) = l), b = 0, r = 1: V is the sender V, K is the sender K
@@ -391,6 +467,89 @@ def check_identity_map_reproduces_input():
         zc = zc * np.exp(1j * pos[:, None, None] * inv[None, None, :])
         assert np.allclose(out[(l, 0)][..., : D // 2], zc.real)
         assert np.allclose(out[(l, 0)][..., D // 2:], zc.imag)
+
+
+def _identity_setup(L, H, D, lengths, seed):
+    d = H * D
+    rng = np.random.default_rng(seed)
+    ends = _ends(lengths)
+    sender = rng.normal(size=(L, 2, len(ends), d))
+    segs = O.layer_segments(O.LAYER_PAPER3, L, L)
+    A = np.zeros((L, 2, 3 * d, d))
+    A[:, :, d:2 * d, :] = np.eye(d)
+    csr = O.alignment_csr(O.ALIGN_TA, [0, len(ends)], [0, len(ends)], ends, ends)
+    return sender, segs, A, np.zeros((L, 2, d)), np.ones((L, 2)), csr, ends
+
+
+def check_identity_rotated_sender_keys():
+    """The identity special case with sender keys stored rotated: same
+    depth, same tokenisation, A = [0; I; 0], b = 0, r = 1, the same RoPE base
+    and the same positions on both sides: un-rotate then rotate reproduces
+    the sender keys, and values pass through unrotated."""
+    L, H, D = 4, 2, 8
+    sender, segs, A, b, r, csr, ends = _identity_setup(L, H, D, [1, 3, 2, 2, 4, 1], 13)
+    n = len(ends)
+    inv = O.rope_inv_freq(10000.0, D)
+    pos = O.receiver_positions([0, n], [7])
+    s_pos = O.sender_positions([0, n], [7])
+    out = O.transfer(sender, csr, segs, A, b, r, H_r=H, D_r=D, pos=pos, inv_freq_r=inv,
+                     sender_rope=(s_pos, inv, H))
+    for l in range(L):
+        assert np.allclose(out[(l, 0)].reshape(n, H * D), sender[l, 0], atol=1e-12)
+        assert np.array_equal(out[(l, 1)].reshape(n, H * D), sender[l, 1])
+
+
+def check_rotated_sender_position_shift():
+    """Sender keys rotated at sender positions p (base theta_s), receiver at
+    p + delta (base theta_r), identity map: in complex form each pair is
+    multiplied by exp(1j ((p + delta) f_r - p f_s))."""
+    L, H, D = 3, 1, 8
+    sender, segs, A, b, r, csr, ends = _identity_setup(L, H, D, [2, 2, 1, 3, 2], 14)
+    n = len(ends)
+    inv_r = O.rope_inv_freq(1e6, D)
+    inv_s = O.rope_inv_freq(5e5, D)
+    pos = O.receiver_positions([0, n], [11])
+    s_pos = O.sender_positions([0, n])
+    out = O.transfer(sender, csr, segs, A, b, r, H_r=H, D_r=D, pos=pos, inv_freq_r=inv_r,
+                     sender_rope=(s_pos, inv_s, H), roles=(0,))
+    for l in range(L):
+        z = sender[l, 0].reshape(n, H, D)
+        zc = z[..., : D // 2] + 1j * z[..., D // 2:]
+        ang = pos[:, None, None] * inv_r[None, None, :] - s_pos[:, None, None] * inv_s[None, None, :]
+        zc = zc * np.exp(1j * ang)
+        assert np.allclose(out[(l, 0)][..., : D // 2], zc.real, atol=1e-12)
+        assert np.allclose(out[(l, 0)][..., D // 2:], zc.imag, atol=1e-12)
+
+
+def check_rotated_sender_unrotates_before_pooling():
+    """Every sender key is one vector v rotated to its own position; overlap
+    mean pooling of the un-rotated keys gives v exactly, whatever the rows'
+    spans, so with the identity map the receiver key is v rotated to the
+    receiver position.  Rotating back after pooling would not give v."""
+    L, H, D = 3, 2, 8
+    d = H * D
+    rng = np.random.default_rng(15)
+    s_end = _ends([2, 1, 3, 1, 1, 4, 2])
+    r_end = _ends([3, 4, 1, 3, 3])
+    assert s_end[-1] == r_end[-1]
+    n_s, n_r = len(s_end), len(r_end)
+    inv = O.rope_inv_freq(10000.0, D)
+    s_pos = O.sender_positions([0, n_s], [5])
+    v = rng.normal(size=(1, H, D))
+    rotated = O.rope(np.repeat(v, n_s, axis=0), s_pos, inv).reshape(n_s, d)
+    sender = np.zeros((L, 2, n_s, d))
+    sender[:, 0] = rotated
+    segs = O.layer_segments(O.LAYER_PAPER3, L, L)
+    A = np.zeros((L, 2, 3 * d, d))
+    A[:, :, d:2 * d, :] = np.eye(d)
+    csr = O.alignment_csr(O.ALIGN_OVERLAP_MEAN, [0, n_s], [0, n_r], s_end, r_end)
+    assert max(csr.row_ptr[j + 1] - csr.row_ptr[j] for j in range(n_r)) > 1
+    pos = O.receiver_positions([0, n_r])
+    out = O.transfer(sender, csr, segs, A, np.zeros((L, 2, d)), np.ones((L, 2)), H_r=H, D_r=D,
+                     pos=pos, inv_freq_r=inv, sender_rope=(s_pos, inv, H), roles=(0,))
+    want = O.rope(np.repeat(v, n_r, axis=0), pos, inv)
+    for l in range(L):
+        assert np.allclose(out[(l, 0)], want, atol=1e-12)
 
 
 def check_affine_structure():
@@ -435,8 +594,11 @@ ALL_CHECKS = [
     check_layer_alignment_closed_form, check_layer_alignment_hand_tables,
     check_layer_interpolation, check_mapper_size_table_f,
     check_rope_two_dim_rotation, check_rope_complex_form, check_rope_relative_position,
-    check_inv_freq, check_key_norm,
-    check_transfer_brute_force, check_identity_map_reproduces_input,
+    check_rope_inverse, check_inv_freq, check_key_norm,
+    check_transfer_brute_force, check_transfer_brute_force_rotated_sender,
+    check_explicit_segments, check_identity_map_reproduces_input,
+    check_identity_rotated_sender_keys, check_rotated_sender_position_shift,
+    check_rotated_sender_unrotates_before_pooling,
     check_affine_structure, check_segment_blocks,
 ]
 

@@ -86,20 +86,61 @@ def _overlap_closed(s_end, r_end):
     return rows
 
 
-def _pool_unweighted(sender_lc, csr, rows):
+def _pool_unweighted(sender_lc, csr, rows, unrotate=None):
     out = []
     for j in rows:
         idx = csr.col[csr.row_ptr[j]:csr.row_ptr[j + 1]]
-        out.append(np.asarray(sender_lc[idx], dtype=np.float64).sum(axis=0))
+        x = np.asarray(sender_lc[idx], dtype=np.float64)
+        if unrotate is not None:
+            s_pos, inv, H_s = unrotate
+            x = O.rope_inverse(x.reshape(len(idx), H_s, -1), np.asarray(s_pos)[idx], inv).reshape(len(idx), -1)
+        out.append(x.sum(axis=0))
     return np.asarray(out)
+
+
+def _rope_inverse_forward(x, pos, inv):
+    # wrong: rotates forward instead of back
+    return O.rope(x, pos, inv)
+
+
+_orig_pooled = O.pooled_features
+
+
+def _pool_then_unrotate(sender_lc, csr, rows, unrotate=None):
+    # wrong: pools the rotated rows, then rotates back once at the row's
+    # first sender position
+    y = _orig_pooled(sender_lc, csr, rows)
+    if unrotate is None:
+        return y
+    s_pos, inv, H_s = unrotate
+    first = csr.col[csr.row_ptr[rows]]
+    n, d = y.shape
+    return O.rope_inverse(y.reshape(n, H_s, d // H_s), np.asarray(s_pos)[first], inv).reshape(n, d)
+
+
+def _explicit_weights_swapped(seg_layer, seg_w):
+    return [[[(int(t), float(w)) for t, w in zip(ts, reversed(ws))] for ts, ws in zip(ls, wl)]
+            for ls, wl in zip(seg_layer, seg_w)]
 
 
 _orig_map_input = O.map_input
 _orig_transfer = O.transfer
 
 
-def _map_input_reversed(sender, csr, segments_l, role, rows):
-    return _orig_map_input(sender, csr, list(reversed(segments_l)), role, rows)
+def _map_input_reversed(sender, csr, segments_l, role, rows, sender_rope=None):
+    return _orig_map_input(sender, csr, list(reversed(segments_l)), role, rows, sender_rope)
+
+
+def _map_input_unrotates_values(sender, csr, segments_l, role, rows, sender_rope=None):
+    # wrong: values are rotated back as well
+    parts = []
+    for seg in segments_l:
+        acc = None
+        for (t, omega) in seg:
+            term = omega * _orig_pooled(sender[t][role], csr, rows, sender_rope)
+            acc = term if acc is None else acc + term
+        parts.append(acc)
+    return np.concatenate(parts, axis=1)
 
 
 def _transfer_no_bias(sender, csr, segments, A, b, r, **kw):
@@ -126,6 +167,10 @@ MUTATIONS = {
     "segments_reversed": ("map_input", _map_input_reversed),
     "bias_dropped": ("transfer", _transfer_no_bias),
     "r_multiplies": ("transfer", _transfer_times_r),
+    "rope_inverse_forward": ("rope_inverse", _rope_inverse_forward),
+    "unrotate_after_pooling": ("pooled_features", _pool_then_unrotate),
+    "values_unrotated": ("map_input", _map_input_unrotates_values),
+    "explicit_weights_swapped": ("explicit_segments", _explicit_weights_swapped),
 }
 
 
@@ -135,3 +180,6 @@ def test_pins_catch_planted_mistake(name, monkeypatch):
     monkeypatch.setattr(O, attr, fn)
     failures = pins.run_all()
     assert failures, f"no pin caught the planted mistake {name!r}"
+    # a mutation with the wrong call signature would "fail" every pin for the
+    # wrong reason; at least one pin must fail on an assertion
+    assert any(msg.startswith("AssertionError") for _, msg in failures), failures
