@@ -83,7 +83,11 @@ typedef enum {
   HF_LAYER_PAPER3 = 0,
   /* One segment: the linear interpolation of sender layers floor(p) and
      floor(p)+1 at p = l (L_S-1)/(L_R-1) (zero-based l): K = d_S. */
-  HF_LAYER_INTERP = 1
+  HF_LAYER_INTERP = 1,
+  /* A caller-given table with the structure of Eq. 2: n_seg segments per
+     receiver layer, segment s = sum over its n_terms terms of
+     h_seg_w * (sender layer h_seg_layer): K = n_seg d_S. */
+  HF_LAYER_EXPLICIT = 2
 } hf_layer_mode;
 
 typedef enum {
@@ -155,15 +159,17 @@ typedef struct {
   const float* d_w;             /* float[nnz] */
 
   /* Folded maps (Eq. 9), device.  d_W is A_final transposed:
-     [L_r][2][d_R][K] row-major in `dtype`, K = 3 d_S (PAPER3) or d_S
-     (INTERP); row n of W[l][c] holds column n of A_final, and segment s of
-     the map input occupies W columns [s d_S, (s+1) d_S). */
+     [L_r][2][d_R][K] row-major in `dtype`, K = 3 d_S (PAPER3), d_S
+     (INTERP) or n_seg d_S (EXPLICIT); row n of W[l][c] holds column n of
+     A_final, and segment s of the map input occupies W columns
+     [s d_S, (s+1) d_S). */
   const void* d_W;
   const float* d_b;             /* float[L_r][2][d_R], b_final */
   const float* h_r;             /* host float[L_r][2], Eq. 3's r (> 0) */
 
   /* Receiver key processing. */
-  double theta_r;               /* RoPE base; <= 0 disables RoPE */
+  double theta_r;               /* RoPE base; <= 0 disables RoPE unless
+                                   h_inv_freq_r is given */
   const float* d_knorm_w;       /* device float[D_r] key RMS-norm weight, or NULL */
   float knorm_eps;
 
@@ -177,6 +183,34 @@ typedef struct {
   int32_t n_blocks;
   int32_t max_blocks_per_req;
   const int32_t* d_block_table; /* device int32[n_req][max_blocks_per_req] */
+
+  /* Optional fields below: a zero-initialised descriptor leaves them off. */
+
+  /* Receiver RoPE inverse frequencies, host float[D_r/2] (for instance a
+     scaled RoPE variant's table); NULL = fp32(theta_r^(-2i/D_r)).  When
+     given, keys are rotated whatever theta_r is. */
+  const float* h_inv_freq_r;
+
+  /* Sender keys that already carry RoPE.  The paper maps keys captured
+     before RoPE (Section 3 opening paragraph); with sender_k_rotated = 1
+     the sender keys hold RoPE at sender positions and every sender key row
+     is rotated back (rotate-half pairs (i, i + D_s/2), angle
+     -pos * inv_freq_s_i) at its own sender position before pooling and
+     blending; values are not touched.  The sender position of token t of
+     request q is s_pos0[q] + t.  Requires D_s/2 a multiple of 8 (bf16) or
+     4 (fp32), D_s dividing 128 (bf16) or 64 (fp32), and d_S a multiple of
+     128 (bf16) or 64 (fp32); slower than the default path (the rotation
+     runs in the operand builder). */
+  int32_t sender_k_rotated;
+  double theta_s;               /* sender RoPE base, used when h_inv_freq_s is NULL */
+  const float* h_inv_freq_s;    /* host float[D_s/2], or NULL */
+  const int32_t* s_pos0;        /* host int32[n_req], or NULL for 0 */
+
+  /* HF_LAYER_EXPLICIT only: host arrays [L_r][n_seg][n_terms]. */
+  int32_t n_seg;                /* 1 .. 3 segments per receiver layer */
+  int32_t n_terms;              /* 1 .. 2 sender layers per segment */
+  const int32_t* h_seg_layer;   /* zero-based sender layers, in [0, L_s) */
+  const float* h_seg_w;         /* finite weights */
 } hf_plan_desc;
 
 typedef struct hf_plan_s* hf_plan;
@@ -186,10 +220,11 @@ hf_status hf_plan_workspace_size(const hf_plan_desc* desc, size_t* bytes);
 
 /*
  * hf_plan_create — validate the descriptor and build the per-transfer
- * metadata on `stream`: the layer table (Eq. 1 or interpolation), RoPE
- * inverse frequencies fp32(theta_r^(-2i/D_r)), the receiver position and
- * destination row of every receiver token, and the runs of identical CSR
- * rows (their map output is identical before RoPE).
+ * metadata on `stream`: the layer table (Eq. 1, interpolation or explicit),
+ * RoPE inverse frequencies (fp32(theta^(-2i/D)) or the caller's tables), the
+ * receiver position and destination row of every receiver token, the
+ * sender position of every sender token (sender_k_rotated only), and the
+ * runs of identical CSR rows (their map output is identical before RoPE).
  * d_workspace: device memory of hf_plan_workspace_size bytes, 256-byte
  * aligned, owned by the caller and reserved for this plan until
  * hf_plan_destroy.  The plan keeps pointers to d_row_ptr, d_col, d_w,
@@ -201,8 +236,9 @@ hf_status hf_plan_create(const hf_plan_desc* desc, void* d_workspace, size_t wor
 /*
  * hf_transfer — write the receiver cache (one kernel launch on `stream`).
  * sender_kv:   device [L_s][2][T_s][H_s][D_s] in the plan's dtype, the
- *              sender's pre-RoPE keys and values (Section 3: keys are mapped
- *              before key normalisation and RoPE); 16-byte aligned.
+ *              sender's keys and values; keys pre-RoPE (Section 3: keys are
+ *              mapped before key normalisation and RoPE) unless the plan
+ *              says sender_k_rotated; 16-byte aligned.
  * receiver_kv: device, layout per desc.paged; 16-byte aligned.  Only the
  *              rows (contiguous) or block slots (paged) of the plan's
  *              receiver tokens are written.

@@ -26,7 +26,7 @@ HF_ERR_DEVICE_CHECK = 5
 HF_ERR_WORKSPACE = 6
 
 ALIGN_MODES = {"ta": 0, "overlap_mean": 1, "same_index": 2}
-LAYER_MODES = {"paper3": 0, "interp": 1}
+LAYER_MODES = {"paper3": 0, "interp": 1, "explicit": 2}
 DTYPES = {"bf16": 0, "f32": 1}
 
 CHECK_BITS = {
@@ -59,6 +59,11 @@ class PlanDesc(ctypes.Structure):
         ("paged", ctypes.c_int32), ("block_size", ctypes.c_int32),
         ("n_blocks", ctypes.c_int32), ("max_blocks_per_req", ctypes.c_int32),
         ("d_block_table", _p),
+        ("h_inv_freq_r", _f32p),
+        ("sender_k_rotated", ctypes.c_int32), ("theta_s", ctypes.c_double),
+        ("h_inv_freq_s", _f32p), ("s_pos0", _i32p),
+        ("n_seg", ctypes.c_int32), ("n_terms", ctypes.c_int32),
+        ("h_seg_layer", _i32p), ("h_seg_w", _f32p),
     ]
 
 
@@ -131,6 +136,14 @@ def _as_i32p(a: np.ndarray):
     return a.ctypes.data_as(_i32p)
 
 
+def _host_f32(a) -> np.ndarray:
+    return np.ascontiguousarray(np.asarray(a, dtype=np.float32).reshape(-1))
+
+
+def _f32_or_null(a: Optional[np.ndarray]):
+    return None if a is None else a.ctypes.data_as(_f32p)
+
+
 def align_build(mode: str, s_tok_ptr, r_tok_ptr, d_s_end, d_r_end, d_row_ptr, d_col, d_w,
                 nnz_capacity: int, d_info, stream=None) -> None:
     """hf_align_build.  Host token pointers (numpy), device arrays (torch)."""
@@ -148,11 +161,25 @@ class Desc:
     def __init__(self, *, L_s, H_s, D_s, L_r, H_r, D_r, dtype, layer_mode, align_mode,
                  s_tok_ptr, r_tok_ptr, d_row_ptr, d_col, d_w, d_W, d_b, r, theta_r,
                  r_pos0=None, d_knorm_w=None, knorm_eps=1e-6, paged=False, block_size=16,
-                 n_blocks=0, max_blocks_per_req=0, d_block_table=None):
+                 n_blocks=0, max_blocks_per_req=0, d_block_table=None, inv_freq_r=None,
+                 sender_k_rotated=False, theta_s=0.0, inv_freq_s=None, s_pos0=None,
+                 seg_layer=None, seg_w=None):
         self._s = _host_i32(s_tok_ptr)
         self._r = _host_i32(r_tok_ptr)
         self._pos0 = None if r_pos0 is None else _host_i32(r_pos0)
+        self._spos0 = None if s_pos0 is None else _host_i32(s_pos0)
         self._hr = np.ascontiguousarray(np.asarray(r, dtype=np.float32).reshape(-1))
+        self._ifr = None if inv_freq_r is None else _host_f32(inv_freq_r)
+        self._ifs = None if inv_freq_s is None else _host_f32(inv_freq_s)
+        n_seg = n_terms = 0
+        self._segl = self._segw = None
+        if seg_layer is not None:
+            sl = np.ascontiguousarray(np.asarray(seg_layer, dtype=np.int32))
+            if sl.ndim != 3:
+                raise ValueError("seg_layer must be [L_r][n_seg][n_terms]")
+            n_seg, n_terms = int(sl.shape[1]), int(sl.shape[2])
+            self._segl = sl.reshape(-1)
+            self._segw = _host_f32(np.broadcast_to(np.asarray(seg_w, dtype=np.float32), sl.shape))
         self.c = PlanDesc(
             L_s=L_s, H_s=H_s, D_s=D_s, L_r=L_r, H_r=H_r, D_r=D_r,
             dtype=DTYPES[dtype], layer_mode=LAYER_MODES[layer_mode],
@@ -163,7 +190,13 @@ class Desc:
             d_W=_dptr(d_W), d_b=_dptr(d_b), h_r=self._hr.ctypes.data_as(_f32p),
             theta_r=float(theta_r), d_knorm_w=_dptr(d_knorm_w), knorm_eps=float(knorm_eps),
             paged=int(bool(paged)), block_size=int(block_size), n_blocks=int(n_blocks),
-            max_blocks_per_req=int(max_blocks_per_req), d_block_table=_dptr(d_block_table))
+            max_blocks_per_req=int(max_blocks_per_req), d_block_table=_dptr(d_block_table),
+            h_inv_freq_r=_f32_or_null(self._ifr), sender_k_rotated=int(bool(sender_k_rotated)),
+            theta_s=float(theta_s), h_inv_freq_s=_f32_or_null(self._ifs),
+            s_pos0=_as_i32p(self._spos0) if self._spos0 is not None else None,
+            n_seg=n_seg, n_terms=n_terms,
+            h_seg_layer=_as_i32p(self._segl) if self._segl is not None else None,
+            h_seg_w=_f32_or_null(self._segw))
 
 
 def plan_workspace_size(desc: Desc) -> int:

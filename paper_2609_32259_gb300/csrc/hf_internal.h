@@ -33,8 +33,12 @@ struct WorkspaceLayout {
   size_t segs;       // LayerSegs[L_r]
   size_t inv_r;      // float[L_r * 2]  (1 / r)
   size_t inv_freq;   // float[D_r / 2]
+  size_t inv_freq_s; // float[D_s / 2]: sender RoPE (sender_k_rotated)
   size_t r_tok_ptr;  // int32[n_req + 1]
   size_t r_pos0;     // int32[n_req]
+  size_t s_tok_ptr;  // int32[n_req + 1]
+  size_t s_pos0;     // int32[n_req]
+  size_t spos;       // int32[T_s] sender RoPE positions (sender_k_rotated), else one word
   size_t run_ptr;    // int32[T_r + 1]: first receiver row of each distinct row
   size_t ucol;       // int32[T_r]: sender column of each distinct row (one-entry rows)
   size_t upos;       // int32[T_r]: RoPE position of each distinct row's first receiver row
@@ -44,18 +48,22 @@ struct WorkspaceLayout {
   size_t total;
 };
 
-WorkspaceLayout workspace_layout(int L_r, int D_r, int n_req, int64_t T_r);
+WorkspaceLayout workspace_layout(const hf_plan_desc& d);
 
 // Constant tables copied into the workspace by the plan kernel (passed by
 // value as a kernel parameter, so plan creation issues no host copies).
 struct PlanTables {
-  int32_t L_r, D_r, n_req;
+  int32_t L_r, D_r, D_s, n_req;
   LayerSegs segs[kMaxLayersR];
   float inv_r[2 * kMaxLayersR];
   float inv_freq[kMaxHeadDim / 2];
+  float inv_freq_s[kMaxHeadDim / 2];
   int32_t r_tok_ptr[kMaxReq + 1];
   int32_t r_pos0[kMaxReq];
+  int32_t s_tok_ptr[kMaxReq + 1];
+  int32_t s_pos0[kMaxReq];
 };
+static_assert(sizeof(PlanTables) < 32000, "PlanTables must fit the kernel parameter space");
 
 }  // namespace hf
 
@@ -65,6 +73,8 @@ struct hf_plan_s {
   int64_t T_s, T_r, nnz_hint;
   int BN, groups, stages;
   bool gather;  // every map input row is a single unweighted sender row
+  bool rope;    // receiver keys get RoPE
+  bool unrot;   // sender keys carry RoPE and are rotated back in the builder
   char* ws;
   size_t ws_bytes;
   hf::WorkspaceLayout lay;

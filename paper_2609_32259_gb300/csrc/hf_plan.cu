@@ -1,7 +1,8 @@
-// Plan creation: descriptor validation, the layer table (Eq. 1 or the
-// interpolation reading), RoPE inverse frequencies, and the per-transfer
-// device metadata (receiver positions and destination rows, runs of
-// identical alignment rows).  Also the error-reporting helpers of the ABI.
+// Plan creation: descriptor validation, the layer table (Eq. 1, the
+// interpolation reading or a caller-given table), RoPE inverse frequencies,
+// and the per-transfer device metadata (receiver positions and destination
+// rows, sender positions for rotated sender keys, runs of identical
+// alignment rows).  Also the error-reporting helpers of the ABI.
 #include <cmath>
 #include <cstdio>
 #include <cstdlib>
@@ -37,7 +38,10 @@ int device_sm_count() {
 
 static size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
-WorkspaceLayout workspace_layout(int L_r, int D_r, int n_req, int64_t T_r) {
+WorkspaceLayout workspace_layout(const hf_plan_desc& d) {
+  const int L_r = d.L_r, D_r = d.D_r, D_s = d.D_s, n_req = d.n_req;
+  const int64_t T_r = d.r_tok_ptr[n_req];
+  const int64_t n_spos = d.sender_k_rotated ? d.s_tok_ptr[n_req] : 0;
   WorkspaceLayout w{};
   size_t off = 0;
   auto take = [&](size_t bytes) {
@@ -50,8 +54,12 @@ WorkspaceLayout workspace_layout(int L_r, int D_r, int n_req, int64_t T_r) {
   w.segs = take(sizeof(LayerSegs) * (size_t)L_r);
   w.inv_r = take(sizeof(float) * 2 * (size_t)L_r);
   w.inv_freq = take(sizeof(float) * (size_t)(D_r / 2 > 0 ? D_r / 2 : 1));
+  w.inv_freq_s = take(sizeof(float) * (size_t)(D_s / 2 > 0 ? D_s / 2 : 1));
   w.r_tok_ptr = take(sizeof(int32_t) * (size_t)(n_req + 1));
   w.r_pos0 = take(sizeof(int32_t) * (size_t)n_req);
+  w.s_tok_ptr = take(sizeof(int32_t) * (size_t)(n_req + 1));
+  w.s_pos0 = take(sizeof(int32_t) * (size_t)n_req);
+  w.spos = take(sizeof(int32_t) * (size_t)(n_spos > 0 ? n_spos : 1));
   w.run_ptr = take(sizeof(int32_t) * (size_t)(T_r + 1));
   w.ucol = take(sizeof(int32_t) * (size_t)(T_r > 0 ? T_r : 1));
   w.upos = take(sizeof(int32_t) * (size_t)(T_r > 0 ? T_r : 1));
@@ -70,8 +78,12 @@ struct PlanDev {
   LayerSegs* segs;
   float* inv_r;
   float* inv_freq;
+  float* inv_freq_s;
   int32_t* r_tok_ptr;
   int32_t* r_pos0;
+  int32_t* s_tok_ptr;
+  int32_t* s_pos0;
+  int32_t* spos;
   int32_t* run_ptr;
   int32_t* ucol;
   int32_t* upos;
@@ -90,6 +102,10 @@ PlanDev plan_dev(const hf_plan_s* p) {
   d.inv_freq = reinterpret_cast<float*>(at(p->lay.inv_freq));
   d.r_tok_ptr = reinterpret_cast<int32_t*>(at(p->lay.r_tok_ptr));
   d.r_pos0 = reinterpret_cast<int32_t*>(at(p->lay.r_pos0));
+  d.inv_freq_s = reinterpret_cast<float*>(at(p->lay.inv_freq_s));
+  d.s_tok_ptr = reinterpret_cast<int32_t*>(at(p->lay.s_tok_ptr));
+  d.s_pos0 = reinterpret_cast<int32_t*>(at(p->lay.s_pos0));
+  d.spos = reinterpret_cast<int32_t*>(at(p->lay.spos));
   d.run_ptr = reinterpret_cast<int32_t*>(at(p->lay.run_ptr));
   d.ucol = reinterpret_cast<int32_t*>(at(p->lay.ucol));
   d.upos = reinterpret_cast<int32_t*>(at(p->lay.upos));
@@ -111,6 +127,19 @@ __global__ void plan_init_kernel(PlanTables t, PlanDev d) {
   for (int i = tid; i < t.D_r / 2; i += blockDim.x) d.inv_freq[i] = t.inv_freq[i];
   for (int i = tid; i <= t.n_req; i += blockDim.x) d.r_tok_ptr[i] = t.r_tok_ptr[i];
   for (int i = tid; i < t.n_req; i += blockDim.x) d.r_pos0[i] = t.r_pos0[i];
+  for (int i = tid; i < t.D_s / 2; i += blockDim.x) d.inv_freq_s[i] = t.inv_freq_s[i];
+  for (int i = tid; i <= t.n_req; i += blockDim.x) d.s_tok_ptr[i] = t.s_tok_ptr[i];
+  for (int i = tid; i < t.n_req; i += blockDim.x) d.s_pos0[i] = t.s_pos0[i];
+}
+
+// Sender RoPE position of every sender token (sender_k_rotated): the
+// request's origin plus the token's index within the request.
+__global__ void plan_spos_kernel(PlanDev d, int64_t T_s, int n_req) {
+  for (int64_t k = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; k < T_s;
+       k += (int64_t)gridDim.x * blockDim.x) {
+    const int q = find_request(d.s_tok_ptr, n_req, k);
+    d.spos[k] = d.s_pos0[q] + static_cast<int32_t>(k - d.s_tok_ptr[q]);
+  }
 }
 
 struct RowArgs {
@@ -211,7 +240,17 @@ void build_layer_table(const hf_plan_desc& d, LayerSegs* out) {
   for (int l = 0; l < d.L_r; ++l) {
     LayerSegs s;
     std::memset(&s, 0, sizeof(s));
-    if (d.layer_mode == HF_LAYER_PAPER3) {
+    if (d.layer_mode == HF_LAYER_EXPLICIT) {
+      s.n_seg = d.n_seg;
+      for (int k = 0; k < d.n_seg; ++k) {
+        s.n_terms[k] = d.n_terms;
+        for (int t = 0; t < d.n_terms; ++t) {
+          const size_t i = ((size_t)l * d.n_seg + k) * d.n_terms + t;
+          s.layer[k][t] = d.h_seg_layer[i];
+          s.w[k][t] = d.h_seg_w[i];
+        }
+      }
+    } else if (d.layer_mode == HF_LAYER_PAPER3) {
       // N(l) = clip(pi - 4, pi, pi + 4) to [1, L_S], one segment each.
       const int pi = proportional_depth(l + 1, d.L_s, d.L_r);
       const int offs[3] = {-4, 0, 4};
@@ -255,8 +294,21 @@ hf_status validate(const hf_plan_desc* d) {
   if (d->L_s < 1 || d->H_s < 1 || d->D_s < 1 || d->L_r < 1 || d->H_r < 1 || d->D_r < 1)
     return bad("shapes must be positive");
   if (d->dtype != HF_BF16 && d->dtype != HF_F32) return bad("unknown dtype");
-  if (d->layer_mode != HF_LAYER_PAPER3 && d->layer_mode != HF_LAYER_INTERP)
+  if (d->layer_mode != HF_LAYER_PAPER3 && d->layer_mode != HF_LAYER_INTERP &&
+      d->layer_mode != HF_LAYER_EXPLICIT)
     return bad("unknown layer mode");
+  if (d->layer_mode == HF_LAYER_EXPLICIT) {
+    if (d->n_seg < 1 || d->n_seg > kMaxSeg) return bad("explicit layer table: n_seg must be 1..3");
+    if (d->n_terms < 1 || d->n_terms > kMaxTerms)
+      return bad("explicit layer table: n_terms must be 1..2");
+    if (!d->h_seg_layer || !d->h_seg_w) return bad("explicit layer table: null arrays");
+    const size_t n = (size_t)d->L_r * d->n_seg * d->n_terms;
+    for (size_t i = 0; i < n; ++i) {
+      if (d->h_seg_layer[i] < 0 || d->h_seg_layer[i] >= d->L_s)
+        return bad("explicit layer table: sender layer out of range");
+      if (!std::isfinite(d->h_seg_w[i])) return bad("explicit layer table: weight not finite");
+    }
+  }
   if (d->align_mode != HF_ALIGN_TA && d->align_mode != HF_ALIGN_OVERLAP_MEAN &&
       d->align_mode != HF_ALIGN_SAME_INDEX)
     return bad("unknown align mode");
@@ -282,6 +334,22 @@ hf_status validate(const hf_plan_desc* d) {
   if (d->D_r % 32 || d->D_r > kMaxHeadDim) return unsup("D_r must be a multiple of 32, <= 256");
   const int BN = (d_r % 256 == 0) ? 256 : 128;
   if (BN % d->D_r) return unsup("a receiver head must fit one 128/256-column tile");
+  if (d->h_inv_freq_r)
+    for (int i = 0; i < d->D_r / 2; ++i)
+      if (!std::isfinite(d->h_inv_freq_r[i])) return bad("h_inv_freq_r not finite");
+  if (d->sender_k_rotated) {
+    if (d->sender_k_rotated != 1) return bad("sender_k_rotated must be 0 or 1");
+    if (!d->h_inv_freq_s && !(d->theta_s > 0.0))
+      return bad("sender_k_rotated needs theta_s > 0 or h_inv_freq_s");
+    if (d->h_inv_freq_s)
+      for (int i = 0; i < d->D_s / 2; ++i)
+        if (!std::isfinite(d->h_inv_freq_s[i])) return bad("h_inv_freq_s not finite");
+    if (d->D_s > kMaxHeadDim) return unsup("sender_k_rotated: D_s above 256");
+    const int chunk = 16 / esize;  // elements per 16-byte chunk
+    if (d->D_s % 2 || (d->D_s / 2) % chunk || (2 * bke) % d->D_s || d_s % (2 * bke))
+      return unsup("sender_k_rotated: D_s/2 must be a multiple of 8 (bf16) or 4 (fp32), D_s must "
+                   "divide 128 (bf16) or 64 (fp32), d_S a multiple of 128 (bf16) or 64 (fp32)");
+  }
   if (d->paged) {
     if (d->block_size < 1 || d->n_blocks < 1 || d->max_blocks_per_req < 1 || !d->d_block_table)
       return bad("paged layout needs block_size, n_blocks, max_blocks_per_req, d_block_table");
@@ -317,6 +385,11 @@ hf_status launch_plan_kernels(hf_plan_s* p, const PlanTables& tables, cudaStream
   plan_rows_kernel<<<grid, 256, 0, stream>>>(a);
   scan_inplace_kernel<ScanSum><<<1, kScanThreads, 0, stream>>>(d.new_flag, p->T_r, nullptr);
   plan_runs_kernel<<<grid, 256, 0, stream>>>(a);
+  if (p->unrot && p->T_s > 0) {
+    const int64_t want_s = (p->T_s + 255) / 256;
+    const int grid_s = static_cast<int>(std::min<int64_t>(want_s, 8LL * device_sm_count()));
+    plan_spos_kernel<<<grid_s, 256, 0, stream>>>(d, p->T_s, p->desc.n_req);
+  }
   HF_CUDA_TRY(cudaGetLastError(), "plan kernels launch");
   return HF_OK;
 }
@@ -326,11 +399,12 @@ hf_status launch_plan_kernels(hf_plan_s* p, const PlanTables& tables, cudaStream
 using namespace hf;
 
 extern "C" hf_status hf_plan_workspace_size(const hf_plan_desc* desc, size_t* bytes) {
-  if (!desc || !bytes || !desc->r_tok_ptr || desc->n_req < 1 || desc->n_req > kMaxReq) {
+  if (!desc || !bytes || !desc->r_tok_ptr || !desc->s_tok_ptr || desc->n_req < 1 ||
+      desc->n_req > kMaxReq) {
     set_error("hf_plan_workspace_size: invalid descriptor");
     return HF_ERR_INVALID_ARGUMENT;
   }
-  *bytes = workspace_layout(desc->L_r, desc->D_r, desc->n_req, desc->r_tok_ptr[desc->n_req]).total;
+  *bytes = workspace_layout(*desc).total;
   return HF_OK;
 }
 
@@ -342,8 +416,7 @@ hf_status plan_build(const hf_plan_desc* desc, void* d_workspace, size_t workspa
                      cudaStream_t stream, hf_plan_s* p, PlanTables* t) {
   const hf_status v = validate(desc);
   if (v != HF_OK) return v;
-  const WorkspaceLayout lay =
-      workspace_layout(desc->L_r, desc->D_r, desc->n_req, desc->r_tok_ptr[desc->n_req]);
+  const WorkspaceLayout lay = workspace_layout(*desc);
   if (!d_workspace || workspace_bytes < lay.total ||
       (reinterpret_cast<uintptr_t>(d_workspace) & 255u)) {
     set_error("hf_plan_create: workspace missing, too small or not 256-byte aligned");
@@ -352,13 +425,24 @@ hf_status plan_build(const hf_plan_desc* desc, void* d_workspace, size_t workspa
   p->desc = *desc;
   p->d_s = desc->H_s * desc->D_s;
   p->d_r = desc->H_r * desc->D_r;
-  p->n_seg = desc->layer_mode == HF_LAYER_PAPER3 ? 3 : 1;
+  p->n_seg = desc->layer_mode == HF_LAYER_PAPER3 ? 3
+             : desc->layer_mode == HF_LAYER_EXPLICIT ? desc->n_seg : 1;
   p->K = p->n_seg * p->d_s;
   p->T_s = desc->s_tok_ptr[desc->n_req];
   p->T_r = desc->r_tok_ptr[desc->n_req];
   p->BN = (p->d_r % 256 == 0) ? 256 : 128;
   p->groups = ((p->BN / 2) % desc->D_r == 0) ? 2 : 1;
-  p->gather = desc->layer_mode == HF_LAYER_PAPER3 && desc->align_mode != HF_ALIGN_OVERLAP_MEAN;
+  // The copy-only operand path needs every segment to be one sender layer
+  // with weight 1, one-entry rows and no rotation.
+  bool one_layer_segments = desc->layer_mode == HF_LAYER_PAPER3;
+  if (desc->layer_mode == HF_LAYER_EXPLICIT && desc->n_terms == 1) {
+    one_layer_segments = true;
+    for (int i = 0; i < desc->L_r * desc->n_seg; ++i)
+      if (desc->h_seg_w[i] != 1.0f) one_layer_segments = false;
+  }
+  p->unrot = desc->sender_k_rotated == 1;
+  p->rope = desc->theta_r > 0.0 || desc->h_inv_freq_r != nullptr;
+  p->gather = one_layer_segments && desc->align_mode != HF_ALIGN_OVERLAP_MEAN && !p->unrot;
   p->ws = static_cast<char*>(d_workspace);
   p->ws_bytes = workspace_bytes;
   p->lay = lay;
@@ -367,20 +451,35 @@ hf_status plan_build(const hf_plan_desc* desc, void* d_workspace, size_t workspa
   p->desc.r_tok_ptr = nullptr;
   p->desc.r_pos0 = nullptr;
   p->desc.h_r = nullptr;
+  p->desc.h_inv_freq_r = nullptr;
+  p->desc.h_inv_freq_s = nullptr;
+  p->desc.s_pos0 = nullptr;
+  p->desc.h_seg_layer = nullptr;
+  p->desc.h_seg_w = nullptr;
 
   std::memset(t, 0, sizeof(*t));
   t->L_r = desc->L_r;
   t->D_r = desc->D_r;
+  t->D_s = p->unrot ? desc->D_s : 0;
   t->n_req = desc->n_req;
   build_layer_table(*desc, t->segs);
   for (int i = 0; i < 2 * desc->L_r; ++i) t->inv_r[i] = static_cast<float>(1.0 / desc->h_r[i]);
   // inv_freq_i = fp32(theta^(-2i/D)) evaluated in double precision
+  // (or the caller's table)
   for (int i = 0; i < desc->D_r / 2; ++i)
-    t->inv_freq[i] = desc->theta_r > 0.0
+    t->inv_freq[i] = desc->h_inv_freq_r ? desc->h_inv_freq_r[i]
+                     : desc->theta_r > 0.0
                          ? static_cast<float>(std::pow(desc->theta_r, -(2.0 * i) / desc->D_r))
                          : 0.0f;
+  if (p->unrot)
+    for (int i = 0; i < desc->D_s / 2; ++i)
+      t->inv_freq_s[i] = desc->h_inv_freq_s
+                             ? desc->h_inv_freq_s[i]
+                             : static_cast<float>(std::pow(desc->theta_s, -(2.0 * i) / desc->D_s));
   for (int q = 0; q <= desc->n_req; ++q) t->r_tok_ptr[q] = desc->r_tok_ptr[q];
   for (int q = 0; q < desc->n_req; ++q) t->r_pos0[q] = desc->r_pos0 ? desc->r_pos0[q] : 0;
+  for (int q = 0; q <= desc->n_req; ++q) t->s_tok_ptr[q] = desc->s_tok_ptr[q];
+  for (int q = 0; q < desc->n_req; ++q) t->s_pos0[q] = desc->s_pos0 ? desc->s_pos0[q] : 0;
   return launch_plan_kernels(p, *t, stream);
 }
 

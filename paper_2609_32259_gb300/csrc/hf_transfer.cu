@@ -60,6 +60,8 @@ struct XferParams {
   const float* inv_r;
   const LayerSegs* segs;
   const float* inv_freq;
+  const float* inv_freq_s;  // sender RoPE (rotated sender keys)
+  const int32_t* spos;      // sender position of every sender token (rotated sender keys)
   const float* knorm_w;
   const int32_t* row_ptr;
   const int32_t* col;
@@ -75,7 +77,7 @@ struct XferParams {
   int L_r, d_s, d_r, D_r;
   int n_kb, atoms_per_seg, last_atoms, BN, n_tiles_n, groups;  // n_kb: stages per tile
   int stages_a, stages_b, lag;  // A ring, B ring, cp.async groups in flight per loader
-  int rope, paged, knorm;
+  int rope, paged, knorm, unrot, D_s;
   float knorm_eps;
   uint32_t idesc;
 };
@@ -227,6 +229,100 @@ __device__ __forceinline__ int find_row(const int32_t* srun, int nrows, int j) {
   return lo;
 }
 
+// One 128-byte atom of operand row t for the builder path: features
+// [kin*kBK, (kin+1)*kBK) of segment `seg`, i.e. sum over the segment's
+// sender layers (weight om) and the row's CSR entries (weight w) of the
+// sender rows, accumulated in fp32 and rounded once into the swizzled layout.
+template <typename T>
+__device__ __forceinline__ void build_atom(const XferParams& P, const LayerSegs& segs, int seg,
+                                           int kin, int c, int e0, int e1, uint8_t* atom, int t) {
+  constexpr int kBK = Elem<T>::kBK;
+  constexpr int kPerChunk = 16 / sizeof(T);
+  const T* sender = reinterpret_cast<const T*>(P.sender);
+  float acc[kBK];
+#pragma unroll
+  for (int i = 0; i < kBK; ++i) acc[i] = 0.f;
+  for (int ti = 0; ti < segs.n_terms[seg]; ++ti) {
+    const int tl = segs.layer[seg][ti];
+    const float om = segs.w[seg][ti];
+    const T* base = sender + (static_cast<int64_t>(tl * 2 + c) * P.T_s) * P.d_s + kin * kBK;
+    for (int e = e0; e < e1; ++e) {
+      const int k = P.col[e];
+      if (k < 0 || k >= P.T_s) continue;  // flagged at plan creation
+      const float wt = om * P.w[e];
+      const uint4* src = reinterpret_cast<const uint4*>(base + static_cast<int64_t>(k) * P.d_s);
+      uint4 x[8];
+#pragma unroll
+      for (int k2 = 0; k2 < 8; ++k2) x[k2] = __ldg(src + k2);
+#pragma unroll
+      for (int k2 = 0; k2 < 8; ++k2) accum16(x[k2], wt, acc + k2 * kPerChunk, (const T*)nullptr);
+    }
+  }
+  uint8_t* dst = atom + t * 128;
+#pragma unroll
+  for (int k2 = 0; k2 < 8; ++k2)
+    *reinterpret_cast<uint4*>(dst + ((k2 ^ (t & 7)) << 4)) =
+        pack16(acc + k2 * kPerChunk, (const T*)nullptr);
+}
+
+// One stage (kAtoms atoms = whole heads of one segment) of operand row t
+// when the sender keys carry RoPE: every sender row is rotated back at its
+// own sender position before the CSR and layer weights are applied, pair
+// (i, i + D_s/2) of each head by the angle -pos * inv_freq_s_i:
+// (x, y) -> (x cos + y sin, y cos - x sin).  Lanes take 16-byte chunks of
+// pairs; the angle uses the same exact-product reduction as the epilogue.
+template <typename T>
+__device__ __forceinline__ void build_stage_unrotated(const XferParams& P, const LayerSegs& segs,
+                                                      int seg, int kin, int c, int e0, int e1,
+                                                      uint8_t* stage, int t) {
+  constexpr int kBK = Elem<T>::kBK;
+  constexpr int kPerChunk = 16 / sizeof(T);
+  const T* sender = reinterpret_cast<const T*>(P.sender);
+  const int hs = P.D_s / 2;
+  const int elem0 = kin * kBK;  // the stage's first feature within the segment
+  for (int pc = 0; pc < kBK / kPerChunk; ++pc) {
+    const int pi = pc * kPerChunk;                 // first pair of the chunk, within the stage
+    const int hh = pi / hs, i0 = pi - hh * hs;     // head within the stage, its frequency index
+    const int ex = hh * P.D_s + i0, ey = ex + hs;  // stage features of the pair halves
+    float f[kPerChunk], ax[kPerChunk], ay[kPerChunk];
+#pragma unroll
+    for (int i = 0; i < kPerChunk; ++i) {
+      f[i] = __ldg(P.inv_freq_s + i0 + i);
+      ax[i] = 0.f;
+      ay[i] = 0.f;
+    }
+    for (int ti = 0; ti < segs.n_terms[seg]; ++ti) {
+      const int tl = segs.layer[seg][ti];
+      const float om = segs.w[seg][ti];
+      const T* base = sender + (static_cast<int64_t>(tl * 2 + c) * P.T_s) * P.d_s + elem0;
+      for (int e = e0; e < e1; ++e) {
+        const int k = P.col[e];
+        if (k < 0 || k >= P.T_s) continue;  // flagged at plan creation
+        const float wt = om * P.w[e];
+        const T* row = base + static_cast<int64_t>(k) * P.d_s;
+        float x[kPerChunk], y[kPerChunk];
+#pragma unroll
+        for (int i = 0; i < kPerChunk; ++i) x[i] = y[i] = 0.f;
+        accum16(__ldg(reinterpret_cast<const uint4*>(row + ex)), 1.f, x, (const T*)nullptr);
+        accum16(__ldg(reinterpret_cast<const uint4*>(row + ey)), 1.f, y, (const T*)nullptr);
+        const int p = __ldg(P.spos + k);
+#pragma unroll
+        for (int i = 0; i < kPerChunk; ++i) {
+          float sn, cs;
+          rope_sincos(p, f[i], &sn, &cs);
+          ax[i] = fmaf(wt, fmaf(x[i], cs, y[i] * sn), ax[i]);
+          ay[i] = fmaf(wt, fmaf(y[i], cs, -x[i] * sn), ay[i]);
+        }
+      }
+    }
+    uint8_t* row_x = stage + (ex / kBK) * kAtomABytes + t * 128;
+    uint8_t* row_y = stage + (ey / kBK) * kAtomABytes + t * 128;
+    const int cx = (ex % kBK) / kPerChunk, cy = (ey % kBK) / kPerChunk;
+    *reinterpret_cast<uint4*>(row_x + ((cx ^ (t & 7)) << 4)) = pack16(ax, (const T*)nullptr);
+    *reinterpret_cast<uint4*>(row_y + ((cy ^ (t & 7)) << 4)) = pack16(ay, (const T*)nullptr);
+  }
+}
+
 // Arrival on the leader CTA's copy of a pair barrier (`bar` is the local
 // offset): a local arrive in the leader, a relaxed remote arrive in the
 // follower.  What is announced is complete and visible before the call.
@@ -324,7 +420,6 @@ template <typename T, bool kGather>
 __global__ void __launch_bounds__(kThreads, 1)
     transfer_kernel(const __grid_constant__ CUtensorMap tmap_w, const XferParams P) {
   constexpr int kBK = Elem<T>::kBK;
-  constexpr int kPerChunk = 16 / sizeof(T);  // elements per 16-byte chunk
   extern __shared__ __align__(1024) uint8_t smem[];
   if (smem_addr(smem) & 1023u) {  // the swizzled stages need 1024-byte alignment
     if (threadIdx.x == 0) atomicOr(P.status, HF_CHECK_INTERNAL);
@@ -653,8 +748,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         default: gather_rows<T, 5>(P, sA, full_a, empty_a, sAbort, t, lane, U, row0, total_tiles, tiles_per_lc, first_tile, tile_step); break;
       }
     } else {
-      // pooled CSR rows and/or blended sender layers: thread t owns tile row t
-      const T* sender = reinterpret_cast<const T*>(P.sender);
+      // pooled CSR rows, blended sender layers and/or rotated sender keys:
+      // thread t owns tile row t
       int stage = 0;
       uint32_t phase = 0;
       bool ok = true;
@@ -666,6 +761,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int u = min(m * kPairRows + row0 + t, U - 1);
         const int j0 = P.run_ptr[u];
         const int e0 = P.row_ptr[j0], e1 = P.row_ptr[j0 + 1];
+        const bool unrot_k = P.unrot && c == 0;
         int seg = 0, kin = 0;  // segment of the next atom, and the atom within it
         for (int kb = 0; kb < P.n_kb; ++kb) {
           if (!mbar_wait(smem_addr(&empty_a[stage]), phase ^ 1)) {
@@ -673,39 +769,24 @@ __global__ void __launch_bounds__(kThreads, 1)
             ok = false;
             break;
           }
-          const int na = kb == P.n_kb - 1 ? P.last_atoms : kAtoms;
-          for (int a = 0; a < na; ++a) {
-          float acc[kBK];
-#pragma unroll
-          for (int i = 0; i < kBK; ++i) acc[i] = 0.f;
-          for (int ti = 0; ti < segs.n_terms[seg]; ++ti) {
-            const int tl = segs.layer[seg][ti];
-            const float om = segs.w[seg][ti];
-            const T* base =
-                sender + (static_cast<int64_t>(tl * 2 + c) * P.T_s) * P.d_s + kin * kBK;
-            for (int e = e0; e < e1; ++e) {
-              const int k = P.col[e];
-              if (k < 0 || k >= P.T_s) continue;  // flagged at plan creation
-              const float wt = om * P.w[e];
-              const uint4* src =
-                  reinterpret_cast<const uint4*>(base + static_cast<int64_t>(k) * P.d_s);
-              uint4 x[8];
-#pragma unroll
-              for (int k2 = 0; k2 < 8; ++k2) x[k2] = __ldg(src + k2);
-#pragma unroll
-              for (int k2 = 0; k2 < 8; ++k2)
-                accum16(x[k2], wt, acc + k2 * kPerChunk, (const T*)nullptr);
+          uint8_t* st = sA + stage * kStageABytes;
+          if (unrot_k) {
+            // the stage is whole heads of one segment (checked at plan creation)
+            build_stage_unrotated<T>(P, segs, seg, kin, c, e0, e1, st, t);
+            kin += kAtoms;
+            if (kin == P.atoms_per_seg) {
+              kin = 0;
+              ++seg;
             }
-          }
-          uint8_t* dst = sA + stage * kStageABytes + a * kAtomABytes + t * 128;
-#pragma unroll
-          for (int k2 = 0; k2 < 8; ++k2)
-            *reinterpret_cast<uint4*>(dst + ((k2 ^ (t & 7)) << 4)) =
-                pack16(acc + k2 * kPerChunk, (const T*)nullptr);
-          if (++kin == P.atoms_per_seg) {
-            kin = 0;
-            ++seg;
-          }
+          } else {
+            const int na = kb == P.n_kb - 1 ? P.last_atoms : kAtoms;
+            for (int a = 0; a < na; ++a) {
+              build_atom<T>(P, segs, seg, kin, c, e0, e1, st + a * kAtomABytes, t);
+              if (++kin == P.atoms_per_seg) {
+                kin = 0;
+                ++seg;
+              }
+            }
           }
           fence_proxy_async_smem();
           __syncwarp();
@@ -876,7 +957,11 @@ hf_status launch_transfer(hf_plan_s* p, const void* sender, void* receiver, cuda
   P.BN = p->BN;
   P.n_tiles_n = p->d_r / p->BN;
   pick_rings(p->BN, &P.stages_a, &P.stages_b, &P.lag);
-  P.rope = d.theta_r > 0.0 ? 1 : 0;
+  P.rope = p->rope ? 1 : 0;
+  P.unrot = p->unrot ? 1 : 0;
+  P.D_s = d.D_s;
+  P.inv_freq_s = reinterpret_cast<const float*>(ws + p->lay.inv_freq_s);
+  P.spos = reinterpret_cast<const int32_t*>(ws + p->lay.spos);
   P.paged = d.paged ? 1 : 0;
   P.knorm = d.d_knorm_w ? 1 : 0;
   P.knorm_eps = d.knorm_eps;

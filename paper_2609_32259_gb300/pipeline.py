@@ -29,12 +29,16 @@ class TransferJob:
     b:        device fp32 [L_r, 2, d_r];  r: host [L_r, 2]
     s_end / r_end: host int32 character-end offsets; s_tok_ptr / r_tok_ptr:
               host request pointers
+    desc_options: the optional descriptor fields of binding.Desc
+              (inv_freq_r, sender_k_rotated, theta_s, inv_freq_s, s_pos0,
+              seg_layer, seg_w)
     """
 
     def __init__(self, *, L_s, H_s, D_s, L_r, H_r, D_r, dtype: str, align_mode: str,
                  layer_mode: str, s_tok_ptr, r_tok_ptr, s_end, r_end, sender, W, b, r,
                  theta_r: float, r_pos0=None, knorm_w=None, knorm_eps=1e-6,
-                 paged: Optional[PagedCache] = None, device="cuda", receiver=None):
+                 paged: Optional[PagedCache] = None, device="cuda", receiver=None,
+                 **desc_options):
         self.device = torch.device(device)
         self.s_tok_ptr = np.asarray(s_tok_ptr, np.int32)
         self.r_tok_ptr = np.asarray(r_tok_ptr, np.int32)
@@ -76,7 +80,7 @@ class TransferJob:
             block_size=paged.block_size if paged else 16,
             n_blocks=paged.n_blocks if paged else 0,
             max_blocks_per_req=paged.block_table.shape[1] if paged else 0,
-            d_block_table=self.block_table)
+            d_block_table=self.block_table, **desc_options)
         ws = B.plan_workspace_size(self.desc)
         self.workspace = torch.empty(ws, dtype=torch.uint8, device=self.device)
         self.plan: Optional[B.Plan] = None
@@ -124,8 +128,12 @@ class TransferJob:
 
 
 def job_from_workload(w, tok, sender, W, b, r, *, paged=None, knorm_w=None, r_pos0=None,
-                      device="cuda", receiver=None) -> TransferJob:
-    """TransferJob for a workloads.Workload and its generated inputs."""
+                      device="cuda", receiver=None, **desc_options) -> TransferJob:
+    """TransferJob for a workloads.Workload and its generated inputs; the
+    workload's optional descriptor fields are passed on."""
+    from . import workloads as W_
+    opts = W_.desc_options(w)
+    opts.update(desc_options)
     pc = None
     if paged is not None:
         pc = PagedCache(paged.block_table, paged.n_blocks, w.block_size)
@@ -134,4 +142,4 @@ def job_from_workload(w, tok, sender, W, b, r, *, paged=None, knorm_w=None, r_po
                        s_tok_ptr=tok.s_tok_ptr, r_tok_ptr=tok.r_tok_ptr, s_end=tok.s_end,
                        r_end=tok.r_end, sender=sender, W=W, b=b, r=r, theta_r=w.theta_r,
                        r_pos0=r_pos0, knorm_w=knorm_w, paged=pc, device=device,
-                       receiver=receiver)
+                       receiver=receiver, **opts)

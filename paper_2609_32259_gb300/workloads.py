@@ -52,7 +52,7 @@ class Workload:
     mean_r: float = 3.6                # receiver characters per token
     dtype: str = "bf16"                # "bf16" or "f32"
     align_mode: str = "ta"             # "ta", "overlap_mean", "same_index"
-    layer_mode: str = "paper3"         # "paper3" or "interp"
+    layer_mode: str = "paper3"         # "paper3", "interp" or "explicit"
     paged: bool = False
     block_size: int = 16
     spare_frac: float = 0.10
@@ -62,6 +62,12 @@ class Workload:
     channel_scales: bool = True
     knorm: bool = False
     r_pos0: Optional[Tuple[int, ...]] = None
+    # optional descriptor fields
+    seg_layer: Optional[tuple] = None  # explicit layer table [L_r][n_seg][n_terms]
+    seg_w: Optional[tuple] = None
+    sender_k_rotated: bool = False     # sender keys stored with RoPE (base theta_s)
+    s_pos0: Optional[Tuple[int, ...]] = None
+    rope_table: bool = False           # receiver RoPE from a caller table (inv_freq_r_table)
 
     @property
     def d_s(self) -> int:
@@ -73,6 +79,8 @@ class Workload:
 
     @property
     def n_seg(self) -> int:
+        if self.layer_mode == "explicit":
+            return len(self.seg_layer[0])
         return 3 if self.layer_mode == "paper3" else 1
 
     @property
@@ -250,6 +258,42 @@ def knorm_weight(w: Workload) -> Optional[np.ndarray]:
 
 def r_pos0(w: Workload) -> Optional[np.ndarray]:
     return None if w.r_pos0 is None else np.asarray(w.r_pos0, np.int32)
+
+
+def s_pos0(w: Workload) -> Optional[np.ndarray]:
+    return None if w.s_pos0 is None else np.asarray(w.s_pos0, np.int32)
+
+
+def inv_freq_r_table(w: Workload) -> Optional[np.ndarray]:
+    """A caller-supplied receiver RoPE frequency table (stand-in for a scaled
+    RoPE variant): D_r/2 fp32 values log-uniform in [1e-6, 1], descending."""
+    if not w.rope_table:
+        return None
+    rng = np.random.default_rng([w.seed, 808])
+    return np.sort(10.0 ** rng.uniform(-6.0, 0.0, size=w.D_r // 2))[::-1].astype(np.float32)
+
+
+def explicit_table(L_s: int, L_r: int, n_seg: int, n_terms: int, seed: int):
+    """A seeded explicit layer table: random sender layers and weights in
+    [-1, 1] (any structure the descriptor allows)."""
+    rng = np.random.default_rng([seed, 909])
+    layers = rng.integers(0, L_s, size=(L_r, n_seg, n_terms))
+    weights = rng.uniform(-1.0, 1.0, size=(L_r, n_seg, n_terms)).astype(np.float32)
+    return (tuple(tuple(tuple(int(x) for x in t) for t in s) for s in layers),
+            tuple(tuple(tuple(float(x) for x in t) for t in s) for s in weights))
+
+
+def desc_options(w: Workload) -> dict:
+    """The optional descriptor fields a workload asks for."""
+    opts = {}
+    if w.layer_mode == "explicit":
+        opts.update(seg_layer=np.asarray(w.seg_layer, np.int32),
+                    seg_w=np.asarray(w.seg_w, np.float32))
+    if w.sender_k_rotated:
+        opts.update(sender_k_rotated=True, theta_s=w.theta_s, s_pos0=s_pos0(w))
+    if w.rope_table:
+        opts.update(inv_freq_r=inv_freq_r_table(w))
+    return opts
 
 
 @dataclass

@@ -76,8 +76,18 @@ class Case:
             self.job.receiver.fill_(sentinel)
         self.csr = O.alignment_csr(w.align_mode, self.tok.s_tok_ptr, self.tok.r_tok_ptr,
                                    self.tok.s_end, self.tok.r_end)
-        self.segs = O.layer_segments(w.layer_mode, w.L_s, w.L_r)
+        if w.layer_mode == "explicit":
+            self.segs = O.explicit_segments(w.seg_layer, np.asarray(w.seg_w, np.float32))
+        else:
+            self.segs = O.layer_segments(w.layer_mode, w.L_s, w.L_r)
         self.pos = O.receiver_positions(self.tok.r_tok_ptr, self.r_pos0)
+        table = W.inv_freq_r_table(w)
+        self.inv_freq_r = (O.rope_inv_freq(w.theta_r, w.D_r) if table is None
+                           else table.astype(np.float64))
+        self.sender_rope = None
+        if w.sender_k_rotated:
+            self.sender_rope = (O.sender_positions(self.tok.s_tok_ptr, W.s_pos0(w)),
+                                O.rope_inv_freq(w.theta_s, w.D_s), w.H_s)
 
     def run(self):
         self.job.step()
@@ -110,9 +120,9 @@ class Case:
     def oracle(self, layers, rows, roles=(0, 1)):
         return O.transfer(RowFetcher(self.sender), self.csr, self.segs, MapFetcher(self.Wm),
                           self.b.cpu().numpy(), self.r, H_r=self.w.H_r, D_r=self.w.D_r,
-                          pos=self.pos, inv_freq_r=O.rope_inv_freq(self.w.theta_r, self.w.D_r),
+                          pos=self.pos, inv_freq_r=self.inv_freq_r,
                           knorm_g=self.knorm_w, knorm_eps=1e-6, layers=layers, rows=rows,
-                          roles=roles)
+                          roles=roles, sender_rope=self.sender_rope)
 
     def check_parity(self, layers=None, rows=None, rel_tol=REL_FRO_TOL, abs_tol=MAX_ABS_TOL):
         layers = list(range(self.w.L_r)) if layers is None else list(layers)

@@ -63,6 +63,16 @@ def _desc(B, **over):
     (dict(H_r=3, D_r=32), 2),                          # d_R not a multiple of 128
     (dict(paged=True, block_size=16, n_blocks=0), 1),  # paged layout incomplete
     (dict(d_W=None), 1),
+    # optional fields
+    (dict(layer_mode="explicit", seg_layer=np.zeros((6, 4, 1)), seg_w=1.0), 1),   # n_seg > 3
+    (dict(layer_mode="explicit", seg_layer=np.zeros((6, 2, 3)), seg_w=1.0), 1),   # n_terms > 2
+    (dict(layer_mode="explicit", seg_layer=np.full((6, 2, 1), 4), seg_w=1.0), 1),  # layer >= L_s
+    (dict(layer_mode="explicit", seg_layer=np.zeros((6, 1, 2)), seg_w=np.nan), 1),
+    (dict(layer_mode="explicit"), 1),                                             # no table
+    (dict(sender_k_rotated=True), 1),                  # no theta_s and no sender table
+    (dict(sender_k_rotated=True, theta_s=1e4, D_s=256, H_s=1), 2),  # head wider than a stage
+    (dict(sender_k_rotated=True, theta_s=1e4, D_s=64, H_s=1), 2),   # d_S = 64: not whole stages
+    (dict(inv_freq_r=np.full(16, np.inf)), 1),
 ])
 def test_plan_create_rejects(B, over, status):
     d = _desc(B, **over)
@@ -120,3 +130,28 @@ def test_binding_fails_loudly_without_library(tmp_path, monkeypatch):
     monkeypatch.setattr(binding, "_LIB", None)
     with pytest.raises(RuntimeError, match="no CPU fallback"):
         binding.lib()
+
+
+def test_optional_fields_validate(B):
+    """The optional descriptor fields pass host validation when consistent
+    (a failure after validation is a CUDA error on this device-less host, or
+    success where a GPU is present)."""
+    ok = [dict(layer_mode="explicit", seg_layer=np.zeros((6, 2, 2)), seg_w=0.5),
+          dict(sender_k_rotated=True, theta_s=5e5, s_pos0=[3]),
+          dict(sender_k_rotated=True, inv_freq_s=np.ones(32)),
+          dict(inv_freq_r=np.linspace(1.0, 1e-3, 16), theta_r=0.0)]
+    for over in ok:
+        d = _desc(B, **over)
+        need = B.plan_workspace_size(d)
+        h = ctypes.c_void_p(0)
+        st = B.lib().hf_plan_create(ctypes.byref(d.c), ctypes.c_void_p(256), need, None,
+                                    ctypes.byref(h))
+        assert st in (B.HF_OK, B.HF_ERR_CUDA), (over, st, B.lib().hf_last_error())
+        if st == B.HF_OK:
+            B.lib().hf_plan_destroy(h)
+
+
+def test_rotated_sender_workspace_holds_sender_positions(B):
+    a = B.plan_workspace_size(_desc(B, s_tok_ptr=[0, 50000]))
+    b = B.plan_workspace_size(_desc(B, s_tok_ptr=[0, 50000], sender_k_rotated=True, theta_s=1e4))
+    assert b - a >= 4 * 50000 - 256

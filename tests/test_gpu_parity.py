@@ -163,7 +163,27 @@ EDGE = {
     "head64": lambda: W.llama_to_ministral(333).with_(L_s=3, L_r=2, H_r=4, D_r=64),
     "batched_small_paged": lambda: W.qwen25_to_llama_batched(n_req=5, lo=1, hi=300, seed=9)
     .with_(L_s=3, L_r=3),
+    # optional descriptor fields
+    "rotated_sender_ta": lambda: W.llama_to_ministral(700).with_(
+        L_s=4, L_r=4, sender_k_rotated=True, s_pos0=(37,), r_pos0=(100,)),
+    "rotated_sender_overlap_interp_f32": lambda: W.tiny().with_(sender_k_rotated=True),
+    "rotated_sender_batched_paged": lambda: W.qwen25_to_llama_batched(
+        n_req=3, lo=50, hi=400, seed=5).with_(L_s=3, L_r=3, sender_k_rotated=True,
+                                              s_pos0=(0, 1000, 50000)),
+    "explicit_two_terms": lambda: _explicit(W.llama_to_ministral(500).with_(L_s=5, L_r=3),
+                                            n_seg=2, n_terms=2),
+    "explicit_one_layer_segments": lambda: _explicit(
+        W.llama_to_ministral(400).with_(L_s=6, L_r=3), n_seg=3, n_terms=1, unit=True),
+    "rope_table": lambda: W.llama_to_ministral(600).with_(L_s=4, L_r=3, rope_table=True,
+                                                          r_pos0=(5000,)),
 }
+
+
+def _explicit(w, n_seg, n_terms, unit=False):
+    layers, weights = W.explicit_table(w.L_s, w.L_r, n_seg, n_terms, seed=w.seed + 1)
+    if unit:  # every segment one sender layer with weight 1: the copy-only operand path
+        weights = tuple(tuple(tuple(1.0 for _ in t) for t in s) for s in weights)
+    return w.with_(layer_mode="explicit", seg_layer=layers, seg_w=weights)
 
 
 @pytest.mark.parametrize("name", sorted(EDGE))
