@@ -19,6 +19,7 @@
  *   hf_plan_workspace_size    bytes of device workspace the plan needs
  *   hf_plan_create            validates, builds per-transfer metadata (device)
  *   hf_transfer               one kernel launch: receiver cache <- Phi(sender)
+ *     (or hf_transfer_host    the same with both caches in host memory)
  *   hf_plan_destroy
  *
  * General rules:
@@ -246,7 +247,35 @@ hf_status hf_plan_create(const hf_plan_desc* desc, void* d_workspace, size_t wor
 hf_status hf_transfer(hf_plan plan, const void* sender_kv, void* receiver_kv,
                       hf_stream_t stream);
 
-/* Frees the plan's host memory.  Does not touch the workspace. */
+/*
+ * hf_transfer_host — the transfer for caches held in page-locked host
+ * memory, with the host<->device copies overlapped with the computation.
+ * The paper moves the sender payload GPU to GPU; this entry point serves
+ * callers whose caches live on the host.
+ * h_sender_kv:   page-locked host [L_s][2][T_s][H_s][D_s] (cudaHostAlloc or
+ *                cudaHostRegister), the layout hf_transfer takes.
+ * d_sender_kv:   device buffer of the same size: the sender layers are
+ *                copied there (only layers 0 .. the highest one the layer
+ *                table reads).
+ * d_receiver_kv: device receiver cache, as for hf_transfer.
+ * h_receiver_kv: page-locked host buffer of the receiver cache's size
+ *                (contiguous or paged layout); every receiver layer is
+ *                copied back whole (a paged pool's untouched blocks too).
+ * n_groups:      receiver layers are processed in n_groups consecutive
+ *                groups (1 .. L_r; 0 = L_r, one per layer): group g's sender
+ *                layers are copied in, its layers computed on `stream`,
+ *                then copied out while later groups proceed.
+ * The call is asynchronous: work starts after earlier work on `stream`, and
+ * `stream` is ordered after the last copy out.  Copies run on two streams
+ * the plan creates on first use (on the current device; released by
+ * hf_plan_destroy).  One call at a time per plan.
+ */
+hf_status hf_transfer_host(hf_plan plan, const void* h_sender_kv, void* d_sender_kv,
+                           void* d_receiver_kv, void* h_receiver_kv, int32_t n_groups,
+                           hf_stream_t stream);
+
+/* Frees the plan's host memory and its copy streams.  Does not touch the
+   workspace. */
 hf_status hf_plan_destroy(hf_plan plan);
 
 /* Synchronises `stream` and returns the plan's device status bits in

@@ -37,7 +37,7 @@ CHECK_BITS = {
 
 EXPORTED = ("hf_align_build", "hf_plan_workspace_size", "hf_plan_create", "hf_transfer",
             "hf_plan_destroy", "hf_plan_device_status", "hf_plan_distinct_rows",
-            "hf_status_string", "hf_last_error", "hf_transfer_noalloc")
+            "hf_status_string", "hf_last_error", "hf_transfer_noalloc", "hf_transfer_host")
 
 _p = ctypes.c_void_p
 _i32p = ctypes.POINTER(ctypes.c_int32)
@@ -95,6 +95,8 @@ def lib() -> ctypes.CDLL:
         L.hf_plan_distinct_rows.argtypes = [_p, _p, _i32p]
         L.hf_transfer_noalloc.argtypes = [ctypes.POINTER(PlanDesc), _p, _p, _p]
         L.hf_transfer_noalloc.restype = ctypes.c_int
+        L.hf_transfer_host.argtypes = [_p, _p, _p, _p, _p, ctypes.c_int32, _p]
+        L.hf_transfer_host.restype = ctypes.c_int
         L.hf_status_string.argtypes = [ctypes.c_int]
         L.hf_status_string.restype = ctypes.c_char_p
         L.hf_last_error.argtypes = []
@@ -237,6 +239,15 @@ def plan_create(desc: Desc, workspace, stream=None) -> Plan:
 def transfer(plan: Plan, sender_kv, receiver_kv, stream=None) -> None:
     _check(lib().hf_transfer(plan.handle, _dptr(sender_kv), _dptr(receiver_kv), _stream(stream)),
            "hf_transfer")
+
+
+def transfer_host(plan: Plan, h_sender_kv, d_sender_kv, d_receiver_kv, h_receiver_kv,
+                  n_groups: int = 0, stream=None) -> None:
+    """hf_transfer_host: caches in page-locked host memory (torch tensors made
+    with pin_memory=True), copies overlapped with the computation."""
+    _check(lib().hf_transfer_host(plan.handle, _dptr(h_sender_kv), _dptr(d_sender_kv),
+                                  _dptr(d_receiver_kv), _dptr(h_receiver_kv), int(n_groups),
+                                  _stream(stream)), "hf_transfer_host")
 
 
 def transfer_noalloc(desc: Desc, sender_kv, receiver_kv, stream=None) -> None:

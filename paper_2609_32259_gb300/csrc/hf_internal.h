@@ -79,6 +79,12 @@ struct hf_plan_s {
   size_t ws_bytes;
   hf::WorkspaceLayout lay;
   int32_t s_tok_ptr_last;
+  int32_t max_sender_layer[hf::kMaxLayersR];  // highest sender layer each receiver layer reads
+  // hf_transfer_host: copy streams and events, created on first use
+  int aux_device = -1;
+  cudaStream_t s_h2d = nullptr, s_d2h = nullptr;
+  cudaEvent_t* events = nullptr;
+  int n_events = 0;
 };
 
 namespace hf {
@@ -90,7 +96,9 @@ int device_sm_count();
 hf_status launch_plan_kernels(hf_plan_s* p, const PlanTables& tables, cudaStream_t stream);
 hf_status plan_build(const hf_plan_desc* desc, void* d_workspace, size_t workspace_bytes,
                      cudaStream_t stream, hf_plan_s* p, PlanTables* t);
-hf_status launch_transfer(hf_plan_s* p, const void* sender, void* receiver, cudaStream_t stream);
+// One transfer-kernel launch over receiver layers [l_begin, l_end) (l_end < 0: all).
+hf_status launch_transfer(hf_plan_s* p, const void* sender, void* receiver, cudaStream_t stream,
+                          int l_begin = 0, int l_end = -1);
 
 }  // namespace hf
 

@@ -3,6 +3,7 @@
 // and the per-transfer device metadata (receiver positions and destination
 // rows, sender positions for rotated sender keys, runs of identical
 // alignment rows).  Also the error-reporting helpers of the ABI.
+#include <algorithm>
 #include <cmath>
 #include <cstdio>
 #include <cstdlib>
@@ -463,6 +464,12 @@ hf_status plan_build(const hf_plan_desc* desc, void* d_workspace, size_t workspa
   t->D_s = p->unrot ? desc->D_s : 0;
   t->n_req = desc->n_req;
   build_layer_table(*desc, t->segs);
+  for (int l = 0; l < desc->L_r; ++l) {
+    int mx = 0;
+    for (int k = 0; k < t->segs[l].n_seg; ++k)
+      for (int i = 0; i < t->segs[l].n_terms[k]; ++i) mx = std::max(mx, t->segs[l].layer[k][i]);
+    p->max_sender_layer[l] = mx;
+  }
   for (int i = 0; i < 2 * desc->L_r; ++i) t->inv_r[i] = static_cast<float>(1.0 / desc->h_r[i]);
   // inv_freq_i = fp32(theta^(-2i/D)) evaluated in double precision
   // (or the caller's table)
@@ -506,6 +513,16 @@ extern "C" hf_status hf_plan_create(const hf_plan_desc* desc, void* d_workspace,
 }
 
 extern "C" hf_status hf_plan_destroy(hf_plan plan) {
+  if (plan && (plan->s_h2d || plan->events)) {
+    int cur = 0;
+    cudaGetDevice(&cur);
+    cudaSetDevice(plan->aux_device);
+    if (plan->s_h2d) cudaStreamDestroy(plan->s_h2d);
+    if (plan->s_d2h) cudaStreamDestroy(plan->s_d2h);
+    for (int i = 0; i < plan->n_events; ++i) cudaEventDestroy(plan->events[i]);
+    delete[] plan->events;
+    cudaSetDevice(cur);
+  }
   delete plan;
   return HF_OK;
 }

@@ -75,6 +75,7 @@ struct XferParams {
   int64_t T_s;        // sender rows per (layer, role)
   int64_t recv_rows;  // receiver rows per (layer, role) in receiver_kv
   int L_r, d_s, d_r, D_r;
+  int l0, n_l;  // receiver layers [l0, l0 + n_l) of this launch
   int n_kb, atoms_per_seg, last_atoms, BN, n_tiles_n, groups;  // n_kb: stages per tile
   int stages_a, stages_b, lag;  // A ring, B ring, cp.async groups in flight per loader
   int rope, paged, knorm, unrot, D_s;
@@ -93,16 +94,17 @@ struct Elem<float> {
   static constexpr int kBK = 32;
 };
 
-// Tile order: role-major, then receiver layer, then 128-row block, then
-// column block.  Consecutive receiver layers of one role share most of their
-// Eq. 1 sender layers, so their A rows are still in L2.  lc = 2 * l + c
-// indexes the maps, biases and receiver cache.
-__device__ __forceinline__ void decode_tile(int tile, int tiles_per_lc, int n_tiles_n, int L_r,
-                                            int* lc, int* m, int* n) {
+// Tile order over the launch's receiver layers [l0, l0 + n_l): role-major,
+// then receiver layer, then 256-row pair block, then column block.
+// Consecutive receiver layers of one role share most of their Eq. 1 sender
+// layers, so their A rows are still in L2.  lc = 2 * l + c indexes the maps,
+// biases and receiver cache.
+__device__ __forceinline__ void decode_tile(int tile, int tiles_per_lc, int n_tiles_n, int n_l,
+                                            int l0, int* lc, int* m, int* n) {
   const int ord = tile / tiles_per_lc;
   const int rem = tile - ord * tiles_per_lc;
-  const int c = ord >= L_r ? 1 : 0;
-  *lc = 2 * (ord - c * L_r) + c;
+  const int c = ord >= n_l ? 1 : 0;
+  *lc = 2 * (l0 + ord - c * n_l) + c;
   *m = rem / n_tiles_n;
   *n = rem - *m * n_tiles_n;
 }
@@ -355,7 +357,7 @@ __device__ __forceinline__ void gather_rows(const XferParams& P, uint8_t* sA, ui
   bool ok = true;
   for (int tile = first_tile; tile < total_tiles && ok; tile += tile_step) {
     int lc, m, n;
-    decode_tile(tile, tiles_per_lc, P.n_tiles_n, P.L_r, &lc, &m, &n);
+    decode_tile(tile, tiles_per_lc, P.n_tiles_n, P.n_l, P.l0, &lc, &m, &n);
     const int l = lc >> 1, c = lc & 1;
     // element offset of each segment's sender layer/role block, for the whole tile
     int64_t seg_base[kMaxSeg];
@@ -485,7 +487,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int U = *P.n_distinct;
   const int m_tiles = (U + kPairRows - 1) / kPairRows;
   const int tiles_per_lc = m_tiles * P.n_tiles_n;
-  const int total_tiles = 2 * P.L_r * tiles_per_lc;
+  const int total_tiles = 2 * P.n_l * tiles_per_lc;
 
   if (warp == 0) {
     // ------------------------------------------------------------ map tiles
@@ -496,7 +498,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       for (int tile = first_tile; tile < total_tiles && ok; tile += tile_step) {
         int lc, m, n;
-        decode_tile(tile, tiles_per_lc, P.n_tiles_n, P.L_r, &lc, &m, &n);
+        decode_tile(tile, tiles_per_lc, P.n_tiles_n, P.n_l, P.l0, &lc, &m, &n);
         for (int kb = 0; kb < P.n_kb; ++kb) {
           if (!mbar_wait(smem_addr(&empty_b[stage]), phase ^ 1)) {
             raise_timeout(P, sAbort);
@@ -620,7 +622,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t acc_phase = 0;
     for (int tile = first_tile; tile < total_tiles; tile += tile_step) {
       int lc, m, n;
-      decode_tile(tile, tiles_per_lc, P.n_tiles_n, P.L_r, &lc, &m, &n);
+      decode_tile(tile, tiles_per_lc, P.n_tiles_n, P.n_l, P.l0, &lc, &m, &n);
       const int c = lc & 1;
       if (!mbar_wait(smem_addr(&tfull[acc]), acc_phase)) {
         raise_timeout(P, sAbort);
@@ -755,7 +757,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       for (int tile = first_tile; tile < total_tiles && ok; tile += tile_step) {
         int lc, m, n;
-        decode_tile(tile, tiles_per_lc, P.n_tiles_n, P.L_r, &lc, &m, &n);
+        decode_tile(tile, tiles_per_lc, P.n_tiles_n, P.n_l, P.l0, &lc, &m, &n);
         const int l = lc >> 1, c = lc & 1;
         const LayerSegs segs = P.segs[l];
         const int u = min(m * kPairRows + row0 + t, U - 1);
@@ -914,9 +916,11 @@ hf_status launch_typed(const CUtensorMap& mw, const XferParams& P, int64_t max_p
 
 }  // namespace
 
-hf_status launch_transfer(hf_plan_s* p, const void* sender, void* receiver, cudaStream_t stream) {
+hf_status launch_transfer(hf_plan_s* p, const void* sender, void* receiver, cudaStream_t stream,
+                          int l_begin, int l_end) {
   const hf_plan_desc& d = p->desc;
-  if (p->T_r == 0) return HF_OK;
+  if (l_end < 0) l_end = d.L_r;
+  if (p->T_r == 0 || l_end <= l_begin) return HF_OK;
   const bool f32 = d.dtype == HF_F32;
   const int esize = f32 ? 4 : 2;
   const int bk = 128 / esize;
@@ -947,6 +951,8 @@ hf_status launch_transfer(hf_plan_s* p, const void* sender, void* receiver, cuda
   P.T_s = p->T_s;
   P.recv_rows = d.paged ? static_cast<int64_t>(d.n_blocks) * d.block_size : p->T_r;
   P.L_r = d.L_r;
+  P.l0 = l_begin;
+  P.n_l = l_end - l_begin;
   P.d_s = p->d_s;
   P.d_r = p->d_r;
   P.D_r = d.D_r;
@@ -968,7 +974,7 @@ hf_status launch_transfer(hf_plan_s* p, const void* sender, void* receiver, cuda
   P.idesc = make_idesc(f32 ? 2u : 1u, kPairRows, p->BN);
   const size_t smem = smem_bytes(p->BN, P.stages_a, P.stages_b);
   const int64_t max_pair_tiles =
-      2LL * d.L_r * ((p->T_r + kPairRows - 1) / kPairRows) * static_cast<int64_t>(P.n_tiles_n);
+      2LL * P.n_l * ((p->T_r + kPairRows - 1) / kPairRows) * static_cast<int64_t>(P.n_tiles_n);
   if (f32)
     return p->gather ? launch_typed<float, true>(mw, P, max_pair_tiles, smem, stream)
                      : launch_typed<float, false>(mw, P, max_pair_tiles, smem, stream);

@@ -100,6 +100,12 @@ class TransferJob:
         B.transfer(self.plan, self.sender if sender is None else sender,
                    self.receiver if receiver is None else receiver, stream)
 
+    def transfer_host(self, h_sender, h_receiver, n_groups=0, stream=None) -> None:
+        """The transfer from/to page-locked host caches; self.sender and
+        self.receiver serve as the device buffers."""
+        B.transfer_host(self.plan, h_sender, self.sender, self.receiver, h_receiver, n_groups,
+                        stream)
+
     def step(self, stream=None) -> None:
         """The whole hot path: alignment CSR, plan metadata, fused map."""
         self.align(stream)
