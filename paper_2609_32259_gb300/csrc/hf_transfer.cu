@@ -94,17 +94,25 @@ struct Elem<float> {
   static constexpr int kBK = 32;
 };
 
-// Tile order over the launch's receiver layers [l0, l0 + n_l): role-major,
-// then receiver layer, then 256-row pair block, then column block.
-// Consecutive receiver layers of one role share most of their Eq. 1 sender
-// layers, so their A rows are still in L2.  lc = 2 * l + c indexes the maps,
+// Tiles of a launch over receiver layers [l0, l0 + n_l): a slot is (layer,
+// 256-row pair block, column block), ordered layer-major so that the slots
+// in flight share their Eq. 1 sender rows and maps in L2; tile = 2 * slot + c
+// covers role c of the slot.  With at least two slots per CTA pair, a pair
+// takes slots first, first + step, ... and both roles of each slot in turn,
+// so that its key tiles (rotated epilogue) and value tiles (copy epilogue)
+// alternate; with fewer, it takes tiles first, first + step, ... (the two
+// roles of a slot on different pairs).  lc = 2 * l + c indexes the maps,
 // biases and receiver cache.
-__device__ __forceinline__ void decode_tile(int tile, int tiles_per_lc, int n_tiles_n, int n_l,
-                                            int l0, int* lc, int* m, int* n) {
-  const int ord = tile / tiles_per_lc;
-  const int rem = tile - ord * tiles_per_lc;
-  const int c = ord >= n_l ? 1 : 0;
-  *lc = 2 * (l0 + ord - c * n_l) + c;
+__device__ __forceinline__ int tile_of(int seq, int first, int step, bool by_slot) {
+  return by_slot ? 2 * (first + (seq >> 1) * step) + (seq & 1) : first + seq * step;
+}
+__device__ __forceinline__ void decode_tile(int tile, int tiles_per_lc, int n_tiles_n, int l0,
+                                            int* lc, int* m, int* n) {
+  const int c = tile & 1;
+  const int slot = tile >> 1;
+  const int ol = slot / tiles_per_lc;
+  const int rem = slot - ol * tiles_per_lc;
+  *lc = 2 * (l0 + ol) + c;
   *m = rem / n_tiles_n;
   *n = rem - *m * n_tiles_n;
 }
@@ -218,6 +226,61 @@ __device__ __forceinline__ void walk_step(Walk& w, int j, int it, const int32_t*
       store4(o + 2 * half, a1);
       store4(o + 3 * half, b1);
     }
+  }
+}
+
+// Epilogue of a tile whose rows need no rotation (values; keys when RoPE and
+// key norm are off): every receiver row of a run is the same row of
+// y = acc / r + b, so each distinct row is converted once into the staging
+// buffer and copied out whole.  Columns go in passes of 256 bytes per row
+// (128 rows x 256 bytes of staging); in a pass, warp (g, sp) converts TMEM
+// lane quarter sp, half g of the pass's columns, then warp e copies the runs
+// of distinct rows e, e + 8, ...: 16 lanes x 16 bytes per receiver row, the
+// two half-warps taking alternate receiver rows of the run.
+template <typename T>
+__device__ __forceinline__ void copy_epilogue(const XferParams& P, uint32_t ta,
+                                              const float* bias_tile, float inv_r, int nrows,
+                                              const int32_t* srun, uint8_t* stg, int g, int row,
+                                              int e, int lane, T* out_lc, int ocol0) {
+  constexpr int kPassCols = 256 / sizeof(T);  // 128 bf16 or 64 fp32 columns
+  constexpr int kHalfCols = kPassCols / 2;
+  constexpr int kPerChunk = 16 / sizeof(T);
+  const int hw = lane >> 4, cidx = lane & 15;
+  for (int pc0 = 0; pc0 < P.BN; pc0 += kPassCols) {
+    uint8_t* srow = stg + row * 256;
+#pragma unroll
+    for (int k = 0; k < kHalfCols; k += 16) {
+      const int col = pc0 + g * kHalfCols + k;
+      uint32_t v[16];
+      tmem_load_16(ta + static_cast<uint32_t>(col), v);
+      float y[16];
+#pragma unroll
+      for (int i = 0; i < 16; i += 4) {
+        const float4 bb = __ldg(reinterpret_cast<const float4*>(bias_tile + col + i));
+        y[i] = fmaf(__uint_as_float(v[i]), inv_r, bb.x);
+        y[i + 1] = fmaf(__uint_as_float(v[i + 1]), inv_r, bb.y);
+        y[i + 2] = fmaf(__uint_as_float(v[i + 2]), inv_r, bb.z);
+        y[i + 3] = fmaf(__uint_as_float(v[i + 3]), inv_r, bb.w);
+      }
+#pragma unroll
+      for (int h = 0; h < 16 / kPerChunk; ++h) {
+        const int chunk = (col - pc0) / kPerChunk + h;  // 0..15 within the 256-byte row
+        *reinterpret_cast<uint4*>(srow + ((chunk ^ (row & 7)) << 4)) =
+            pack16(y + h * kPerChunk, (const T*)nullptr);
+      }
+    }
+    named_barrier_sync(1, 256);
+    for (int u = e; u < nrows; u += 8) {
+      const uint4 val = *reinterpret_cast<const uint4*>(stg + u * 256 + ((cidx ^ (u & 7)) << 4));
+      const int je = srun[u + 1];
+      for (int j = srun[u] + hw; j < je; j += 2) {
+        const int drow = P.paged ? __ldg(P.dst_row + j) : j;
+        if (drow >= 0)
+          *reinterpret_cast<uint4*>(out_lc + static_cast<int64_t>(drow) * P.d_r + ocol0 + pc0 +
+                                    cidx * kPerChunk) = val;
+      }
+    }
+    named_barrier_sync(1, 256);
   }
 }
 
@@ -347,6 +410,7 @@ __device__ __forceinline__ void gather_rows(const XferParams& P, uint8_t* sA, ui
                                             int lane, int U, int row0, int total_tiles,
                                             int tiles_per_lc, int first_tile, int tile_step) {
   constexpr int kBK = Elem<T>::kBK;
+  const bool by_slot = total_tiles >= 4 * tile_step;  // as in transfer_kernel
   constexpr int kPerChunk = 16 / sizeof(T);
   const T* sender = reinterpret_cast<const T*>(P.sender);
   const int stages = P.stages_a;
@@ -355,9 +419,10 @@ __device__ __forceinline__ void gather_rows(const XferParams& P, uint8_t* sA, ui
   uint32_t phase = 0;
   int pending = 0;  // committed groups whose stage arrival is still owed
   bool ok = true;
-  for (int tile = first_tile; tile < total_tiles && ok; tile += tile_step) {
+  for (int seq = 0, tile = tile_of(0, first_tile, tile_step, by_slot); tile < total_tiles && ok;
+       tile = tile_of(++seq, first_tile, tile_step, by_slot)) {
     int lc, m, n;
-    decode_tile(tile, tiles_per_lc, P.n_tiles_n, P.n_l, P.l0, &lc, &m, &n);
+    decode_tile(tile, tiles_per_lc, P.n_tiles_n, P.l0, &lc, &m, &n);
     const int l = lc >> 1, c = lc & 1;
     // element offset of each segment's sender layer/role block, for the whole tile
     int64_t seg_base[kMaxSeg];
@@ -488,6 +553,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int m_tiles = (U + kPairRows - 1) / kPairRows;
   const int tiles_per_lc = m_tiles * P.n_tiles_n;
   const int total_tiles = 2 * P.n_l * tiles_per_lc;
+  const bool by_slot = total_tiles >= 4 * tile_step;
 
   if (warp == 0) {
     // ------------------------------------------------------------ map tiles
@@ -496,9 +562,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       int stage = 0;
       uint32_t phase = 0;
       bool ok = true;
-      for (int tile = first_tile; tile < total_tiles && ok; tile += tile_step) {
+      for (int seq = 0, tile = tile_of(0, first_tile, tile_step, by_slot); tile < total_tiles && ok;
+       tile = tile_of(++seq, first_tile, tile_step, by_slot)) {
         int lc, m, n;
-        decode_tile(tile, tiles_per_lc, P.n_tiles_n, P.n_l, P.l0, &lc, &m, &n);
+        decode_tile(tile, tiles_per_lc, P.n_tiles_n, P.l0, &lc, &m, &n);
         for (int kb = 0; kb < P.n_kb; ++kb) {
           if (!mbar_wait(smem_addr(&empty_b[stage]), phase ^ 1)) {
             raise_timeout(P, sAbort);
@@ -543,7 +610,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       int acc = 0;
       uint32_t acc_phase = 0;
       bool ok = true;
-      for (int tile = first_tile; tile < total_tiles && ok; tile += tile_step) {
+      for (int seq = 0, tile = tile_of(0, first_tile, tile_step, by_slot); tile < total_tiles && ok;
+       tile = tile_of(++seq, first_tile, tile_step, by_slot)) {
         if (!mbar_wait(smem_addr(&tempty[acc]), acc_phase ^ 1)) {
           raise_timeout(P, sAbort);
           break;
@@ -620,9 +688,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int ps = lane >> 2, qq = lane & 3;  // row slot 0..7, pair quad 0..3
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int tile = first_tile; tile < total_tiles; tile += tile_step) {
+    for (int seq = 0, tile = tile_of(0, first_tile, tile_step, by_slot); tile < total_tiles;
+       tile = tile_of(++seq, first_tile, tile_step, by_slot)) {
       int lc, m, n;
-      decode_tile(tile, tiles_per_lc, P.n_tiles_n, P.n_l, P.l0, &lc, &m, &n);
+      decode_tile(tile, tiles_per_lc, P.n_tiles_n, P.l0, &lc, &m, &n);
       const int c = lc & 1;
       if (!mbar_wait(smem_addr(&tfull[acc]), acc_phase)) {
         raise_timeout(P, sAbort);
@@ -652,6 +721,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                             (static_cast<uint32_t>(sp * 32) << 16);
         T* const out_lc = reinterpret_cast<T*>(P.receiver) +
                           (static_cast<int64_t>(lc) * P.recv_rows) * P.d_r;
+        if (c == 1 || (!P.rope && !P.knorm)) {
+          copy_epilogue<T>(P, ta, bias + n * P.BN, inv_r, nrows, sRun,
+                           reinterpret_cast<uint8_t*>(sStg), g, row, e, lane, out_lc, n * P.BN);
+        } else
         for (int hp = 0; hp < n_pairs; ++hp) {
           const bool stages_head = g == 0 || two_heads;
           const int tcol = (2 * hp + g) * D;            // accumulator column of this warp's head
@@ -755,9 +828,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       int stage = 0;
       uint32_t phase = 0;
       bool ok = true;
-      for (int tile = first_tile; tile < total_tiles && ok; tile += tile_step) {
+      for (int seq = 0, tile = tile_of(0, first_tile, tile_step, by_slot); tile < total_tiles && ok;
+       tile = tile_of(++seq, first_tile, tile_step, by_slot)) {
         int lc, m, n;
-        decode_tile(tile, tiles_per_lc, P.n_tiles_n, P.n_l, P.l0, &lc, &m, &n);
+        decode_tile(tile, tiles_per_lc, P.n_tiles_n, P.l0, &lc, &m, &n);
         const int l = lc >> 1, c = lc & 1;
         const LayerSegs segs = P.segs[l];
         const int u = min(m * kPairRows + row0 + t, U - 1);
