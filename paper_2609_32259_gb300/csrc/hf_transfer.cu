@@ -154,13 +154,16 @@ __device__ __forceinline__ uint4 pack16(const float* a, const float*) {
                     __float_as_uint(a[3]));
 }
 
+// Receiver-cache stores are streaming stores (st.global.cs, evict first):
+// the output is written once and should not push map tiles and sender rows,
+// which other tiles read again, out of L2.
 __device__ __forceinline__ void store4(__nv_bfloat16* p, const float4& v) {
   const __nv_bfloat162 x = __floats2bfloat162_rn(v.x, v.y), y = __floats2bfloat162_rn(v.z, v.w);
-  *reinterpret_cast<uint2*>(p) =
-      make_uint2(*reinterpret_cast<const uint32_t*>(&x), *reinterpret_cast<const uint32_t*>(&y));
+  __stcs(reinterpret_cast<uint2*>(p),
+         make_uint2(*reinterpret_cast<const uint32_t*>(&x), *reinterpret_cast<const uint32_t*>(&y)));
 }
 __device__ __forceinline__ void store4(float* p, const float4& v) {
-  *reinterpret_cast<float4*>(p) = v;
+  __stcs(reinterpret_cast<float4*>(p), v);
 }
 
 // Rotates the pairs (x[k], y[k]) by the angles with cosines c[k], sines s[k].
@@ -276,8 +279,9 @@ __device__ __forceinline__ void copy_epilogue(const XferParams& P, uint32_t ta,
       for (int j = srun[u] + hw; j < je; j += 2) {
         const int drow = P.paged ? __ldg(P.dst_row + j) : j;
         if (drow >= 0)
-          *reinterpret_cast<uint4*>(out_lc + static_cast<int64_t>(drow) * P.d_r + ocol0 + pc0 +
-                                    cidx * kPerChunk) = val;
+          __stcs(reinterpret_cast<uint4*>(out_lc + static_cast<int64_t>(drow) * P.d_r + ocol0 +
+                                          pc0 + cidx * kPerChunk),
+                 val);
       }
     }
     named_barrier_sync(1, 256);
