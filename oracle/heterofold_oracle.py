@@ -353,13 +353,16 @@ def key_norm(x: np.ndarray, g: np.ndarray, eps: float) -> np.ndarray:
 # The transfer (Eq. 2 + Eq. 9)
 # ---------------------------------------------------------------------------
 
-def pooled_features(sender_lc, csr: CSR, rows: np.ndarray, unrotate=None) -> np.ndarray:
+def pooled_features(sender_lc, csr: CSR, rows: np.ndarray, unrotate=None,
+                    row_of=None) -> np.ndarray:
     """Pool one sender layer/role over the alignment rows: for receiver row j,
     sum_k w_k * c_k over the row's entries (a single copy for TA).
 
     unrotate: None, or (s_pos, inv_freq_s, H_s) for sender keys stored with
-    RoPE: each sender row k is first rotated back at its position s_pos[k]
-    (rope_inverse), then weighted and summed."""
+    RoPE: each sender token k is first rotated back at its position s_pos[k]
+    (rope_inverse), then weighted and summed.
+    row_of: None (sender token k is cache row k), or the cache row of every
+    sender token (a message span inside a longer sender cache)."""
     starts = csr.row_ptr[rows]
     ends = csr.row_ptr[rows + 1]
     if np.any(ends <= starts):
@@ -367,7 +370,8 @@ def pooled_features(sender_lc, csr: CSR, rows: np.ndarray, unrotate=None) -> np.
     lengths = ends - starts
     entry = np.concatenate([np.arange(a, b) for a, b in zip(starts, ends)])
     cols = csr.col[entry]
-    feats = np.asarray(sender_lc[cols], dtype=np.float64)
+    feats = np.asarray(sender_lc[cols if row_of is None else np.asarray(row_of)[cols]],
+                       dtype=np.float64)
     if unrotate is not None:
         s_pos, inv_freq_s, H_s = unrotate
         n, d_s = feats.shape
@@ -379,19 +383,19 @@ def pooled_features(sender_lc, csr: CSR, rows: np.ndarray, unrotate=None) -> np.
 
 
 def map_input(sender, csr: CSR, segments_l, role: int, rows: np.ndarray,
-              sender_rope=None) -> np.ndarray:
+              sender_rope=None, sender_row_of=None) -> np.ndarray:
     """Eq. 2: the concatenated map input x for receiver layer l and role c.
 
     Segment s is the weighted sum of its sender layers' pooled features;
     the segments are concatenated along the feature axis.  sender_rope
-    (keys only): see pooled_features' unrotate.
+    (keys only): see pooled_features' unrotate; sender_row_of: its row_of.
     """
     unrot = sender_rope if role == ROLE_K else None
     parts = []
     for seg in segments_l:
         acc = None
         for (t, omega) in seg:
-            term = omega * pooled_features(sender[t][role], csr, rows, unrot)
+            term = omega * pooled_features(sender[t][role], csr, rows, unrot, sender_row_of)
             acc = term if acc is None else acc + term
         parts.append(acc)
     return np.concatenate(parts, axis=1)
@@ -403,7 +407,7 @@ def transfer(sender, csr: CSR, segments, A, b, r, *, H_r: int, D_r: int,
              layers: Optional[Iterable[int]] = None,
              rows: Optional[np.ndarray] = None,
              roles: Iterable[int] = (ROLE_K, ROLE_V),
-             sender_rope=None) -> Dict[Tuple[int, int], np.ndarray]:
+             sender_rope=None, sender_row_of=None) -> Dict[Tuple[int, int], np.ndarray]:
     """The receiver cache entries for the requested layers, roles and rows.
 
     sender:  indexable as sender[t][c] -> [T_s, d_S] array (any float dtype)
@@ -415,6 +419,9 @@ def transfer(sender, csr: CSR, segments, A, b, r, *, H_r: int, D_r: int,
     sender_rope: None (sender keys captured before RoPE, the paper's case) or
              (s_pos, inv_freq_s, H_s) when the sender keys carry RoPE at
              sender positions s_pos: they are rotated back before pooling.
+    sender_row_of: None, or the sender-cache row of every sender token of
+             the alignment (message spans: only a span of each request's
+             sender cache is transferred, Appendix "HiddenBench Evaluation").
 
     Returns {(l, c): [n_rows, H_r, D_r] float64}.  Eq. 9:
     Phi(x) = (x / r) A + b, reshaped to receiver heads; keys then get the
@@ -426,7 +433,7 @@ def transfer(sender, csr: CSR, segments, A, b, r, *, H_r: int, D_r: int,
     out: Dict[Tuple[int, int], np.ndarray] = {}
     for l in layers:
         for c in roles:
-            x = map_input(sender, csr, segments[l], c, rows, sender_rope)
+            x = map_input(sender, csr, segments[l], c, rows, sender_rope, sender_row_of)
             A_lc = np.asarray(A[l][c], dtype=np.float64)
             if A_lc.shape != (x.shape[1], H_r * D_r):
                 raise ValueError(f"map shape {A_lc.shape} does not match input "
@@ -451,6 +458,16 @@ def token_positions(tok_ptr: Sequence[int], pos0: Optional[Sequence[int]] = None
         for t in range(int(tok_ptr[q + 1]) - int(tok_ptr[q])):
             pos.append(base + t)
     return np.asarray(pos, dtype=np.int64)
+
+
+def span_rows(s_tok_ptr: Sequence[int], s_row0: Sequence[int]) -> np.ndarray:
+    """Sender-cache row of every concatenated sender token when request q's
+    tokens are the span starting at cache row s_row0[q]."""
+    out = []
+    for q in range(len(s_tok_ptr) - 1):
+        for t in range(int(s_tok_ptr[q + 1]) - int(s_tok_ptr[q])):
+            out.append(int(s_row0[q]) + t)
+    return np.asarray(out, dtype=np.int64)
 
 
 def receiver_positions(r_tok_ptr: Sequence[int], r_pos0: Optional[Sequence[int]] = None) -> np.ndarray:

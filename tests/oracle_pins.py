@@ -321,7 +321,7 @@ def _tiny_problem(seed, align_mode, layer_mode, L_s=3, L_r=4, H_s=2, D_s=4, H_r=
                 H_r=H_r, D_r=D_r, d_s=d_s, s_end=s_end, r_end=r_end)
 
 
-def _transfer_brute(P, knorm_g=None, eps=1e-6, srope=None):
+def _transfer_brute(P, knorm_g=None, eps=1e-6, srope=None, row_of=None):
     """Every output element from the definitions, with Python loops.
     srope = (s_pos, inv_freq_s, H_s): sender keys carry RoPE and each sender
     feature is rotated back at its token's position before it is used."""
@@ -329,6 +329,19 @@ def _transfer_brute(P, knorm_g=None, eps=1e-6, srope=None):
     H_r, D_r, d_s, inv, pos = P["H_r"], P["D_r"], P["d_s"], P["inv"], P["pos"]
 
     def feature(t, c, k, d):
+        if row_of is not None:  # sender token k lives at cache row row_of[k]
+            kr = row_of[k]
+            v = sender[t, c, kr, d]
+            if srope is None or c != 0:
+                return v
+            s_pos, inv_s, H_s = srope
+            D_s = d_s // H_s
+            h, i = divmod(d, D_s)
+            hs = D_s // 2
+            ang = s_pos[k] * inv_s[i % hs]
+            if i < hs:
+                return v * math.cos(ang) + sender[t, c, kr, h * D_s + i + hs] * math.sin(ang)
+            return v * math.cos(ang) - sender[t, c, kr, h * D_s + i - hs] * math.sin(ang)
         v = sender[t, c, k, d]
         if srope is None or c != 0:
             return v
@@ -413,6 +426,42 @@ def check_transfer_brute_force_rotated_sender():
         ref = _transfer_brute(P, srope=(s_pos, inv_s, 2))
         for key in ref:
             assert np.allclose(got[key], ref[key], rtol=1e-10, atol=1e-10), (seed, key)
+
+
+def check_message_spans():
+    """Message spans: request q's sender tokens are the cache rows
+    s_row0[q] .. s_row0[q] + n_q - 1 of a longer sender cache.  Brute force
+    with explicit row arithmetic, and the same transfer on a cache that holds
+    only the spans (concatenated) gives the same result."""
+    rng = np.random.default_rng(16)
+    L_s, L_r, H, D = 3, 4, 2, 4
+    d = H * D
+    s_ends = [_ends([2, 1, 3, 2]), _ends([1, 2, 2])]          # two messages
+    r_ends = [_ends([3, 1, 2, 2]), _ends([2, 3])]
+    s_ptr = [0, 4, 7]
+    r_ptr = [0, 4, 6]
+    s_row0 = [10, 3]                                          # spans inside a 20-row cache
+    rows = O.span_rows(s_ptr, s_row0)
+    assert rows.tolist() == [10, 11, 12, 13, 3, 4, 5]
+    cache = rng.normal(size=(L_s, 2, 20, d))
+    csr = O.alignment_csr(O.ALIGN_OVERLAP_MEAN, s_ptr, r_ptr, sum(s_ends, []), sum(r_ends, []))
+    segs = O.layer_segments(O.LAYER_PAPER3, L_s, L_r)
+    A = rng.normal(size=(L_r, 2, 3 * d, d)) / math.sqrt(3 * d)
+    b = rng.normal(size=(L_r, 2, d)) * 0.1
+    r = rng.uniform(0.5, 2.0, size=(L_r, 2))
+    inv = O.rope_inv_freq(10000.0, D)
+    pos = O.receiver_positions(r_ptr, [100, 7])
+    s_pos = O.sender_positions(s_ptr, [40, 9])
+    P = dict(sender=cache, segs=segs, A=A, b=b, r=r, csr=csr, inv=inv, pos=pos, H_r=H, D_r=D, d_s=d)
+    srope = (s_pos, O.rope_inv_freq(5e5, D), H)
+    got = _run_oracle(P, sender_rope=srope, sender_row_of=rows)
+    ref = _transfer_brute(P, srope=srope, row_of=rows)
+    for key in ref:
+        assert np.allclose(got[key], ref[key], rtol=1e-10, atol=1e-10), key
+    packed = cache[:, :, rows, :]                              # the spans alone
+    alone = _run_oracle(dict(P, sender=packed), sender_rope=srope)
+    for key in ref:
+        assert np.allclose(alone[key], got[key], rtol=1e-12, atol=1e-12), key
 
 
 def check_explicit_segments():
@@ -596,7 +645,7 @@ ALL_CHECKS = [
     check_rope_two_dim_rotation, check_rope_complex_form, check_rope_relative_position,
     check_rope_inverse, check_inv_freq, check_key_norm,
     check_transfer_brute_force, check_transfer_brute_force_rotated_sender,
-    check_explicit_segments, check_identity_map_reproduces_input,
+    check_explicit_segments, check_message_spans, check_identity_map_reproduces_input,
     check_identity_rotated_sender_keys, check_rotated_sender_position_shift,
     check_rotated_sender_unrotates_before_pooling,
     check_affine_structure, check_segment_blocks,

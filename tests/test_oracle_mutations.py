@@ -86,11 +86,12 @@ def _overlap_closed(s_end, r_end):
     return rows
 
 
-def _pool_unweighted(sender_lc, csr, rows, unrotate=None):
+def _pool_unweighted(sender_lc, csr, rows, unrotate=None, row_of=None):
     out = []
     for j in rows:
         idx = csr.col[csr.row_ptr[j]:csr.row_ptr[j + 1]]
-        x = np.asarray(sender_lc[idx], dtype=np.float64)
+        x = np.asarray(sender_lc[idx if row_of is None else np.asarray(row_of)[idx]],
+                       dtype=np.float64)
         if unrotate is not None:
             s_pos, inv, H_s = unrotate
             x = O.rope_inverse(x.reshape(len(idx), H_s, -1), np.asarray(s_pos)[idx], inv).reshape(len(idx), -1)
@@ -106,16 +107,21 @@ def _rope_inverse_forward(x, pos, inv):
 _orig_pooled = O.pooled_features
 
 
-def _pool_then_unrotate(sender_lc, csr, rows, unrotate=None):
+def _pool_then_unrotate(sender_lc, csr, rows, unrotate=None, row_of=None):
     # wrong: pools the rotated rows, then rotates back once at the row's
     # first sender position
-    y = _orig_pooled(sender_lc, csr, rows)
+    y = _orig_pooled(sender_lc, csr, rows, None, row_of)
     if unrotate is None:
         return y
     s_pos, inv, H_s = unrotate
     first = csr.col[csr.row_ptr[rows]]
     n, d = y.shape
     return O.rope_inverse(y.reshape(n, H_s, d // H_s), np.asarray(s_pos)[first], inv).reshape(n, d)
+
+
+def _span_rows_from_zero(s_tok_ptr, s_row0):
+    # wrong: ignores the span origins
+    return np.arange(int(s_tok_ptr[-1]), dtype=np.int64)
 
 
 def _explicit_weights_swapped(seg_layer, seg_w):
@@ -127,17 +133,20 @@ _orig_map_input = O.map_input
 _orig_transfer = O.transfer
 
 
-def _map_input_reversed(sender, csr, segments_l, role, rows, sender_rope=None):
-    return _orig_map_input(sender, csr, list(reversed(segments_l)), role, rows, sender_rope)
+def _map_input_reversed(sender, csr, segments_l, role, rows, sender_rope=None,
+                        sender_row_of=None):
+    return _orig_map_input(sender, csr, list(reversed(segments_l)), role, rows, sender_rope,
+                           sender_row_of)
 
 
-def _map_input_unrotates_values(sender, csr, segments_l, role, rows, sender_rope=None):
+def _map_input_unrotates_values(sender, csr, segments_l, role, rows, sender_rope=None,
+                                sender_row_of=None):
     # wrong: values are rotated back as well
     parts = []
     for seg in segments_l:
         acc = None
         for (t, omega) in seg:
-            term = omega * _orig_pooled(sender[t][role], csr, rows, sender_rope)
+            term = omega * _orig_pooled(sender[t][role], csr, rows, sender_rope, sender_row_of)
             acc = term if acc is None else acc + term
         parts.append(acc)
     return np.concatenate(parts, axis=1)
@@ -171,6 +180,7 @@ MUTATIONS = {
     "unrotate_after_pooling": ("pooled_features", _pool_then_unrotate),
     "values_unrotated": ("map_input", _map_input_unrotates_values),
     "explicit_weights_swapped": ("explicit_segments", _explicit_weights_swapped),
+    "span_rows_from_zero": ("span_rows", _span_rows_from_zero),
 }
 
 
