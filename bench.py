@@ -236,7 +236,7 @@ def run_reference(args):
     w = workload(args.workload)
     tok = W.tokens(w)
     dev = torch.device("cuda") if torch.cuda.is_available() else torch.device("cpu")
-    sender = W.sender_kv(w, tok.T_s, dev)
+    sender = W.sender_kv(w, W.sender_cache_rows(w, tok), dev)
     Wm, b, r = W.maps(w, dev)
     per_step = max(1.0, min(8.0, 150.0 / max(1, args.steps + args.warmup)))
     samp = sized_oracle_sample(w, tok, sender, Wm, b, r, per_step)
@@ -290,7 +290,7 @@ def run_ours(args):
 
     w = workload(args.workload)
     tok = W.tokens(w)
-    sender = W.sender_kv(w, tok.T_s, dev)
+    sender = W.sender_kv(w, W.sender_cache_rows(w, tok), dev)
     Wm, b, r = W.maps(w, dev)
     paged = W.paged_layout(w, tok) if w.paged else None
     job = pipeline.job_from_workload(w, tok, sender, Wm, b, r, paged=paged, device=dev)

@@ -207,6 +207,16 @@ typedef struct {
   const float* h_inv_freq_s;    /* host float[D_s/2], or NULL */
   const int32_t* s_pos0;        /* host int32[n_req], or NULL for 0 */
 
+  /* Message spans (Appendix "HiddenBench Evaluation": only the K/V states
+     of a message that follows a context are mapped).  s_row0 (host
+     int32[n_req], or NULL): request q's sender tokens are the sender-cache
+     rows s_row0[q] .. s_row0[q] + (s_tok_ptr[q+1] - s_tok_ptr[q]) - 1; the
+     CSR columns still count the concatenated span tokens.  sender_rows:
+     rows per (layer, role) in sender_kv (0: T_s = s_tok_ptr[n_req]); every
+     span must lie inside it. */
+  const int32_t* s_row0;
+  int64_t sender_rows;
+
   /* HF_LAYER_EXPLICIT only: host arrays [L_r][n_seg][n_terms]. */
   int32_t n_seg;                /* 1 .. 3 segments per receiver layer */
   int32_t n_terms;              /* 1 .. 2 sender layers per segment */
@@ -236,7 +246,8 @@ hf_status hf_plan_create(const hf_plan_desc* desc, void* d_workspace, size_t wor
 
 /*
  * hf_transfer — write the receiver cache (one kernel launch on `stream`).
- * sender_kv:   device [L_s][2][T_s][H_s][D_s] in the plan's dtype, the
+ * sender_kv:   device [L_s][2][sender_rows][H_s][D_s] (sender_rows = T_s
+ *              unless the plan maps message spans) in the plan's dtype, the
  *              sender's keys and values; keys pre-RoPE (Section 3: keys are
  *              mapped before key normalisation and RoPE) unless the plan
  *              says sender_k_rotated; 16-byte aligned.
@@ -252,8 +263,9 @@ hf_status hf_transfer(hf_plan plan, const void* sender_kv, void* receiver_kv,
  * memory, with the host<->device copies overlapped with the computation.
  * The paper moves the sender payload GPU to GPU; this entry point serves
  * callers whose caches live on the host.
- * h_sender_kv:   page-locked host [L_s][2][T_s][H_s][D_s] (cudaHostAlloc or
- *                cudaHostRegister), the layout hf_transfer takes.
+ * h_sender_kv:   page-locked host [L_s][2][sender_rows][H_s][D_s]
+ *                (cudaHostAlloc or cudaHostRegister), the layout hf_transfer
+ *                takes.
  * d_sender_kv:   device buffer of the same size: the sender layers are
  *                copied there (only layers 0 .. the highest one the layer
  *                table reads).

@@ -62,6 +62,7 @@ class PlanDesc(ctypes.Structure):
         ("h_inv_freq_r", _f32p),
         ("sender_k_rotated", ctypes.c_int32), ("theta_s", ctypes.c_double),
         ("h_inv_freq_s", _f32p), ("s_pos0", _i32p),
+        ("s_row0", _i32p), ("sender_rows", ctypes.c_int64),
         ("n_seg", ctypes.c_int32), ("n_terms", ctypes.c_int32),
         ("h_seg_layer", _i32p), ("h_seg_w", _f32p),
     ]
@@ -165,11 +166,12 @@ class Desc:
                  r_pos0=None, d_knorm_w=None, knorm_eps=1e-6, paged=False, block_size=16,
                  n_blocks=0, max_blocks_per_req=0, d_block_table=None, inv_freq_r=None,
                  sender_k_rotated=False, theta_s=0.0, inv_freq_s=None, s_pos0=None,
-                 seg_layer=None, seg_w=None):
+                 seg_layer=None, seg_w=None, s_row0=None, sender_rows=0):
         self._s = _host_i32(s_tok_ptr)
         self._r = _host_i32(r_tok_ptr)
         self._pos0 = None if r_pos0 is None else _host_i32(r_pos0)
         self._spos0 = None if s_pos0 is None else _host_i32(s_pos0)
+        self._srow0 = None if s_row0 is None else _host_i32(s_row0)
         self._hr = np.ascontiguousarray(np.asarray(r, dtype=np.float32).reshape(-1))
         self._ifr = None if inv_freq_r is None else _host_f32(inv_freq_r)
         self._ifs = None if inv_freq_s is None else _host_f32(inv_freq_s)
@@ -196,6 +198,8 @@ class Desc:
             h_inv_freq_r=_f32_or_null(self._ifr), sender_k_rotated=int(bool(sender_k_rotated)),
             theta_s=float(theta_s), h_inv_freq_s=_f32_or_null(self._ifs),
             s_pos0=_as_i32p(self._spos0) if self._spos0 is not None else None,
+            s_row0=_as_i32p(self._srow0) if self._srow0 is not None else None,
+            sender_rows=int(sender_rows),
             n_seg=n_seg, n_terms=n_terms,
             h_seg_layer=_as_i32p(self._segl) if self._segl is not None else None,
             h_seg_w=_f32_or_null(self._segw))

@@ -96,7 +96,7 @@ extern "C" hf_status hf_transfer_host(hf_plan plan, const void* h_sender_kv, voi
 
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
   const size_t esize = d.dtype == HF_BF16 ? 2 : 4;
-  const size_t sender_layer = 2 * static_cast<size_t>(plan->T_s) * plan->d_s * esize;
+  const size_t sender_layer = 2 * static_cast<size_t>(plan->s_rows) * plan->d_s * esize;
   const int64_t recv_rows = d.paged ? static_cast<int64_t>(d.n_blocks) * d.block_size : plan->T_r;
   const size_t recv_layer = 2 * static_cast<size_t>(recv_rows) * plan->d_r * esize;
   const char* hs = static_cast<const char*>(h_sender_kv);

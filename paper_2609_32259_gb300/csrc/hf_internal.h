@@ -39,6 +39,8 @@ struct WorkspaceLayout {
   size_t s_tok_ptr;  // int32[n_req + 1]
   size_t s_pos0;     // int32[n_req]
   size_t spos;       // int32[T_s] sender RoPE positions (sender_k_rotated), else one word
+  size_t s_row0;     // int32[n_req] sender-cache row of each request's span
+  size_t srow;       // int32[T_s] sender-cache row of each aligned token (spans), else one word
   size_t run_ptr;    // int32[T_r + 1]: first receiver row of each distinct row
   size_t ucol;       // int32[T_r]: sender column of each distinct row (one-entry rows)
   size_t upos;       // int32[T_r]: RoPE position of each distinct row's first receiver row
@@ -62,6 +64,7 @@ struct PlanTables {
   int32_t r_pos0[kMaxReq];
   int32_t s_tok_ptr[kMaxReq + 1];
   int32_t s_pos0[kMaxReq];
+  int32_t s_row0[kMaxReq];
 };
 static_assert(sizeof(PlanTables) < 32000, "PlanTables must fit the kernel parameter space");
 
@@ -75,6 +78,8 @@ struct hf_plan_s {
   bool gather;  // every map input row is a single unweighted sender row
   bool rope;    // receiver keys get RoPE
   bool unrot;   // sender keys carry RoPE and are rotated back in the builder
+  bool span;    // aligned sender tokens are spans inside a longer sender cache
+  int64_t s_rows;  // sender-cache rows per (layer, role)
   char* ws;
   size_t ws_bytes;
   hf::WorkspaceLayout lay;

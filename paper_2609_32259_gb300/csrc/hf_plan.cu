@@ -43,6 +43,7 @@ WorkspaceLayout workspace_layout(const hf_plan_desc& d) {
   const int L_r = d.L_r, D_r = d.D_r, D_s = d.D_s, n_req = d.n_req;
   const int64_t T_r = d.r_tok_ptr[n_req];
   const int64_t n_spos = d.sender_k_rotated ? d.s_tok_ptr[n_req] : 0;
+  const int64_t n_srow = d.s_row0 ? d.s_tok_ptr[n_req] : 0;
   WorkspaceLayout w{};
   size_t off = 0;
   auto take = [&](size_t bytes) {
@@ -61,6 +62,8 @@ WorkspaceLayout workspace_layout(const hf_plan_desc& d) {
   w.s_tok_ptr = take(sizeof(int32_t) * (size_t)(n_req + 1));
   w.s_pos0 = take(sizeof(int32_t) * (size_t)n_req);
   w.spos = take(sizeof(int32_t) * (size_t)(n_spos > 0 ? n_spos : 1));
+  w.s_row0 = take(sizeof(int32_t) * (size_t)n_req);
+  w.srow = take(sizeof(int32_t) * (size_t)(n_srow > 0 ? n_srow : 1));
   w.run_ptr = take(sizeof(int32_t) * (size_t)(T_r + 1));
   w.ucol = take(sizeof(int32_t) * (size_t)(T_r > 0 ? T_r : 1));
   w.upos = take(sizeof(int32_t) * (size_t)(T_r > 0 ? T_r : 1));
@@ -85,6 +88,8 @@ struct PlanDev {
   int32_t* s_tok_ptr;
   int32_t* s_pos0;
   int32_t* spos;
+  int32_t* s_row0;
+  int32_t* srow;
   int32_t* run_ptr;
   int32_t* ucol;
   int32_t* upos;
@@ -107,6 +112,8 @@ PlanDev plan_dev(const hf_plan_s* p) {
   d.s_tok_ptr = reinterpret_cast<int32_t*>(at(p->lay.s_tok_ptr));
   d.s_pos0 = reinterpret_cast<int32_t*>(at(p->lay.s_pos0));
   d.spos = reinterpret_cast<int32_t*>(at(p->lay.spos));
+  d.s_row0 = reinterpret_cast<int32_t*>(at(p->lay.s_row0));
+  d.srow = reinterpret_cast<int32_t*>(at(p->lay.srow));
   d.run_ptr = reinterpret_cast<int32_t*>(at(p->lay.run_ptr));
   d.ucol = reinterpret_cast<int32_t*>(at(p->lay.ucol));
   d.upos = reinterpret_cast<int32_t*>(at(p->lay.upos));
@@ -131,15 +138,20 @@ __global__ void plan_init_kernel(PlanTables t, PlanDev d) {
   for (int i = tid; i < t.D_s / 2; i += blockDim.x) d.inv_freq_s[i] = t.inv_freq_s[i];
   for (int i = tid; i <= t.n_req; i += blockDim.x) d.s_tok_ptr[i] = t.s_tok_ptr[i];
   for (int i = tid; i < t.n_req; i += blockDim.x) d.s_pos0[i] = t.s_pos0[i];
+  for (int i = tid; i < t.n_req; i += blockDim.x) d.s_row0[i] = t.s_row0[i];
 }
 
-// Sender RoPE position of every sender token (sender_k_rotated): the
-// request's origin plus the token's index within the request.
-__global__ void plan_spos_kernel(PlanDev d, int64_t T_s, int n_req) {
+// Per aligned sender token: its RoPE position (sender_k_rotated), the
+// request's origin plus the token's index within the request; and its
+// sender-cache row (message spans), the span's first row plus that index.
+__global__ void plan_sender_kernel(PlanDev d, int64_t T_s, int n_req, int want_pos,
+                                   int want_row) {
   for (int64_t k = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; k < T_s;
        k += (int64_t)gridDim.x * blockDim.x) {
     const int q = find_request(d.s_tok_ptr, n_req, k);
-    d.spos[k] = d.s_pos0[q] + static_cast<int32_t>(k - d.s_tok_ptr[q]);
+    const int32_t t = static_cast<int32_t>(k - d.s_tok_ptr[q]);
+    if (want_pos) d.spos[k] = d.s_pos0[q] + t;
+    if (want_row) d.srow[k] = d.s_row0[q] + t;
   }
 }
 
@@ -154,6 +166,7 @@ struct RowArgs {
   int n_req;
   int paged, block_size, n_blocks, max_blocks;
   int single_entry;  // rows must be one entry of weight 1
+  int span;          // map sender tokens to cache rows through d.srow
 };
 
 __device__ __forceinline__ void flag(int32_t* status, int bits) { atomicOr(status, bits); }
@@ -218,7 +231,7 @@ __global__ void plan_runs_kernel(RowArgs a) {
       d.run_ptr[u] = static_cast<int32_t>(j);
       int32_t k = a.col[a.row_ptr[j]];
       if (k < 0 || k >= a.T_s) k = 0;  // flagged by plan_rows_kernel
-      d.ucol[u] = k;
+      d.ucol[u] = a.span ? d.srow[k] : k;  // the sender-cache row
       d.upos[u] = d.pos[j];
     }
     if (j == a.T_r - 1) {
@@ -355,7 +368,19 @@ hf_status validate(const hf_plan_desc* d) {
     if (d->block_size < 1 || d->n_blocks < 1 || d->max_blocks_per_req < 1 || !d->d_block_table)
       return bad("paged layout needs block_size, n_blocks, max_blocks_per_req, d_block_table");
   }
-  const long long rows = (long long)d->L_s * 2 * d->s_tok_ptr[d->n_req];
+  const int64_t T_s = d->s_tok_ptr[d->n_req];
+  if (d->sender_rows < 0) return bad("sender_rows must be >= 0");
+  const int64_t s_rows = d->sender_rows > 0 ? d->sender_rows : T_s;
+  if (d->s_row0) {
+    for (int q = 0; q < d->n_req; ++q) {
+      const int64_t n_q = d->s_tok_ptr[q + 1] - d->s_tok_ptr[q];
+      if (d->s_row0[q] < 0 || d->s_row0[q] + n_q > s_rows)
+        return bad("a message span lies outside the sender cache (s_row0, sender_rows)");
+    }
+  } else if (s_rows < T_s) {
+    return bad("sender_rows is smaller than the aligned sender tokens");
+  }
+  const long long rows = (long long)d->L_s * 2 * s_rows;
   if (rows >= (1LL << 31)) return unsup("sender cache has more than 2^31 rows");
   return HF_OK;
 }
@@ -381,16 +406,18 @@ hf_status launch_plan_kernels(hf_plan_s* p, const PlanTables& tables, cudaStream
   a.n_blocks = p->desc.n_blocks;
   a.max_blocks = p->desc.max_blocks_per_req;
   a.single_entry = p->desc.align_mode != HF_ALIGN_OVERLAP_MEAN;
+  a.span = p->span ? 1 : 0;
   const int64_t want = (p->T_r + 255) / 256;
   const int grid = static_cast<int>(std::min<int64_t>(want, 8LL * device_sm_count()));
   plan_rows_kernel<<<grid, 256, 0, stream>>>(a);
   scan_inplace_kernel<ScanSum><<<1, kScanThreads, 0, stream>>>(d.new_flag, p->T_r, nullptr);
-  plan_runs_kernel<<<grid, 256, 0, stream>>>(a);
-  if (p->unrot && p->T_s > 0) {
+  if ((p->unrot || p->span) && p->T_s > 0) {
     const int64_t want_s = (p->T_s + 255) / 256;
     const int grid_s = static_cast<int>(std::min<int64_t>(want_s, 8LL * device_sm_count()));
-    plan_spos_kernel<<<grid_s, 256, 0, stream>>>(d, p->T_s, p->desc.n_req);
+    plan_sender_kernel<<<grid_s, 256, 0, stream>>>(d, p->T_s, p->desc.n_req, p->unrot ? 1 : 0,
+                                                   p->span ? 1 : 0);
   }
+  plan_runs_kernel<<<grid, 256, 0, stream>>>(a);
   HF_CUDA_TRY(cudaGetLastError(), "plan kernels launch");
   return HF_OK;
 }
@@ -430,6 +457,8 @@ hf_status plan_build(const hf_plan_desc* desc, void* d_workspace, size_t workspa
              : desc->layer_mode == HF_LAYER_EXPLICIT ? desc->n_seg : 1;
   p->K = p->n_seg * p->d_s;
   p->T_s = desc->s_tok_ptr[desc->n_req];
+  p->span = desc->s_row0 != nullptr;
+  p->s_rows = desc->sender_rows > 0 ? desc->sender_rows : p->T_s;
   p->T_r = desc->r_tok_ptr[desc->n_req];
   p->BN = (p->d_r % 256 == 0) ? 256 : 128;
   p->groups = ((p->BN / 2) % desc->D_r == 0) ? 2 : 1;
@@ -455,6 +484,7 @@ hf_status plan_build(const hf_plan_desc* desc, void* d_workspace, size_t workspa
   p->desc.h_inv_freq_r = nullptr;
   p->desc.h_inv_freq_s = nullptr;
   p->desc.s_pos0 = nullptr;
+  p->desc.s_row0 = nullptr;
   p->desc.h_seg_layer = nullptr;
   p->desc.h_seg_w = nullptr;
 
@@ -487,6 +517,7 @@ hf_status plan_build(const hf_plan_desc* desc, void* d_workspace, size_t workspa
   for (int q = 0; q < desc->n_req; ++q) t->r_pos0[q] = desc->r_pos0 ? desc->r_pos0[q] : 0;
   for (int q = 0; q <= desc->n_req; ++q) t->s_tok_ptr[q] = desc->s_tok_ptr[q];
   for (int q = 0; q < desc->n_req; ++q) t->s_pos0[q] = desc->s_pos0 ? desc->s_pos0[q] : 0;
+  for (int q = 0; q < desc->n_req; ++q) t->s_row0[q] = desc->s_row0 ? desc->s_row0[q] : 0;
   return launch_plan_kernels(p, *t, stream);
 }
 

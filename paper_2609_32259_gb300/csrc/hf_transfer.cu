@@ -72,7 +72,9 @@ struct XferParams {
   const int32_t* dst_row;
   const int32_t* n_distinct;
   int32_t* status;
-  int64_t T_s;        // sender rows per (layer, role)
+  int64_t T_s;        // aligned sender tokens (CSR column range)
+  int64_t s_rows;     // sender-cache rows per (layer, role)
+  const int32_t* srow;  // cache row of each aligned sender token (message spans), or null
   int64_t recv_rows;  // receiver rows per (layer, role) in receiver_kv
   int L_r, d_s, d_r, D_r;
   int l0, n_l;  // receiver layers [l0, l0 + n_l) of this launch
@@ -314,12 +316,13 @@ __device__ __forceinline__ void build_atom(const XferParams& P, const LayerSegs&
   for (int ti = 0; ti < segs.n_terms[seg]; ++ti) {
     const int tl = segs.layer[seg][ti];
     const float om = segs.w[seg][ti];
-    const T* base = sender + (static_cast<int64_t>(tl * 2 + c) * P.T_s) * P.d_s + kin * kBK;
+    const T* base = sender + (static_cast<int64_t>(tl * 2 + c) * P.s_rows) * P.d_s + kin * kBK;
     for (int e = e0; e < e1; ++e) {
       const int k = P.col[e];
       if (k < 0 || k >= P.T_s) continue;  // flagged at plan creation
       const float wt = om * P.w[e];
-      const uint4* src = reinterpret_cast<const uint4*>(base + static_cast<int64_t>(k) * P.d_s);
+      const int64_t kr = P.srow ? __ldg(P.srow + k) : k;
+      const uint4* src = reinterpret_cast<const uint4*>(base + kr * P.d_s);
       uint4 x[8];
 #pragma unroll
       for (int k2 = 0; k2 < 8; ++k2) x[k2] = __ldg(src + k2);
@@ -363,12 +366,13 @@ __device__ __forceinline__ void build_stage_unrotated(const XferParams& P, const
     for (int ti = 0; ti < segs.n_terms[seg]; ++ti) {
       const int tl = segs.layer[seg][ti];
       const float om = segs.w[seg][ti];
-      const T* base = sender + (static_cast<int64_t>(tl * 2 + c) * P.T_s) * P.d_s + elem0;
+      const T* base = sender + (static_cast<int64_t>(tl * 2 + c) * P.s_rows) * P.d_s + elem0;
       for (int e = e0; e < e1; ++e) {
         const int k = P.col[e];
         if (k < 0 || k >= P.T_s) continue;  // flagged at plan creation
         const float wt = om * P.w[e];
-        const T* row = base + static_cast<int64_t>(k) * P.d_s;
+        const int64_t kr = P.srow ? __ldg(P.srow + k) : k;
+        const T* row = base + kr * P.d_s;
         float x[kPerChunk], y[kPerChunk];
 #pragma unroll
         for (int i = 0; i < kPerChunk; ++i) x[i] = y[i] = 0.f;
@@ -432,7 +436,7 @@ __device__ __forceinline__ void gather_rows(const XferParams& P, uint8_t* sA, ui
     int64_t seg_base[kMaxSeg];
 #pragma unroll
     for (int s2 = 0; s2 < kMaxSeg; ++s2)
-      seg_base[s2] = (static_cast<int64_t>(P.segs[l].layer[s2][0] * 2 + c) * P.T_s) * P.d_s;
+      seg_base[s2] = (static_cast<int64_t>(P.segs[l].layer[s2][0] * 2 + c) * P.s_rows) * P.d_s;
     int64_t roff[8];
     uint32_t doff[8];
 #pragma unroll
@@ -1027,6 +1031,8 @@ hf_status launch_transfer(hf_plan_s* p, const void* sender, void* receiver, cuda
   P.n_distinct = reinterpret_cast<const int32_t*>(ws + p->lay.n_distinct);
   P.status = reinterpret_cast<int32_t*>(ws + p->lay.status);
   P.T_s = p->T_s;
+  P.s_rows = p->s_rows;
+  P.srow = p->span ? reinterpret_cast<const int32_t*>(ws + p->lay.srow) : nullptr;
   P.recv_rows = d.paged ? static_cast<int64_t>(d.n_blocks) * d.block_size : p->T_r;
   P.L_r = d.L_r;
   P.l0 = l_begin;

@@ -138,7 +138,7 @@ def job_from_workload(w, tok, sender, W, b, r, *, paged=None, knorm_w=None, r_po
     """TransferJob for a workloads.Workload and its generated inputs; the
     workload's optional descriptor fields are passed on."""
     from . import workloads as W_
-    opts = W_.desc_options(w)
+    opts = W_.desc_options(w, tok)
     opts.update(desc_options)
     pc = None
     if paged is not None:

@@ -68,6 +68,7 @@ class Workload:
     sender_k_rotated: bool = False     # sender keys stored with RoPE (base theta_s)
     s_pos0: Optional[Tuple[int, ...]] = None
     rope_table: bool = False           # receiver RoPE from a caller table (inv_freq_r_table)
+    span_gap: int = 0                  # message spans: cache rows before each request's span
 
     @property
     def d_s(self) -> int:
@@ -283,9 +284,28 @@ def explicit_table(L_s: int, L_r: int, n_seg: int, n_terms: int, seed: int):
             tuple(tuple(tuple(float(x) for x in t) for t in s) for s in weights))
 
 
-def desc_options(w: Workload) -> dict:
+def span_layout(w: Workload, tok) -> Optional[Tuple[np.ndarray, int]]:
+    """Message spans: each request's sender span sits after span_gap context
+    rows of its own, so request q's span starts at cache row
+    (q + 1) * span_gap + s_tok_ptr[q]; returns (s_row0, sender_rows)."""
+    if w.span_gap <= 0:
+        return None
+    ptr = np.asarray(tok.s_tok_ptr, np.int64)
+    s_row0 = (np.arange(1, len(ptr)) * w.span_gap + ptr[:-1]).astype(np.int32)
+    return s_row0, int(ptr[-1] + (len(ptr) - 1) * w.span_gap)
+
+
+def sender_cache_rows(w: Workload, tok) -> int:
+    sp = span_layout(w, tok)
+    return tok.T_s if sp is None else sp[1]
+
+
+def desc_options(w: Workload, tok=None) -> dict:
     """The optional descriptor fields a workload asks for."""
     opts = {}
+    if w.span_gap > 0:
+        s_row0, rows = span_layout(w, tok)
+        opts.update(s_row0=s_row0, sender_rows=rows)
     if w.layer_mode == "explicit":
         opts.update(seg_layer=np.asarray(w.seg_layer, np.int32),
                     seg_w=np.asarray(w.seg_w, np.float32))

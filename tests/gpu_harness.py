@@ -64,7 +64,7 @@ class Case:
         self.w = w
         self.dev = torch.device(device)
         self.tok = W.tokens(w)
-        self.sender = W.sender_kv(w, self.tok.T_s, self.dev)
+        self.sender = W.sender_kv(w, W.sender_cache_rows(w, self.tok), self.dev)
         self.Wm, self.b, self.r = W.maps(w, self.dev)
         self.paged = W.paged_layout(w, self.tok) if w.paged else None
         self.knorm_w = W.knorm_weight(w)
@@ -84,6 +84,8 @@ class Case:
         table = W.inv_freq_r_table(w)
         self.inv_freq_r = (O.rope_inv_freq(w.theta_r, w.D_r) if table is None
                            else table.astype(np.float64))
+        sp = W.span_layout(w, self.tok)
+        self.sender_row_of = None if sp is None else O.span_rows(self.tok.s_tok_ptr, sp[0])
         self.sender_rope = None
         if w.sender_k_rotated:
             self.sender_rope = (O.sender_positions(self.tok.s_tok_ptr, W.s_pos0(w)),
@@ -122,7 +124,8 @@ class Case:
                           self.b.cpu().numpy(), self.r, H_r=self.w.H_r, D_r=self.w.D_r,
                           pos=self.pos, inv_freq_r=self.inv_freq_r,
                           knorm_g=self.knorm_w, knorm_eps=1e-6, layers=layers, rows=rows,
-                          roles=roles, sender_rope=self.sender_rope)
+                          roles=roles, sender_rope=self.sender_rope,
+                          sender_row_of=self.sender_row_of)
 
     def check_parity(self, layers=None, rows=None, rel_tol=REL_FRO_TOL, abs_tol=MAX_ABS_TOL):
         layers = list(range(self.w.L_r)) if layers is None else list(layers)

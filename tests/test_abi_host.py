@@ -73,6 +73,9 @@ def _desc(B, **over):
     (dict(sender_k_rotated=True, theta_s=1e4, D_s=256, H_s=1), 2),  # head wider than a stage
     (dict(sender_k_rotated=True, theta_s=1e4, D_s=64, H_s=1), 2),   # d_S = 64: not whole stages
     (dict(inv_freq_r=np.full(16, np.inf)), 1),
+    (dict(s_row0=[3], sender_rows=7), 1),             # span of 5 rows from row 3 > 7 rows
+    (dict(s_row0=[-1], sender_rows=70), 1),
+    (dict(sender_rows=4), 1),                         # fewer cache rows than sender tokens
 ])
 def test_plan_create_rejects(B, over, status):
     d = _desc(B, **over)
@@ -139,7 +142,8 @@ def test_optional_fields_validate(B):
     ok = [dict(layer_mode="explicit", seg_layer=np.zeros((6, 2, 2)), seg_w=0.5),
           dict(sender_k_rotated=True, theta_s=5e5, s_pos0=[3]),
           dict(sender_k_rotated=True, inv_freq_s=np.ones(32)),
-          dict(inv_freq_r=np.linspace(1.0, 1e-3, 16), theta_r=0.0)]
+          dict(inv_freq_r=np.linspace(1.0, 1e-3, 16), theta_r=0.0),
+          dict(s_row0=[60], sender_rows=65)]
     for over in ok:
         d = _desc(B, **over)
         need = B.plan_workspace_size(d)

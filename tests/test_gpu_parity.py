@@ -176,6 +176,12 @@ EDGE = {
         W.llama_to_ministral(400).with_(L_s=6, L_r=3), n_seg=3, n_terms=1, unit=True),
     "rope_table": lambda: W.llama_to_ministral(600).with_(L_s=4, L_r=3, rope_table=True,
                                                           r_pos0=(5000,)),
+    # message spans after a context (only the span's K/V is mapped)
+    "message_spans_batched_paged": lambda: W.qwen25_to_llama_batched(
+        n_req=3, lo=40, hi=160, seed=12).with_(L_s=4, L_r=3, span_gap=700),
+    "message_span_rotated_overlap": lambda: W.llama_to_ministral(150).with_(
+        L_s=3, L_r=3, span_gap=2000, sender_k_rotated=True, s_pos0=(2000,),
+        align_mode="overlap_mean", r_pos0=(1500,)),
 }
 
 
