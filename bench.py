@@ -432,10 +432,115 @@ def run_ours(args):
     return 0
 
 
+def run_batch(args):
+    """A three-agent message round: six directions (every family pair), each
+    a message span after a context, transferred by one hf_transfer_batch
+    call per step; the same directions one hf_transfer after another are
+    timed beside it."""
+    import numpy as np
+    import torch
+    if not torch.cuda.is_available():
+        print(json.dumps({"error": "no CUDA device"}))
+        return 1
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    import __graft_entry__ as g
+    g.build()
+    from paper_2609_32259_gb300 import binding as B, pipeline, workloads as W
+    ws = W.message_round()
+    jobs, works = [], []
+    for w in ws:
+        tok = W.tokens(w)
+        sender = W.sender_kv(w, W.sender_cache_rows(w, tok), dev)
+        Wm, b, r = W.maps(w, dev)
+        jobs.append(pipeline.job_from_workload(w, tok, sender, Wm, b, r, device=dev))
+        works.append((w, tok))
+    stream = torch.cuda.current_stream(dev)
+
+    def prepare():
+        for j in jobs:
+            j.align(stream)
+            j.make_plan(stream)
+
+    def batch():
+        B.transfer_batch([j.plan for j in jobs], [j.sender for j in jobs],
+                         [j.receiver for j in jobs], stream)
+
+    def sequential():
+        for j in jobs:
+            j.transfer(stream)
+
+    for _ in range(max(3, args.warmup)):
+        prepare()
+        batch()
+        sequential()
+    torch.cuda.synchronize()
+    status = max(j.device_status() for j in jobs)
+    flops = bytes_ = 0.0
+    T_total = 0
+    for (w, tok), j in zip(works, jobs):
+        _, col, _ = j.csr()
+        f, by = algorithmic_work(w, tok, j.distinct_rows(), int(np.unique(col).size))
+        flops += f
+        bytes_ += by
+        T_total += tok.T_r
+    res = {}
+    clocks = ClockSampler(0)
+    clocks.start()
+    time.sleep(0.3)
+    for name, fn in (("batch", batch), ("sequential", sequential)):
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(args.steps)]
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        t0.record(stream)
+        for i in range(args.steps):
+            prepare()
+            ev[i][0].record(stream)
+            fn()
+            ev[i][1].record(stream)
+        t1.record(stream)
+        torch.cuda.synchronize()
+        res[name] = (t0.elapsed_time(t1) / args.steps,
+                     statistics.mean(a.elapsed_time(bb) for a, bb in ev))
+    clk = clocks.stop()
+    step_ms, kern_ms = res["batch"]
+    hbm_gbs, tflops, tflops_sust, src = peaks()
+    t_k = kern_ms * 1e-3
+    if flops / (tflops * 1e12) >= bytes_ / (hbm_gbs * 1e9):
+        roof = {"bound": "tensor", "achieved": flops / t_k / 1e12, "peak": tflops,
+                "unit": "TFLOP/s", "frac": flops / t_k / 1e12 / tflops}
+    else:
+        roof = {"bound": "hbm", "achieved": bytes_ / t_k / 1e9, "peak": hbm_gbs,
+                "unit": "GB/s", "frac": bytes_ / t_k / 1e9 / hbm_gbs}
+    roof.update({"traffic": None, "peak_source": src, "kernel": "transfer_kernel x6",
+                 "kernel_ms": kern_ms, "flop_alg": flops, "bytes_alg": bytes_})
+    line = {
+        "metric": METRIC, "value": T_total / (step_ms * 1e-3), "unit": UNIT, "n_gpus": 1,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_ms,
+        "us_per_transfer_kernel": kern_ms * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": "message_round_6x160", "directions": [w.name for w in ws],
+                   "T_r_total": T_total, "context_tokens": ws[0].span_gap,
+                   "sequential_kernel_ms": res["sequential"][1],
+                   "sequential_step_ms": res["sequential"][0],
+                   "l2": "inputs smaller than L2 (no flush; maps 1.2 GB are not)",
+                   "parallelism": "single"},
+        "roofline": roof, "cpu_baseline": None, "e2e": None, "clocks": clk,
+        "gpu_launches": (8 * len(jobs)) * args.steps, "device_status": status,
+    }
+    print(json.dumps(line), flush=True)
+    for j in jobs:
+        j.close()
+    return 0
+
+
 def main():
     args = parse()
     if args.impl == "reference":
         return run_reference(args)
+    if args.workload == "message_round":
+        return run_batch(args)
     return run_ours(args)
 
 

@@ -286,6 +286,20 @@ hf_status hf_transfer_host(hf_plan plan, const void* h_sender_kv, void* d_sender
                            void* d_receiver_kv, void* h_receiver_kv, int32_t n_groups,
                            hf_stream_t stream);
 
+/*
+ * hf_transfer_batch — several transfer directions in one call (a
+ * multi-agent round sends each message to receivers of other model
+ * families; Appendix "HiddenBench Evaluation").  Direction i is
+ * hf_transfer(plans[i], sender_kv[i], receiver_kv[i]); the kernels run on
+ * streams of a per-device pool forked from `stream`, so each direction's
+ * CTA pairs start as the previous one's retire, and `stream` is ordered
+ * after all of them.  n in [0, 16]; a plan appears at most once; the
+ * receiver caches must not overlap.  Asynchronous; the pool's streams are
+ * created on the first call on a device.
+ */
+hf_status hf_transfer_batch(const hf_plan* plans, const void* const* sender_kv,
+                            void* const* receiver_kv, int32_t n, hf_stream_t stream);
+
 /* Frees the plan's host memory and its copy streams.  Does not touch the
    workspace. */
 hf_status hf_plan_destroy(hf_plan plan);

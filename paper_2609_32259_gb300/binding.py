@@ -37,7 +37,8 @@ CHECK_BITS = {
 
 EXPORTED = ("hf_align_build", "hf_plan_workspace_size", "hf_plan_create", "hf_transfer",
             "hf_plan_destroy", "hf_plan_device_status", "hf_plan_distinct_rows",
-            "hf_status_string", "hf_last_error", "hf_transfer_noalloc", "hf_transfer_host")
+            "hf_status_string", "hf_last_error", "hf_transfer_noalloc", "hf_transfer_host",
+            "hf_transfer_batch")
 
 _p = ctypes.c_void_p
 _i32p = ctypes.POINTER(ctypes.c_int32)
@@ -98,6 +99,8 @@ def lib() -> ctypes.CDLL:
         L.hf_transfer_noalloc.restype = ctypes.c_int
         L.hf_transfer_host.argtypes = [_p, _p, _p, _p, _p, ctypes.c_int32, _p]
         L.hf_transfer_host.restype = ctypes.c_int
+        L.hf_transfer_batch.argtypes = [_p, _p, _p, ctypes.c_int32, _p]
+        L.hf_transfer_batch.restype = ctypes.c_int
         L.hf_status_string.argtypes = [ctypes.c_int]
         L.hf_status_string.restype = ctypes.c_char_p
         L.hf_last_error.argtypes = []
@@ -252,6 +255,15 @@ def transfer_host(plan: Plan, h_sender_kv, d_sender_kv, d_receiver_kv, h_receive
     _check(lib().hf_transfer_host(plan.handle, _dptr(h_sender_kv), _dptr(d_sender_kv),
                                   _dptr(d_receiver_kv), _dptr(h_receiver_kv), int(n_groups),
                                   _stream(stream)), "hf_transfer_host")
+
+
+def transfer_batch(plans, senders, receivers, stream=None) -> None:
+    """hf_transfer_batch: direction i = (plans[i], senders[i], receivers[i])."""
+    n = len(plans)
+    hp = (ctypes.c_void_p * max(n, 1))(*[p.handle for p in plans])
+    sp = (ctypes.c_void_p * max(n, 1))(*[_dptr(x) for x in senders])
+    rp = (ctypes.c_void_p * max(n, 1))(*[_dptr(x) for x in receivers])
+    _check(lib().hf_transfer_batch(hp, sp, rp, n, _stream(stream)), "hf_transfer_batch")
 
 
 def transfer_noalloc(desc: Desc, sender_kv, receiver_kv, stream=None) -> None:

@@ -16,6 +16,7 @@ constexpr int kMaxLayersR = 128;     // receiver layers
 constexpr int kMaxSeg = 3;           // map input segments per receiver layer
 constexpr int kMaxTerms = 2;         // sender layers blended into one segment
 constexpr int kMaxHeadDim = 256;
+constexpr int kMaxBatch = 16;        // directions per hf_transfer_batch call
 
 // One receiver layer's map input: n_seg segments of d_S features each;
 // segment s is sum_t w[s][t] * (pooled sender layer layer[s][t]).

@@ -140,6 +140,41 @@ def ministral_to_llama(T_r: int) -> Workload:
 
 SWEEP_TOKENS = (256, 512, 1024, 4096, 16384, 32768, 65536, 131072)
 
+# Model shapes (layers, KV heads, head width, RoPE base, characters per token).
+MODEL_SHAPES = {
+    "llama8b": (32, 8, 128, 500000.0, 4.0),
+    "qwen25_7b": (28, 4, 128, 1e6, 3.6),
+    "ministral": (40, 8, 128, 1e8, 3.6),
+}
+
+
+def direction(sender: str, receiver: str, T_r: int, seed: int, **kw) -> Workload:
+    """A transfer between two of MODEL_SHAPES."""
+    Ls, Hs, Ds, ths, ms = MODEL_SHAPES[sender]
+    Lr, Hr, Dr, thr, mr = MODEL_SHAPES[receiver]
+    return Workload(f"{sender}_to_{receiver}_{T_r}", L_s=Ls, H_s=Hs, D_s=Ds, L_r=Lr, H_r=Hr,
+                    D_r=Dr, theta_s=ths, theta_r=thr, r_tokens=(T_r,), mean_s=ms, mean_r=mr,
+                    seed=seed, **kw)
+
+
+def message_round(msg_tokens: int = 160, ctx_tokens: int = 2048, seed: int = 20):
+    """One communication round of three agents of different families (the
+    multi-agent setting of the paper's HiddenBench evaluation): every agent's
+    message goes to the two others, six directions.  Each message is a span
+    of msg_tokens receiver tokens that follows ctx_tokens of context in the
+    sender's cache; the receiver places it after its own context."""
+    names = ("llama8b", "qwen25_7b", "ministral")
+    out = []
+    k = 0
+    for a in names:
+        for b in names:
+            if a == b:
+                continue
+            out.append(direction(a, b, msg_tokens, seed + k, span_gap=ctx_tokens,
+                                 r_pos0=(ctx_tokens,)))
+            k += 1
+    return out
+
 
 # ---------------------------------------------------------------------------
 # Segmentations

@@ -1,0 +1,56 @@
+"""hf_transfer_batch: the six directions of a three-agent message round
+(message spans after a context, every family pair) in one call.  Each
+direction must equal, bit for bit, its own hf_transfer (the same kernel on
+the same inputs), and match the fp64 oracle within the parity tolerance."""
+
+import numpy as np
+import pytest
+import torch
+
+from gpu_harness import Case
+from paper_2609_32259_gb300 import binding as B
+from paper_2609_32259_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+SENTINEL = 99.0
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import __graft_entry__ as g
+
+    g.build()
+
+
+def test_message_round_batch_matches_single_transfers_and_oracle():
+    cases = [Case(w, sentinel=SENTINEL).run() for w in W.message_round(msg_tokens=160)]
+    single = [c.job.receiver.clone() for c in cases]
+    for c in cases:
+        c.job.receiver.fill_(SENTINEL)
+    B.transfer_batch([c.job.plan for c in cases], [c.sender for c in cases],
+                     [c.job.receiver for c in cases])
+    torch.cuda.synchronize()
+    for c, ref in zip(cases, single):
+        assert torch.equal(c.job.receiver, ref), c.w.name
+        c.check_parity()
+
+
+def test_batch_of_one_and_empty_batch():
+    c = Case(W.message_round(msg_tokens=40)[1], sentinel=SENTINEL).run()
+    ref = c.job.receiver.clone()
+    c.job.receiver.fill_(SENTINEL)
+    B.transfer_batch([c.job.plan], [c.sender], [c.job.receiver])
+    B.transfer_batch([], [], [])
+    torch.cuda.synchronize()
+    assert torch.equal(c.job.receiver, ref)
+
+
+def test_batch_rejects_a_repeated_plan():
+    c = Case(W.message_round(msg_tokens=40)[0]).run()
+    with pytest.raises(B.HFError) as e:
+        B.transfer_batch([c.job.plan, c.job.plan], [c.sender, c.sender],
+                         [c.job.receiver, c.job.receiver])
+    assert e.value.status == B.HF_ERR_INVALID_ARGUMENT
