@@ -23,6 +23,9 @@ What it computes (arxiv 2609.32259, "HeteroFold"):
   clipped neighbourhood N(l) = (pi-4, pi, pi+4); plus the two-layer linear
   interpolation reading.
 * Feature concatenation, Eq. 2: x = [c^{t1} || c^{t2} || c^{t3}].
+* The output-aware low-rank correction, Eq. 7: y_hat = y0 + (y0 B) G with
+  y0 = (x / r) A + b, and its folding, Eq. 9: A_final = A (I + B G),
+  b_final = b (I + B G).
 * The folded inference map, Eq. 9: Phi(x) = (x / r) A_final + b_final,
   one map per receiver layer and role, reshaped to receiver KV heads; keys
   then get the receiver's key normalisation and RoPE at receiver positions
@@ -468,6 +471,46 @@ def span_rows(s_tok_ptr: Sequence[int], s_row0: Sequence[int]) -> np.ndarray:
         for t in range(int(s_tok_ptr[q + 1]) - int(s_tok_ptr[q])):
             out.append(int(s_row0[q]) + t)
     return np.asarray(out, dtype=np.int64)
+
+
+def fold(A: np.ndarray, b: np.ndarray, B: np.ndarray, G: np.ndarray):
+    """Eq. 9 (folding for inference): A_final = A (I + B G), b_final =
+    b (I + B G), for one receiver layer and role.  A: [K, d_R], b: [d_R],
+    B: [d_R, rho], G: [rho, d_R]."""
+    A = np.asarray(A, dtype=np.float64)
+    b = np.asarray(b, dtype=np.float64)
+    M = np.eye(A.shape[1]) + np.asarray(B, dtype=np.float64) @ np.asarray(G, dtype=np.float64)
+    return A @ M, b @ M
+
+
+def transfer_unfused(sender, csr: CSR, segments, A, b, r, B, G, *, H_r: int, D_r: int,
+                     pos: np.ndarray, inv_freq_r: np.ndarray,
+                     knorm_g: Optional[np.ndarray] = None, knorm_eps: float = 1e-6,
+                     layers: Optional[Iterable[int]] = None,
+                     rows: Optional[np.ndarray] = None,
+                     roles: Iterable[int] = (ROLE_K, ROLE_V)) -> Dict[Tuple[int, int], np.ndarray]:
+    """The receiver cache entries with the correction applied unfolded,
+    in the order the paper defines it: y0 = (x / r) A + b (Eq. 5, the
+    Recolor map), y_hat = y0 + (y0 B) G (Eq. 7), then heads, key norm and RoPE as in
+    transfer().  B[l][c]: [d_R, rho], G[l][c]: [rho, d_R]."""
+    n_rows_total = csr.n_rows
+    rows = np.arange(n_rows_total) if rows is None else np.asarray(rows, dtype=np.int64)
+    layers = range(len(segments)) if layers is None else layers
+    out: Dict[Tuple[int, int], np.ndarray] = {}
+    for l in layers:
+        for c in roles:
+            x = map_input(sender, csr, segments[l], c, rows)
+            A_lc = np.asarray(A[l][c], dtype=np.float64)
+            y0 = (x / float(r[l][c])) @ A_lc + np.asarray(b[l][c], dtype=np.float64)
+            y = y0 + (y0 @ np.asarray(B[l][c], dtype=np.float64)) @ np.asarray(G[l][c],
+                                                                               dtype=np.float64)
+            y = y.reshape(len(rows), H_r, D_r)
+            if c == ROLE_K:
+                if knorm_g is not None:
+                    y = key_norm(y, knorm_g, knorm_eps)
+                y = rope(y, np.asarray(pos)[rows], inv_freq_r)
+            out[(l, c)] = y
+    return out
 
 
 def receiver_positions(r_tok_ptr: Sequence[int], r_pos0: Optional[Sequence[int]] = None) -> np.ndarray:

@@ -518,6 +518,56 @@ def check_identity_map_reproduces_input():
         assert np.allclose(out[(l, 0)][..., D // 2:], zc.imag)
 
 
+def check_fold_closed_forms():
+    """Eq. 9 folding: G = 0 leaves the map unchanged; a rank-1 correction
+    B = u, G = v^T gives A + (A u) v^T element by element; B = e_i, G = -e_i^T
+    removes output feature i (I + B G is a projector)."""
+    rng = np.random.default_rng(17)
+    K, d, rho = 7, 5, 3
+    A = rng.normal(size=(K, d))
+    b = rng.normal(size=d)
+    Af, bf = O.fold(A, b, rng.normal(size=(d, rho)), np.zeros((rho, d)))
+    assert np.array_equal(Af, A) and np.array_equal(bf, b)
+    u = rng.normal(size=(d, 1))
+    v = rng.normal(size=(1, d))
+    Af, bf = O.fold(A, b, u, v)
+    for k in range(K):
+        au = sum(A[k, n] * u[n, 0] for n in range(d))
+        for n in range(d):
+            assert abs(Af[k, n] - (A[k, n] + au * v[0, n])) < 1e-12
+    bu = sum(b[n] * u[n, 0] for n in range(d))
+    assert np.allclose(bf, b + bu * v[0])
+    i = 2
+    e = np.zeros((d, 1))
+    e[i, 0] = 1.0
+    Af, bf = O.fold(A, b, e, -e.T)
+    assert np.allclose(Af[:, i], 0.0) and abs(bf[i]) < 1e-12
+    keep = [n for n in range(d) if n != i]
+    assert np.allclose(Af[:, keep], A[:, keep]) and np.allclose(bf[keep], b[keep])
+
+
+def check_fold_equals_unfused_correction():
+    """Eq. 7 applied at transfer time (y0 + (y0 B) G, then key norm and RoPE)
+    equals the transfer with the Eq. 9 folded maps, keys and values."""
+    P = _tiny_problem(18, O.ALIGN_OVERLAP_MEAN, O.LAYER_PAPER3)
+    rng = np.random.default_rng(18)
+    L_r, d_r = P["A"].shape[0], P["A"].shape[3]
+    Bm = rng.normal(size=(L_r, 2, d_r, 2)) * 0.3
+    Gm = rng.normal(size=(L_r, 2, 2, d_r)) * 0.3
+    Af = np.zeros_like(P["A"])
+    bf = np.zeros_like(P["b"])
+    for l in range(L_r):
+        for c in range(2):
+            Af[l, c], bf[l, c] = O.fold(P["A"][l, c], P["b"][l, c], Bm[l, c], Gm[l, c])
+    g = rng.uniform(0.5, 1.5, size=P["D_r"])
+    folded = _run_oracle(dict(P, A=Af, b=bf), knorm_g=g)
+    unfused = O.transfer_unfused(P["sender"], P["csr"], P["segs"], P["A"], P["b"], P["r"], Bm, Gm,
+                                 H_r=P["H_r"], D_r=P["D_r"], pos=P["pos"], inv_freq_r=P["inv"],
+                                 knorm_g=g)
+    for key in unfused:
+        assert np.allclose(folded[key], unfused[key], rtol=1e-10, atol=1e-10), key
+
+
 def _identity_setup(L, H, D, lengths, seed):
     d = H * D
     rng = np.random.default_rng(seed)
@@ -648,6 +698,7 @@ ALL_CHECKS = [
     check_explicit_segments, check_message_spans, check_identity_map_reproduces_input,
     check_identity_rotated_sender_keys, check_rotated_sender_position_shift,
     check_rotated_sender_unrotates_before_pooling,
+    check_fold_closed_forms, check_fold_equals_unfused_correction,
     check_affine_structure, check_segment_blocks,
 ]
 

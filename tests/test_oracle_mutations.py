@@ -124,6 +124,18 @@ def _span_rows_from_zero(s_tok_ptr, s_row0):
     return np.arange(int(s_tok_ptr[-1]), dtype=np.int64)
 
 
+def _fold_without_identity(A, b, B, G):
+    # wrong: A B G instead of A (I + B G)
+    M = np.asarray(B, dtype=np.float64) @ np.asarray(G, dtype=np.float64)
+    return np.asarray(A, dtype=np.float64) @ M, np.asarray(b, dtype=np.float64) @ M
+
+
+def _fold_bias_unchanged(A, b, B, G):
+    # wrong: the bias is not folded
+    M = np.eye(np.asarray(A).shape[1]) + np.asarray(B) @ np.asarray(G)
+    return np.asarray(A, dtype=np.float64) @ M, np.asarray(b, dtype=np.float64)
+
+
 def _explicit_weights_swapped(seg_layer, seg_w):
     return [[[(int(t), float(w)) for t, w in zip(ts, reversed(ws))] for ts, ws in zip(ls, wl)]
             for ls, wl in zip(seg_layer, seg_w)]
@@ -181,6 +193,8 @@ MUTATIONS = {
     "values_unrotated": ("map_input", _map_input_unrotates_values),
     "explicit_weights_swapped": ("explicit_segments", _explicit_weights_swapped),
     "span_rows_from_zero": ("span_rows", _span_rows_from_zero),
+    "fold_without_identity": ("fold", _fold_without_identity),
+    "fold_bias_unchanged": ("fold", _fold_bias_unchanged),
 }
 
 
