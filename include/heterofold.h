@@ -333,6 +333,26 @@ hf_status hf_plan_distinct_rows(hf_plan plan, hf_stream_t stream, int32_t* n_row
 hf_status hf_transfer_noalloc(const hf_plan_desc* desc, const void* sender_kv,
                               void* receiver_kv, hf_stream_t stream);
 
+/*
+ * hf_fold — folds the output-aware low-rank correction of Eq. 7,
+ * y_hat = y0 + (y0 B) G, into the affine maps (Eq. 9):
+ * A_final = A (I + B G), b_final = b (I + B G), for n_maps maps at once
+ * (e.g. every receiver layer and role), in the layout hf_plan_desc takes.
+ * Offline: run once per model pair, before plans that use the maps.
+ * d_W:       device [n_maps][d_R][K] in `dtype`: W = A^T, as d_W of
+ *            hf_plan_desc.
+ * d_b:       device float[n_maps][d_R].
+ * d_B:       device float[n_maps][d_R][rank]; d_G: float[n_maps][rank][d_R].
+ * d_W_final: device, like d_W (may be d_W itself: folded in place);
+ *            rounded once to `dtype`.
+ * d_b_final: device float[n_maps][d_R] (may be d_b).
+ * rank 4, 8, 16 or 32 (the paper uses 16); K even; d_W, d_W_final and
+ * d_B 16-byte aligned.  Asynchronous on `stream`.
+ */
+hf_status hf_fold(hf_dtype dtype, int32_t n_maps, int32_t d_R, int64_t K, int32_t rank,
+                  const void* d_W, const float* d_b, const float* d_B, const float* d_G,
+                  void* d_W_final, float* d_b_final, hf_stream_t stream);
+
 const char* hf_status_string(hf_status status);
 const char* hf_last_error(void);
 

@@ -38,7 +38,7 @@ CHECK_BITS = {
 EXPORTED = ("hf_align_build", "hf_plan_workspace_size", "hf_plan_create", "hf_transfer",
             "hf_plan_destroy", "hf_plan_device_status", "hf_plan_distinct_rows",
             "hf_status_string", "hf_last_error", "hf_transfer_noalloc", "hf_transfer_host",
-            "hf_transfer_batch")
+            "hf_transfer_batch", "hf_fold")
 
 _p = ctypes.c_void_p
 _i32p = ctypes.POINTER(ctypes.c_int32)
@@ -101,6 +101,9 @@ def lib() -> ctypes.CDLL:
         L.hf_transfer_host.restype = ctypes.c_int
         L.hf_transfer_batch.argtypes = [_p, _p, _p, ctypes.c_int32, _p]
         L.hf_transfer_batch.restype = ctypes.c_int
+        L.hf_fold.argtypes = [ctypes.c_int, ctypes.c_int32, ctypes.c_int32, ctypes.c_int64,
+                              ctypes.c_int32, _p, _p, _p, _p, _p, _p, _p]
+        L.hf_fold.restype = ctypes.c_int
         L.hf_status_string.argtypes = [ctypes.c_int]
         L.hf_status_string.restype = ctypes.c_char_p
         L.hf_last_error.argtypes = []
@@ -264,6 +267,15 @@ def transfer_batch(plans, senders, receivers, stream=None) -> None:
     sp = (ctypes.c_void_p * max(n, 1))(*[_dptr(x) for x in senders])
     rp = (ctypes.c_void_p * max(n, 1))(*[_dptr(x) for x in receivers])
     _check(lib().hf_transfer_batch(hp, sp, rp, n, _stream(stream)), "hf_transfer_batch")
+
+
+def fold(dtype: str, W, b, B, G, W_final, b_final, stream=None) -> None:
+    """hf_fold (Eq. 9): W [n_maps, d_R, K], b [n_maps, d_R], B [n_maps, d_R, rank],
+    G [n_maps, rank, d_R] (torch device tensors; W_final/b_final may alias)."""
+    n_maps, d_R, K = (int(x) for x in W.shape)
+    rank = int(B.shape[-1])
+    _check(lib().hf_fold(DTYPES[dtype], n_maps, d_R, K, rank, _dptr(W), _dptr(b), _dptr(B),
+                         _dptr(G), _dptr(W_final), _dptr(b_final), _stream(stream)), "hf_fold")
 
 
 def transfer_noalloc(desc: Desc, sender_kv, receiver_kv, stream=None) -> None:
