@@ -23,6 +23,12 @@ What it computes (arxiv 2609.32259, "HeteroFold"):
   clipped neighbourhood N(l) = (pi-4, pi, pi+4); plus the two-layer linear
   interpolation reading.
 * Feature concatenation, Eq. 2: x = [c^{t1} || c^{t2} || c^{t3}].
+* Recolor fitting (Section 3.2 "Moment-Matched Recoloring", Eq. 3-5): the
+  sender RMS r over weighted samples (Eq. 3), weighted means and
+  covariances of Z = X / r and Y, whitening and Procrustes alignment through
+  the thin SVD of Sigma_Z^{-1/2} Sigma_ZY Sigma_Y^{-1/2} = U Lambda Q^T,
+  R* = U Q^T (Eq. 4), and A = Sigma_Z^{-1/2} R* Sigma_Y^{1/2},
+  b = mu_Y - mu_Z A (Eq. 5).
 * The output-aware low-rank correction, Eq. 7: y_hat = y0 + (y0 B) G with
   y0 = (x / r) A + b, and its folding, Eq. 9: A_final = A (I + B G),
   b_final = b (I + B G).
@@ -471,6 +477,59 @@ def span_rows(s_tok_ptr: Sequence[int], s_row0: Sequence[int]) -> np.ndarray:
         for t in range(int(s_tok_ptr[q + 1]) - int(s_tok_ptr[q])):
             out.append(int(s_row0[q]) + t)
     return np.asarray(out, dtype=np.int64)
+
+
+def sender_rms(X: np.ndarray, w: np.ndarray) -> float:
+    """Eq. 3: r = sqrt(sum_n w_n |x_n|^2 / (d~_S sum_n w_n)), one scalar over
+    all weighted samples and feature dimensions."""
+    X = np.asarray(X, dtype=np.float64)
+    w = np.asarray(w, dtype=np.float64)
+    return float(np.sqrt(np.sum(w * np.sum(X * X, axis=1)) / (X.shape[1] * np.sum(w))))
+
+
+def weighted_moments(Z: np.ndarray, Y: np.ndarray, w: np.ndarray):
+    """Weighted means, covariances and cross-covariance (normalised by
+    sum w): mu_Z, mu_Y, Sigma_Z, Sigma_Y, Sigma_ZY."""
+    Z = np.asarray(Z, dtype=np.float64)
+    Y = np.asarray(Y, dtype=np.float64)
+    w = np.asarray(w, dtype=np.float64)
+    W = np.sum(w)
+    mu_z = (w @ Z) / W
+    mu_y = (w @ Y) / W
+    Zc = Z - mu_z
+    Yc = Y - mu_y
+    return (mu_z, mu_y, (Zc * w[:, None]).T @ Zc / W, (Yc * w[:, None]).T @ Yc / W,
+            (Zc * w[:, None]).T @ Yc / W)
+
+
+def _sym_power(S: np.ndarray, p: float) -> np.ndarray:
+    """S^p of a symmetric positive definite matrix through its eigenvectors."""
+    lam, V = np.linalg.eigh(S)
+    return (V * lam ** p) @ V.T
+
+
+def recolor(X: np.ndarray, Y: np.ndarray, w: np.ndarray, reg: float = 0.0):
+    """Recolor fit (Eq. 3-5) for one receiver layer and role.
+
+    X: [N, d~_S] sender features (Eq. 2 concatenation), Y: [N, d_R] receiver
+    targets, w: [N] sample weights.  reg: numerical stabilisation, read as a
+    ridge of reg * (mean eigenvalue) added to each covariance (the paper
+    stabilises without giving the form).  Returns (A [d~_S, d_R], b [d_R], r).
+    """
+    r = sender_rms(X, w)
+    Z = np.asarray(X, dtype=np.float64) / r
+    mu_z, mu_y, S_z, S_y, S_zy = weighted_moments(Z, Y, w)
+    if reg > 0.0:
+        S_z = S_z + reg * np.trace(S_z) / S_z.shape[0] * np.eye(S_z.shape[0])
+        S_y = S_y + reg * np.trace(S_y) / S_y.shape[0] * np.eye(S_y.shape[0])
+    Sz_ih = _sym_power(S_z, -0.5)
+    Sy_ih = _sym_power(S_y, -0.5)
+    Sy_h = _sym_power(S_y, 0.5)
+    U, _lam, Qt = np.linalg.svd(Sz_ih @ S_zy @ Sy_ih, full_matrices=False)
+    R = U @ Qt
+    A = Sz_ih @ R @ Sy_h
+    b = mu_y - mu_z @ A
+    return A, b, r
 
 
 def fold(A: np.ndarray, b: np.ndarray, B: np.ndarray, G: np.ndarray):

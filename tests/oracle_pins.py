@@ -518,6 +518,74 @@ def check_identity_map_reproduces_input():
         assert np.allclose(out[(l, 0)][..., D // 2:], zc.imag)
 
 
+def _recolor_data(seed, N, d_s, d_r, noise):
+    rng = np.random.default_rng(seed)
+    X = rng.normal(size=(N, d_s)) @ rng.normal(size=(d_s, d_s)) * 0.7 + rng.normal(size=d_s)
+    A_true = rng.normal(size=(d_s, d_r)) / np.sqrt(d_s)
+    Y = X @ A_true + 0.3 + noise * rng.normal(size=(N, d_r))
+    w = rng.uniform(0.5, 2.0, size=N)
+    return X, Y, w
+
+
+def check_sender_rms():
+    """Eq. 3: samples all of squared norm d~ s^2 give r = s, whatever the
+    weights; doubling every weight leaves r unchanged."""
+    rng = np.random.default_rng(19)
+    X = rng.normal(size=(50, 6))
+    X = X / np.linalg.norm(X, axis=1, keepdims=True) * np.sqrt(6) * 1.7
+    w = rng.uniform(0.1, 3.0, size=50)
+    assert abs(O.sender_rms(X, w) - 1.7) < 1e-12
+    X2 = rng.normal(size=(40, 5))
+    assert abs(O.sender_rms(X2, w[:40]) - O.sender_rms(X2, 2 * w[:40])) < 1e-12
+    # brute force
+    num = sum(w[n] * sum(X2[n, j] ** 2 for j in range(5)) for n in range(40))
+    assert abs(O.sender_rms(X2, w[:40]) - math.sqrt(num / (5 * sum(w[:40])))) < 1e-12
+
+
+def check_weighted_moments_brute_force():
+    rng = np.random.default_rng(20)
+    Z = rng.normal(size=(30, 4))
+    Y = rng.normal(size=(30, 3))
+    w = rng.uniform(0.2, 2.0, size=30)
+    mu_z, mu_y, S_z, S_y, S_zy = O.weighted_moments(Z, Y, w)
+    W = sum(w)
+    for i in range(4):
+        m = sum(w[n] * Z[n, i] for n in range(30)) / W
+        assert abs(mu_z[i] - m) < 1e-12
+        for j in range(3):
+            my = sum(w[n] * Y[n, j] for n in range(30)) / W
+            c = sum(w[n] * (Z[n, i] - m) * (Y[n, j] - my) for n in range(30)) / W
+            assert abs(S_zy[i, j] - c) < 1e-12
+    assert np.allclose(S_z, S_z.T) and np.allclose(S_y, S_y.T)
+
+
+def check_recolor_moment_identities():
+    """Eq. 5 (unregularised, nonsingular, d~_S >= d_R): mu_Z A + b = mu_Y and
+    A^T Sigma_Z A = Sigma_Y."""
+    X, Y, w = _recolor_data(21, 400, 7, 5, 0.5)
+    A, b, r = O.recolor(X, Y, w)
+    mu_z, mu_y, S_z, S_y, _ = O.weighted_moments(X / r, Y, w)
+    assert np.allclose(mu_z @ A + b, mu_y, atol=1e-10)
+    assert np.allclose(A.T @ S_z @ A, S_y, atol=1e-9)
+
+
+def check_recolor_recovers_an_exact_rotation():
+    """If Y = Z Q + c with Q orthogonal (d~_S = d_R), then Sigma_ZY =
+    Sigma_Z Q, the whitened cross-covariance is Q itself, R* = Q, and the
+    fit returns A = Q, b = c exactly."""
+    rng = np.random.default_rng(22)
+    d = 6
+    X = rng.normal(size=(300, d)) @ rng.normal(size=(d, d)) + 2.0
+    w = rng.uniform(0.5, 1.5, size=300)
+    Q, _ = np.linalg.qr(rng.normal(size=(d, d)))
+    c = rng.normal(size=d)
+    r = O.sender_rms(X, w)
+    Y = (X / r) @ Q + c
+    A, b, r2 = O.recolor(X, Y, w)
+    assert abs(r2 - r) < 1e-12
+    assert np.allclose(A, Q, atol=1e-9) and np.allclose(b, c, atol=1e-9)
+
+
 def check_fold_closed_forms():
     """Eq. 9 folding: G = 0 leaves the map unchanged; a rank-1 correction
     B = u, G = v^T gives A + (A u) v^T element by element; B = e_i, G = -e_i^T
@@ -699,6 +767,8 @@ ALL_CHECKS = [
     check_identity_rotated_sender_keys, check_rotated_sender_position_shift,
     check_rotated_sender_unrotates_before_pooling,
     check_fold_closed_forms, check_fold_equals_unfused_correction,
+    check_sender_rms, check_weighted_moments_brute_force, check_recolor_moment_identities,
+    check_recolor_recovers_an_exact_rotation,
     check_affine_structure, check_segment_blocks,
 ]
 

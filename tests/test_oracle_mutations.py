@@ -136,6 +136,40 @@ def _fold_bias_unchanged(A, b, B, G):
     return np.asarray(A, dtype=np.float64) @ M, np.asarray(b, dtype=np.float64)
 
 
+def _rms_unweighted(X, w):
+    X = np.asarray(X, dtype=np.float64)
+    return float(np.sqrt(np.mean(X * X)))
+
+
+_orig_recolor = O.recolor
+
+
+def _recolor_transposed_rotation(X, Y, w, reg=0.0):
+    # wrong: the transposed rotation (R*^T) where it is square
+    r = O.sender_rms(X, w)
+    Z = np.asarray(X, dtype=np.float64) / r
+    mu_z, mu_y, S_z, S_y, S_zy = O.weighted_moments(Z, Y, w)
+    lz, Vz = np.linalg.eigh(S_z)
+    ly, Vy = np.linalg.eigh(S_y)
+    Sz_ih = (Vz * lz ** -0.5) @ Vz.T
+    Sy_ih = (Vy * ly ** -0.5) @ Vy.T
+    Sy_h = (Vy * ly ** 0.5) @ Vy.T
+    U, _, Qt = np.linalg.svd(Sz_ih @ S_zy @ Sy_ih, full_matrices=False)
+    R = U @ Qt
+    A = Sz_ih @ (R.T if R.shape[0] == R.shape[1] else R) @ Sy_h
+    return A, mu_y - mu_z @ A, r
+
+
+def _recolor_no_whitening(X, Y, w, reg=0.0):
+    # wrong: Procrustes on the raw cross-covariance
+    r = O.sender_rms(X, w)
+    Z = np.asarray(X, dtype=np.float64) / r
+    mu_z, mu_y, S_z, S_y, S_zy = O.weighted_moments(Z, Y, w)
+    U, _, Qt = np.linalg.svd(S_zy, full_matrices=False)
+    A = U @ Qt
+    return A, mu_y - mu_z @ A, r
+
+
 def _explicit_weights_swapped(seg_layer, seg_w):
     return [[[(int(t), float(w)) for t, w in zip(ts, reversed(ws))] for ts, ws in zip(ls, wl)]
             for ls, wl in zip(seg_layer, seg_w)]
@@ -195,6 +229,9 @@ MUTATIONS = {
     "span_rows_from_zero": ("span_rows", _span_rows_from_zero),
     "fold_without_identity": ("fold", _fold_without_identity),
     "fold_bias_unchanged": ("fold", _fold_bias_unchanged),
+    "rms_unweighted": ("sender_rms", _rms_unweighted),
+    "recolor_transposed_rotation": ("recolor", _recolor_transposed_rotation),
+    "recolor_no_whitening": ("recolor", _recolor_no_whitening),
 }
 
 
