@@ -353,6 +353,35 @@ hf_status hf_fold(hf_dtype dtype, int32_t n_maps, int32_t d_R, int64_t K, int32_
                   const void* d_W, const float* d_b, const float* d_B, const float* d_G,
                   void* d_W_final, float* d_b_final, hf_stream_t stream);
 
+/*
+ * hf_recolor_fit — the Recolor initialisation of one map (Section 3.2,
+ * Eq. 3-5) from N weighted aligned sample pairs: r (Eq. 3), weighted means
+ * and covariances of Z = X / r and Y, R* the orthogonal polar factor of
+ * Sigma_Z^{-1/2} Sigma_ZY Sigma_Y^{-1/2} (the U Q^T of its thin SVD,
+ * Eq. 4), A = Sigma_Z^{-1/2} R* Sigma_Y^{1/2} and b = mu_Y - mu_Z A (Eq. 5).
+ * Offline (once per map before calibration and folding).
+ * d_X:  device [N][d_S] in `dtype`: Eq. 2 concatenated sender features
+ *       (d_S here is the map input width, 3 d_S of the plan in paper mode).
+ * d_Y:  device [N][d_R] in `dtype`: receiver targets.
+ * d_w:  device float[N], positive sample weights.
+ * reg:  numerical stabilisation: reg * (mean eigenvalue) is added to each
+ *       covariance's diagonal (0: none; the paper does not give its form).
+ * d_W_out: device [d_R][d_S] in `dtype`: A^T, the layout of hf_plan_desc's
+ *       d_W; d_b_out: device float[d_R]; h_r_out: host float, r (or NULL);
+ *       h_iters_out: host int32[3] (or NULL), the iterations taken by the
+ *       roots of Sigma_Z and Sigma_Y and by the polar factor.
+ * d_workspace: hf_recolor_workspace_size bytes, 256-byte aligned.
+ * Requires d_S >= d_R and N * d_S < 2^31.  Matrix roots and the polar
+ * factor use Newton-Schulz iterations in fp32; the call synchronises
+ * `stream` (convergence checks) and returns HF_ERR_DEVICE_CHECK if an
+ * iteration does not converge (raise reg).
+ */
+hf_status hf_recolor_workspace_size(int64_t N, int32_t d_S, int32_t d_R, size_t* bytes);
+hf_status hf_recolor_fit(hf_dtype dtype, int64_t N, int32_t d_S, int32_t d_R, const void* d_X,
+                         const void* d_Y, const float* d_w, float reg, void* d_W_out,
+                         float* d_b_out, float* h_r_out, int32_t* h_iters_out,
+                         void* d_workspace, size_t workspace_bytes, hf_stream_t stream);
+
 const char* hf_status_string(hf_status status);
 const char* hf_last_error(void);
 

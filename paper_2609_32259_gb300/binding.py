@@ -38,7 +38,7 @@ CHECK_BITS = {
 EXPORTED = ("hf_align_build", "hf_plan_workspace_size", "hf_plan_create", "hf_transfer",
             "hf_plan_destroy", "hf_plan_device_status", "hf_plan_distinct_rows",
             "hf_status_string", "hf_last_error", "hf_transfer_noalloc", "hf_transfer_host",
-            "hf_transfer_batch", "hf_fold")
+            "hf_transfer_batch", "hf_fold", "hf_recolor_workspace_size", "hf_recolor_fit")
 
 _p = ctypes.c_void_p
 _i32p = ctypes.POINTER(ctypes.c_int32)
@@ -104,6 +104,13 @@ def lib() -> ctypes.CDLL:
         L.hf_fold.argtypes = [ctypes.c_int, ctypes.c_int32, ctypes.c_int32, ctypes.c_int64,
                               ctypes.c_int32, _p, _p, _p, _p, _p, _p, _p]
         L.hf_fold.restype = ctypes.c_int
+        L.hf_recolor_workspace_size.argtypes = [ctypes.c_int64, ctypes.c_int32, ctypes.c_int32,
+                                                ctypes.POINTER(ctypes.c_size_t)]
+        L.hf_recolor_workspace_size.restype = ctypes.c_int
+        L.hf_recolor_fit.argtypes = [ctypes.c_int, ctypes.c_int64, ctypes.c_int32, ctypes.c_int32,
+                                     _p, _p, _p, ctypes.c_float, _p, _p, _f32p, _i32p, _p,
+                                     ctypes.c_size_t, _p]
+        L.hf_recolor_fit.restype = ctypes.c_int
         L.hf_status_string.argtypes = [ctypes.c_int]
         L.hf_status_string.restype = ctypes.c_char_p
         L.hf_last_error.argtypes = []
@@ -276,6 +283,30 @@ def fold(dtype: str, W, b, B, G, W_final, b_final, stream=None) -> None:
     rank = int(B.shape[-1])
     _check(lib().hf_fold(DTYPES[dtype], n_maps, d_R, K, rank, _dptr(W), _dptr(b), _dptr(B),
                          _dptr(G), _dptr(W_final), _dptr(b_final), _stream(stream)), "hf_fold")
+
+
+def recolor_workspace_size(N: int, d_S: int, d_R: int) -> int:
+    n = ctypes.c_size_t(0)
+    _check(lib().hf_recolor_workspace_size(int(N), int(d_S), int(d_R), ctypes.byref(n)),
+           "hf_recolor_workspace_size")
+    return int(n.value)
+
+
+def recolor_fit(dtype: str, X, Y, w, W_out, b_out, workspace, reg: float = 0.0,
+                stream=None, return_iters: bool = False):
+    """hf_recolor_fit (Eq. 3-5): X [N, d_S], Y [N, d_R], w [N] device tensors;
+    writes W_out [d_R, d_S] (= A^T) and b_out [d_R]; returns r (and the three
+    iteration counts with return_iters)."""
+    N, d_S = (int(x) for x in X.shape)
+    d_R = int(Y.shape[1])
+    r = ctypes.c_float(0.0)
+    its = (ctypes.c_int32 * 3)()
+    nbytes = int(workspace.numel() * workspace.element_size())
+    _check(lib().hf_recolor_fit(DTYPES[dtype], N, d_S, d_R, _dptr(X), _dptr(Y), _dptr(w),
+                                float(reg), _dptr(W_out), _dptr(b_out), ctypes.byref(r),
+                                its, _dptr(workspace), nbytes, _stream(stream)),
+           "hf_recolor_fit")
+    return (float(r.value), list(its)) if return_iters else float(r.value)
 
 
 def transfer_noalloc(desc: Desc, sender_kv, receiver_kv, stream=None) -> None:

@@ -24,7 +24,7 @@ LIB_NAME = "libheterofold.so"
 LIB_PATH = os.path.join(PKG_DIR, LIB_NAME)
 
 SOURCES = ["hf_align.cu", "hf_plan.cu", "hf_transfer.cu", "hf_noalloc.cu", "hf_host.cu",
-           "hf_batch.cu", "hf_fold.cu"]
+           "hf_batch.cu", "hf_fold.cu", "hf_recolor.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",
          "--expt-relaxed-constexpr"]

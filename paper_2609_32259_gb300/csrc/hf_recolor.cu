@@ -1,0 +1,471 @@
+// hf_recolor_fit: the Recolor initialisation of one map (Section 3.2,
+// Eq. 3-5) on the GPU, from weighted aligned sample pairs (X, Y, w):
+//   r = sqrt(sum w |x|^2 / (d_S sum w))                               (Eq. 3)
+//   Z = X / r; weighted means and covariances of Z and Y
+//   R* = polar factor of Sigma_Z^{-1/2} Sigma_ZY Sigma_Y^{-1/2}      (Eq. 4)
+//   A = Sigma_Z^{-1/2} R* Sigma_Y^{1/2},  b = mu_Y - mu_Z A           (Eq. 5)
+// Matrix square roots and the polar factor use Newton-Schulz iterations, so
+// every step is a matrix product or an elementwise pass: the coupled
+// iteration T = (3I - Z Y) / 2, Y <- Y T, Z <- T Z turns Y_0 = S / c,
+// Z_0 = I into (S / c)^{1/2} and (S / c)^{-1/2}; X <- X (3I - X^T X) / 2
+// turns X_0 = M / |M|_F into the orthogonal polar factor U Q^T of
+// M = U Lambda Q^T (full column rank), which is the R* of Eq. 4.
+// Offline (once per map, before folding); fp32 products on the CUDA cores.
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <string>
+#include <utility>
+
+#include <cuda_bf16.h>
+
+#include "hf_internal.h"
+
+namespace hf {
+namespace {
+
+constexpr int kTM = 128, kTN = 128, kTK = 8;  // SGEMM block tile
+constexpr int kGemmThreads = 256;             // 16 x 16 threads, 8 x 8 outputs each
+
+// C[M x N] = alpha * op(A) op(B) + beta * C, row-major C with leading
+// dimension ldc; op(A)(i, k) = A[i * a_i + k * a_k], op(B)(k, j) =
+// B[k * b_k + j * b_j] (strides express transposes).  Tiles of 128 x 128
+// with 8-deep k steps in shared memory; bounds-checked for any size.
+__global__ void __launch_bounds__(kGemmThreads) sgemm_kernel(
+    int M, int N, int K, float alpha, const float* __restrict__ A, int64_t a_i, int64_t a_k,
+    const float* __restrict__ B, int64_t b_k, int64_t b_j, float beta, float* C, int64_t ldc) {
+  __shared__ float As[kTK][kTM];
+  __shared__ float Bs[kTK][kTN];
+  const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;
+  const int i0 = blockIdx.y * kTM, j0 = blockIdx.x * kTN;
+  float acc[8][8];
+#pragma unroll
+  for (int a = 0; a < 8; ++a)
+#pragma unroll
+    for (int b = 0; b < 8; ++b) acc[a][b] = 0.f;
+  // loaders: the 1024 elements of each tile, 4 per thread; the tile index
+  // runs fastest along the operand's contiguous dimension
+  const bool a_kfast = a_k == 1, b_jfast = b_j == 1;
+  for (int k0 = 0; k0 < K; k0 += kTK) {
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int idx = threadIdx.x + e * kGemmThreads;
+      int ii, kk;
+      if (a_kfast) { ii = idx / kTK; kk = idx % kTK; } else { kk = idx / kTM; ii = idx % kTM; }
+      const int gi = i0 + ii, gk = k0 + kk;
+      As[kk][ii] = (gi < M && gk < K) ? A[gi * a_i + gk * a_k] : 0.f;
+      int jj, kb;
+      if (b_jfast) { kb = idx / kTN; jj = idx % kTN; } else { jj = idx / kTK; kb = idx % kTK; }
+      const int gj = j0 + jj, gk2 = k0 + kb;
+      Bs[kb][jj] = (gj < N && gk2 < K) ? B[gk2 * b_k + gj * b_j] : 0.f;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < kTK; ++kk) {
+      float a[8], b[8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        a[q] = As[kk][ty * 8 + q];
+        b[q] = Bs[kk][tx * 8 + q];
+      }
+#pragma unroll
+      for (int p = 0; p < 8; ++p)
+#pragma unroll
+        for (int q = 0; q < 8; ++q) acc[p][q] = fmaf(a[p], b[q], acc[p][q]);
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int p = 0; p < 8; ++p) {
+    const int gi = i0 + ty * 8 + p;
+    if (gi >= M) continue;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      const int gj = j0 + tx * 8 + q;
+      if (gj >= N) continue;
+      float* c = C + gi * ldc + gj;
+      *c = beta == 0.f ? alpha * acc[p][q] : fmaf(alpha, acc[p][q], beta * *c);
+    }
+  }
+}
+
+hf_status sgemm(cudaStream_t s, int M, int N, int K, float alpha, const float* A, int64_t a_i,
+                int64_t a_k, const float* B, int64_t b_k, int64_t b_j, float beta, float* C,
+                int64_t ldc) {
+  dim3 grid((N + kTN - 1) / kTN, (M + kTM - 1) / kTM);
+  sgemm_kernel<<<grid, kGemmThreads, 0, s>>>(M, N, K, alpha, A, a_i, a_k, B, b_k, b_j, beta, C,
+                                             ldc);
+  HF_CUDA_TRY(cudaGetLastError(), "hf_recolor_fit: product launch");
+  return HF_OK;
+}
+
+__device__ __forceinline__ float ld(const __nv_bfloat16* p) { return __bfloat162float(*p); }
+__device__ __forceinline__ float ld(const float* p) { return *p; }
+
+// Column sums of w X and w Y, sum w, and sum w |x|^2 (fp64 accumulation).
+template <typename T>
+__global__ void rc_stats_kernel(const T* X, const T* Y, const float* w, int64_t N, int dx,
+                                int dy, double* sx, double* sy, double* sw_ss) {
+  const int d = dx + dy;
+  const int col = blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t rows = (N + gridDim.y - 1) / gridDim.y;
+  const int64_t n0 = blockIdx.y * rows, n1 = min(N, n0 + rows);
+  double s = 0.0, ssq = 0.0, swt = 0.0;
+  if (col < d) {
+    for (int64_t n = n0; n < n1; ++n) {
+      const double wn = w[n];
+      const double v = col < dx ? ld(X + n * dx + col) : ld(Y + n * dy + (col - dx));
+      s += wn * v;
+      if (col < dx) ssq += wn * v * v;
+      if (col == 0) swt += wn;
+    }
+    atomicAdd(col < dx ? sx + col : sy + (col - dx), s);
+    if (col < dx) atomicAdd(sw_ss + 1, ssq);
+    if (col == 0) atomicAdd(sw_ss, swt);
+  }
+}
+
+// fp32 means mu_x (of X, not yet divided by r), mu_y, and [1 / W, 1 / r].
+__global__ void rc_mean_kernel(const double* sx, const double* sy, const double* sw_ss, int dx,
+                               int dy, float* mu, float* scal) {
+  const double W = sw_ss[0];
+  for (int c = blockIdx.x * blockDim.x + threadIdx.x; c < dx + dy; c += gridDim.x * blockDim.x)
+    mu[c] = static_cast<float>((c < dx ? sx[c] : sy[c - dx]) / W);
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    scal[0] = static_cast<float>(1.0 / W);
+    scal[1] = static_cast<float>(1.0 / sqrt(sw_ss[1] / (static_cast<double>(dx) * W)));
+  }
+}
+
+// Xc = sqrt(w / W) (x - mu_x) / r and Yc = sqrt(w / W) (y - mu_y), fp32.
+template <typename T>
+__global__ void rc_center_kernel(const T* X, const T* Y, const float* w, int64_t N, int dx,
+                                 int dy, const float* mu, const float* scal, float* Xc,
+                                 float* Yc) {
+  const int d = dx + dy;
+  const float inv_w = scal[0], inv_r = scal[1];
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < N * d;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t n = i / d;
+    const int c = static_cast<int>(i - n * d);
+    const float sc = sqrtf(w[n] * inv_w);
+    if (c < dx)
+      Xc[n * dx + c] = sc * (ld(X + n * dx + c) - mu[c]) * inv_r;
+    else
+      Yc[n * dy + (c - dx)] = sc * (ld(Y + n * dy + (c - dx)) - mu[c]);
+  }
+}
+
+// S += reg * trace(S) / d * I  (one block).
+__global__ void rc_ridge_kernel(float* S, int d, float reg) {
+  __shared__ float tr;
+  if (threadIdx.x == 0) {
+    double t = 0.0;
+    for (int i = 0; i < d; ++i) t += S[static_cast<int64_t>(i) * d + i];
+    tr = static_cast<float>(t / d);
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < d; i += blockDim.x) S[static_cast<int64_t>(i) * d + i] += reg * tr;
+}
+
+// out = a * in + b * I (square, or the leading square of a d x e matrix when
+// only scaling: b = 0).
+__global__ void rc_affine_kernel(float* out, const float* in, int64_t n_el, int cols, float a,
+                                 float b) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n_el;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t r = i / cols, c = i - r * cols;
+    out[i] = a * (in ? in[i] : 0.f) + (r == c ? b : 0.f);
+  }
+}
+
+// sum of squares (fp64) of x, or of (x - I) when minus_identity.
+__global__ void rc_sumsq_kernel(const float* x, int64_t n_el, int cols, int minus_identity,
+                                double* out) {
+  double s = 0.0;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n_el;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t r = i / cols, c = i - r * cols;
+    const double v = x[i] - (minus_identity && r == c ? 1.0 : 0.0);
+    s += v * v;
+  }
+  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+  if ((threadIdx.x & 31) == 0) atomicAdd(out, s);
+}
+
+// b = mu_y - mu_z A;  W_out = A^T in the output type.
+template <typename T>
+__global__ void rc_output_kernel(const float* A, int dx, int dy, const double* sx,
+                                 const double* sy, const double* sw_ss, T* W_out, float* b_out) {
+  const double W = sw_ss[0];
+  const double r = sqrt(sw_ss[1] / (static_cast<double>(dx) * W));
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < (int64_t)dx * dy;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t j = i / dx, k = i - j * dx;  // W_out[j][k] = A[k][j]
+    W_out[i] = T(A[k * dy + j]);
+  }
+  for (int j = blockIdx.x * blockDim.x + threadIdx.x; j < dy; j += gridDim.x * blockDim.x) {
+    double s = sy[j] / W;
+    for (int k = 0; k < dx; ++k) s -= (sx[k] / W / r) * A[static_cast<int64_t>(k) * dy + j];
+    b_out[j] = static_cast<float>(s);
+  }
+}
+
+struct Rc {
+  size_t stats, mu, xc, yc, sz, sy, szy, p1, p2, p3, p4, sz_ih, sy_ih, sy_h, m, x1, x2, xtx, a,
+      total;
+};
+
+Rc rc_layout(int64_t N, int dx, int dy) {
+  Rc L{};
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = off;
+    off = (off + bytes + 255) / 256 * 256;
+    return at;
+  };
+  const size_t f = sizeof(float);
+  const size_t dmax = static_cast<size_t>(dx > dy ? dx : dy);
+  L.stats = take(sizeof(double) * (dx + dy + 4));
+  L.mu = take(f * (dx + dy + 2));
+  L.xc = take(f * N * dx);
+  L.yc = take(f * N * dy);
+  L.sz = take(f * dx * dx);
+  L.sy = take(f * dy * dy);
+  L.szy = take(f * dx * dy);
+  L.p1 = take(f * dmax * dmax);
+  L.p2 = take(f * dmax * dmax);
+  L.p3 = take(f * dmax * dmax);
+  L.p4 = take(f * dmax * dmax);
+  L.sz_ih = take(f * dx * dx);
+  L.sy_ih = take(f * dy * dy);
+  L.sy_h = take(f * dy * dy);
+  L.m = take(f * dx * dy);
+  L.x1 = take(f * dx * dy);
+  L.x2 = take(f * dx * dy);
+  L.xtx = take(f * dy * dy);
+  L.a = take(f * dx * dy);
+  L.total = off;
+  return L;
+}
+
+hf_status read_double(cudaStream_t s, const double* d, double* h) {
+  HF_CUDA_TRY(cudaMemcpyAsync(h, d, sizeof(double), cudaMemcpyDeviceToHost, s), "read back");
+  HF_CUDA_TRY(cudaStreamSynchronize(s), "synchronize");
+  return HF_OK;
+}
+
+constexpr int kMaxIter = 80;
+constexpr double kTol = 2e-5;  // |X - I|_F / sqrt(d) at convergence
+
+// Convergence test of an iteration's residual e (checked every 4 steps):
+// below the tolerance, or no longer falling once small (the fp32 floor).
+bool converged(double e, double* prev) {
+  const bool done = e < kTol || (e < 1e-3 && e >= 0.5 * *prev);
+  *prev = e;
+  return done;
+}
+
+// Newton-Schulz square root and inverse square root of the SPD matrix S
+// (d x d): root = S^{1/2}, inv_root = S^{-1/2}.  Y, Z, T, U are d x d work.
+hf_status ns_sqrt(cudaStream_t s, const float* S, int d, float* Y, float* Z, float* T, float* U,
+                  float* root, float* inv_root, double* dscr, int* iters) {
+  const int64_t n_el = static_cast<int64_t>(d) * d;
+  const int grid = 1024;
+  double c2 = 0.0;
+  HF_CUDA_TRY(cudaMemsetAsync(dscr, 0, sizeof(double), s), "clear");
+  rc_sumsq_kernel<<<grid, 256, 0, s>>>(S, n_el, d, 0, dscr);
+  hf_status st = read_double(s, dscr, &c2);
+  if (st != HF_OK) return st;
+  const double c = sqrt(c2);
+  if (!(c > 0.0)) {
+    set_error("hf_recolor_fit: a covariance is zero");
+    return HF_ERR_INVALID_ARGUMENT;
+  }
+  rc_affine_kernel<<<grid, 256, 0, s>>>(Y, S, n_el, d, static_cast<float>(1.0 / c), 0.f);
+  rc_affine_kernel<<<grid, 256, 0, s>>>(Z, nullptr, n_el, d, 0.f, 1.f);
+  int it = 0;
+  double prev = 1e30;
+  for (; it < kMaxIter; ++it) {
+    // T = 1.5 I - 0.5 Z Y
+    rc_affine_kernel<<<grid, 256, 0, s>>>(T, nullptr, n_el, d, 0.f, 1.5f);
+    if ((st = sgemm(s, d, d, d, -0.5f, Z, d, 1, Y, d, 1, 1.f, T, d)) != HF_OK) return st;
+    if (it % 4 == 3) {
+      double e2 = 0.0;
+      HF_CUDA_TRY(cudaMemsetAsync(dscr, 0, sizeof(double), s), "clear");
+      // |I - Z Y| = 2 |T - I|
+      rc_sumsq_kernel<<<grid, 256, 0, s>>>(T, n_el, d, 1, dscr);
+      if ((st = read_double(s, dscr, &e2)) != HF_OK) return st;
+      if (converged(2.0 * sqrt(e2 / d), &prev)) break;
+    }
+    if ((st = sgemm(s, d, d, d, 1.f, Y, d, 1, T, d, 1, 0.f, U, d)) != HF_OK) return st;  // Y T
+    std::swap(Y, U);
+    if ((st = sgemm(s, d, d, d, 1.f, T, d, 1, Z, d, 1, 0.f, U, d)) != HF_OK) return st;  // T Z
+    std::swap(Z, U);
+  }
+  *iters = it;
+  rc_affine_kernel<<<grid, 256, 0, s>>>(root, Y, n_el, d, static_cast<float>(sqrt(c)), 0.f);
+  rc_affine_kernel<<<grid, 256, 0, s>>>(inv_root, Z, n_el, d, static_cast<float>(1.0 / sqrt(c)),
+                                        0.f);
+  HF_CUDA_TRY(cudaGetLastError(), "hf_recolor_fit: iteration launch");
+  return HF_OK;
+}
+
+// Orthogonal polar factor of M (dx x dy, dx >= dy, full column rank):
+// X <- X (3I - X^T X) / 2 from X_0 = M / |M|_F.  Result in *out (one of the
+// two buffers).
+hf_status ns_polar(cudaStream_t s, const float* M, int dx, int dy, float* X, float* X2,
+                   float* P, double* dscr, float** out, int* iters) {
+  const int64_t n_el = static_cast<int64_t>(dx) * dy, p_el = static_cast<int64_t>(dy) * dy;
+  const int grid = 1024;
+  double m2 = 0.0;
+  HF_CUDA_TRY(cudaMemsetAsync(dscr, 0, sizeof(double), s), "clear");
+  rc_sumsq_kernel<<<grid, 256, 0, s>>>(M, n_el, dy, 0, dscr);
+  hf_status st = read_double(s, dscr, &m2);
+  if (st != HF_OK) return st;
+  if (!(m2 > 0.0)) {
+    set_error("hf_recolor_fit: the cross-covariance is zero");
+    return HF_ERR_INVALID_ARGUMENT;
+  }
+  rc_affine_kernel<<<grid, 256, 0, s>>>(X, M, n_el, dy, static_cast<float>(1.0 / sqrt(m2)), 0.f);
+  int it = 0;
+  double prev = 1e30;
+  for (; it < kMaxIter; ++it) {
+    // P = X^T X
+    if ((st = sgemm(s, dy, dy, dx, 1.f, X, 1, dy, X, dy, 1, 0.f, P, dy)) != HF_OK) return st;
+    if (it % 4 == 3) {
+      double e2 = 0.0;
+      HF_CUDA_TRY(cudaMemsetAsync(dscr, 0, sizeof(double), s), "clear");
+      rc_sumsq_kernel<<<grid, 256, 0, s>>>(P, p_el, dy, 1, dscr);
+      if ((st = read_double(s, dscr, &e2)) != HF_OK) return st;
+      if (converged(sqrt(e2 / dy), &prev)) break;
+    }
+    // X2 = 1.5 X - 0.5 X P
+    rc_affine_kernel<<<grid, 256, 0, s>>>(X2, X, n_el, dy, 1.5f, 0.f);
+    if ((st = sgemm(s, dx, dy, dy, -0.5f, X, dy, 1, P, dy, 1, 1.f, X2, dy)) != HF_OK) return st;
+    std::swap(X, X2);
+  }
+  *iters = it;
+  *out = X;
+  HF_CUDA_TRY(cudaGetLastError(), "hf_recolor_fit: iteration launch");
+  return HF_OK;
+}
+
+template <typename T>
+hf_status recolor_typed(int64_t N, int dx, int dy, const void* Xv, const void* Yv, const float* w,
+                        float reg, void* W_out, float* b_out, float* h_r, int32_t* h_iters,
+                        char* ws, cudaStream_t s) {
+  const Rc L = rc_layout(N, dx, dy);
+  double* stats = reinterpret_cast<double*>(ws + L.stats);
+  double* sx = stats;
+  double* sy = sx + dx;
+  double* sw_ss = sy + dy;    // [0] sum w, [1] sum w |x|^2
+  double* dscr = sw_ss + 2;   // scratch scalar
+  auto F = [&](size_t off) { return reinterpret_cast<float*>(ws + off); };
+  const T* X = static_cast<const T*>(Xv);
+  const T* Y = static_cast<const T*>(Yv);
+  HF_CUDA_TRY(cudaMemsetAsync(stats, 0, sizeof(double) * (dx + dy + 4), s), "clear");
+  const int d = dx + dy;
+  dim3 sgrid((d + 255) / 256, static_cast<unsigned>(std::min<int64_t>(N, 256)));
+  rc_stats_kernel<T><<<sgrid, 256, 0, s>>>(X, Y, w, N, dx, dy, sx, sy, sw_ss);
+  float* mu = F(L.mu);
+  rc_mean_kernel<<<(d + 255) / 256, 256, 0, s>>>(sx, sy, sw_ss, dx, dy, mu, mu + d);
+  rc_center_kernel<T><<<2048, 256, 0, s>>>(X, Y, w, N, dx, dy, mu, mu + d, F(L.xc), F(L.yc));
+  HF_CUDA_TRY(cudaGetLastError(), "hf_recolor_fit: moments launch");
+  hf_status st;
+  // Sigma_Z = Xc^T Xc, Sigma_Y = Yc^T Yc, Sigma_ZY = Xc^T Yc
+  if ((st = sgemm(s, dx, dx, N, 1.f, F(L.xc), 1, dx, F(L.xc), dx, 1, 0.f, F(L.sz), dx)) != HF_OK)
+    return st;
+  if ((st = sgemm(s, dy, dy, N, 1.f, F(L.yc), 1, dy, F(L.yc), dy, 1, 0.f, F(L.sy), dy)) != HF_OK)
+    return st;
+  if ((st = sgemm(s, dx, dy, N, 1.f, F(L.xc), 1, dx, F(L.yc), dy, 1, 0.f, F(L.szy), dy)) != HF_OK)
+    return st;
+  if (reg > 0.f) {
+    rc_ridge_kernel<<<1, 256, 0, s>>>(F(L.sz), dx, reg);
+    rc_ridge_kernel<<<1, 256, 0, s>>>(F(L.sy), dy, reg);
+  }
+  int it1 = 0, it2 = 0, it3 = 0;
+  if ((st = ns_sqrt(s, F(L.sz), dx, F(L.p1), F(L.p2), F(L.p3), F(L.p4), F(L.p4) /*unused root*/,
+                    F(L.sz_ih), dscr, &it1)) != HF_OK)
+    return st;
+  if ((st = ns_sqrt(s, F(L.sy), dy, F(L.p1), F(L.p2), F(L.p3), F(L.p4), F(L.sy_h), F(L.sy_ih),
+                    dscr, &it2)) != HF_OK)
+    return st;
+  // M = Sigma_Z^{-1/2} Sigma_ZY Sigma_Y^{-1/2}
+  if ((st = sgemm(s, dx, dy, dx, 1.f, F(L.sz_ih), dx, 1, F(L.szy), dy, 1, 0.f, F(L.x2), dy)) != HF_OK)
+    return st;
+  if ((st = sgemm(s, dx, dy, dy, 1.f, F(L.x2), dy, 1, F(L.sy_ih), dy, 1, 0.f, F(L.m), dy)) != HF_OK)
+    return st;
+  float* R = nullptr;
+  if ((st = ns_polar(s, F(L.m), dx, dy, F(L.x1), F(L.x2), F(L.xtx), dscr, &R, &it3)) != HF_OK)
+    return st;
+  // A = Sigma_Z^{-1/2} R* Sigma_Y^{1/2}
+  float* tmp = R == F(L.x1) ? F(L.x2) : F(L.x1);
+  if ((st = sgemm(s, dx, dy, dx, 1.f, F(L.sz_ih), dx, 1, R, dy, 1, 0.f, tmp, dy)) != HF_OK) return st;
+  if ((st = sgemm(s, dx, dy, dy, 1.f, tmp, dy, 1, F(L.sy_h), dy, 1, 0.f, F(L.a), dy)) != HF_OK)
+    return st;
+  rc_output_kernel<T><<<1024, 256, 0, s>>>(F(L.a), dx, dy, sx, sy, sw_ss, static_cast<T*>(W_out),
+                                           b_out);
+  HF_CUDA_TRY(cudaGetLastError(), "hf_recolor_fit: output launch");
+  double h[2];
+  HF_CUDA_TRY(cudaMemcpyAsync(h, sw_ss, sizeof(h), cudaMemcpyDeviceToHost, s), "read back");
+  HF_CUDA_TRY(cudaStreamSynchronize(s), "synchronize");
+  if (h_r) *h_r = static_cast<float>(std::sqrt(h[1] / (static_cast<double>(dx) * h[0])));
+  if (h_iters) {
+    h_iters[0] = it1;
+    h_iters[1] = it2;
+    h_iters[2] = it3;
+  }
+  if (it1 >= kMaxIter || it2 >= kMaxIter || it3 >= kMaxIter) {
+    set_error("hf_recolor_fit: an iteration did not converge (ill-conditioned covariances: "
+              "raise reg)");
+    return HF_ERR_DEVICE_CHECK;
+  }
+  return HF_OK;
+}
+
+}  // namespace
+}  // namespace hf
+
+using namespace hf;
+
+extern "C" hf_status hf_recolor_workspace_size(int64_t N, int32_t d_S, int32_t d_R,
+                                               size_t* bytes) {
+  if (!bytes || N < 2 || d_S < 1 || d_R < 1 || d_S < d_R) {
+    set_error("hf_recolor_workspace_size: need N >= 2 and d_S >= d_R >= 1");
+    return HF_ERR_INVALID_ARGUMENT;
+  }
+  *bytes = rc_layout(N, d_S, d_R).total;
+  return HF_OK;
+}
+
+extern "C" hf_status hf_recolor_fit(hf_dtype dtype, int64_t N, int32_t d_S, int32_t d_R,
+                                    const void* d_X, const void* d_Y, const float* d_w, float reg,
+                                    void* d_W_out, float* d_b_out, float* h_r_out,
+                                    int32_t* h_iters_out, void* d_workspace,
+                                    size_t workspace_bytes, hf_stream_t stream_) {
+  if (dtype != HF_BF16 && dtype != HF_F32) {
+    set_error("hf_recolor_fit: unknown dtype");
+    return HF_ERR_INVALID_ARGUMENT;
+  }
+  if (N < 2 || d_S < 1 || d_R < 1 || d_S < d_R || N * static_cast<int64_t>(d_S) >= (1LL << 31)) {
+    set_error("hf_recolor_fit: need N >= 2, d_S >= d_R >= 1 and N x d_S < 2^31");
+    return HF_ERR_INVALID_ARGUMENT;
+  }
+  if (!d_X || !d_Y || !d_w || !d_W_out || !d_b_out || !(reg >= 0.f)) {
+    set_error("hf_recolor_fit: null pointer or negative reg");
+    return HF_ERR_INVALID_ARGUMENT;
+  }
+  if (!d_workspace || workspace_bytes < rc_layout(N, d_S, d_R).total ||
+      (reinterpret_cast<uintptr_t>(d_workspace) & 255u)) {
+    set_error("hf_recolor_fit: workspace missing, too small or not 256-byte aligned");
+    return HF_ERR_WORKSPACE;
+  }
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream_);
+  char* ws = static_cast<char*>(d_workspace);
+  if (dtype == HF_BF16)
+    return recolor_typed<__nv_bfloat16>(N, d_S, d_R, d_X, d_Y, d_w, reg, d_W_out, d_b_out,
+                                        h_r_out, h_iters_out, ws, s);
+  return recolor_typed<float>(N, d_S, d_R, d_X, d_Y, d_w, reg, d_W_out, d_b_out, h_r_out,
+                              h_iters_out, ws, s);
+}
