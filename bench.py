@@ -360,13 +360,19 @@ def run_ours(args):
         e2e_mean = statistics.mean(per_step)
         e2e_ms = statistics.median(per_step)
         e2e_value, (e2e_ms, e2e_mean) = aggregate([e2e_ms, e2e_mean], tok.T_r, world)
-        h2d = (sender.numel() * sender.element_size() + h_s_end.numel() * 4 +
-               h_r_end.numel() * 4)
+        # hf_transfer_host reads only the referenced sender rows when every
+        # alignment row is one sender token (here: Token Alignment, Eq. 1)
+        one_token_rows = (w.align_mode in ("ta", "same_index") and w.layer_mode == "paper3"
+                          and not w.sender_k_rotated)
+        sender_bytes = (w.L_s * 2 * U * w.d_s * sender.element_size() if one_token_rows
+                        else sender.numel() * sender.element_size())
+        h2d = sender_bytes + h_s_end.numel() * 4 + h_r_end.numel() * 4
         d2h = job.receiver.numel() * job.receiver.element_size()
         e2e = {"value": e2e_value, "unit": UNIT, "ms_per_step": e2e_ms,
                "ms_per_step_mean": e2e_mean, "steps": n_e2e, "statistic": "median step",
                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
-               "api": "hf_align_build + hf_plan_create + hf_transfer_host (pinned host caches)"}
+               "api": "hf_align_build + hf_plan_create + hf_transfer_host (pinned host caches)",
+               "sender_read": "referenced rows only" if one_token_rows else "whole layers"}
         del h_sender, h_recv
 
     hbm_gbs, tflops, tflops_sust, src = peaks()

@@ -267,8 +267,12 @@ hf_status hf_transfer(hf_plan plan, const void* sender_kv, void* receiver_kv,
  *                (cudaHostAlloc or cudaHostRegister), the layout hf_transfer
  *                takes.
  * d_sender_kv:   device buffer of the same size: the sender layers are
- *                copied there (only layers 0 .. the highest one the layer
- *                table reads).
+ *                brought there (only layers 0 .. the highest one the layer
+ *                table reads).  When every alignment row is one sender
+ *                token (Token Alignment, same-index, no rotated keys), only
+ *                the referenced rows are read, by a gather kernel through
+ *                the mapped host memory; other rows of d_sender_kv are left
+ *                as they were.  Otherwise whole layers are copied.
  * d_receiver_kv: device receiver cache, as for hf_transfer.
  * h_receiver_kv: page-locked host buffer of the receiver cache's size
  *                (contiguous or paged layout); every receiver layer is

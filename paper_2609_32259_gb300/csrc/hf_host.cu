@@ -1,9 +1,12 @@
 // hf_transfer_host: one transfer whose sender and receiver caches live in
 // page-locked host memory.  The receiver layers are split into groups; the
-// sender layers a group reads are copied in (one copy engine), the group's
-// layers are computed on the caller's stream, and the finished receiver
-// layers are copied out (the other copy engine) while later groups are still
-// being copied in and computed.
+// sender layers a group reads are brought in, the group's layers are
+// computed on the caller's stream, and the finished receiver layers are
+// copied out (a copy engine) while later groups are still being brought in
+// and computed.  When every alignment row is one sender token (Token
+// Alignment, same-index) only the referenced sender rows are read: a small
+// gather kernel reads them from the mapped host memory (about a quarter of
+// the sender cache for Token Alignment); otherwise whole layers are copied.
 #include <algorithm>
 #include <cstring>
 #include <string>
@@ -13,7 +16,7 @@
 namespace hf {
 namespace {
 
-hf_status require_pinned(const void* ptr, const char* what) {
+hf_status require_pinned(const void* ptr, const char* what, const void** dev_alias = nullptr) {
   cudaPointerAttributes a;
   std::memset(&a, 0, sizeof(a));
   const cudaError_t e = cudaPointerGetAttributes(&a, ptr);
@@ -22,7 +25,32 @@ hf_status require_pinned(const void* ptr, const char* what) {
     set_error(std::string("hf_transfer_host: ") + what + " is not page-locked host memory");
     return HF_ERR_INVALID_ARGUMENT;
   }
+  if (dev_alias) *dev_alias = a.devicePointer;
   return HF_OK;
+}
+
+// Copies the referenced sender rows (ucol[0 .. U), U read on the device) of
+// sender layers [t0, t1), both roles, from mapped host memory into the same
+// rows of the device sender cache: 16 bytes per thread, one row's chunks on
+// consecutive threads.  Few registers and no shared memory, so its blocks
+// fit beside the transfer kernel's.
+__global__ void __launch_bounds__(256) gather_sender_rows(const uint4* __restrict__ src,
+                                                          uint4* __restrict__ dst,
+                                                          const int32_t* __restrict__ ucol,
+                                                          const int32_t* __restrict__ n_distinct,
+                                                          int t0, int t1, int64_t s_rows,
+                                                          int chunks) {
+  const int64_t U = *n_distinct;
+  const int64_t total = static_cast<int64_t>(t1 - t0) * 2 * U * chunks;
+  for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t rest = i / chunks;
+    const int64_t ch = i - rest * chunks;
+    const int64_t lcs = rest / U;             // (t - t0) * 2 + c
+    const int64_t u = rest - lcs * U;
+    const int64_t row = (2 * static_cast<int64_t>(t0) + lcs) * s_rows + ucol[u];
+    dst[row * chunks + ch] = src[row * chunks + ch];
+  }
 }
 
 // The plan's two copy streams (created on first use, on the current device)
@@ -84,8 +112,14 @@ extern "C" hf_status hf_transfer_host(hf_plan plan, const void* h_sender_kv, voi
     set_error("hf_transfer_host: device caches and maps must be 16-byte aligned");
     return HF_ERR_INVALID_ARGUMENT;
   }
-  hf_status s = require_pinned(h_sender_kv, "h_sender_kv");
+  const void* h_sender_dev = nullptr;  // the sender cache as the device addresses it
+  hf_status s = require_pinned(h_sender_kv, "h_sender_kv", &h_sender_dev);
   if (s != HF_OK) return s;
+  const size_t row_bytes = static_cast<size_t>(plan->d_s) * (d.dtype == HF_BF16 ? 2 : 4);
+  const bool gather = plan->gather && h_sender_dev != nullptr && row_bytes % 16 == 0 &&
+                      (reinterpret_cast<uintptr_t>(h_sender_dev) & 15u) == 0;
+  const int32_t* ucol = reinterpret_cast<const int32_t*>(plan->ws + plan->lay.ucol);
+  const int32_t* n_distinct = reinterpret_cast<const int32_t*>(plan->ws + plan->lay.n_distinct);
   s = require_pinned(h_receiver_kv, "h_receiver_kv");
   if (s != HF_OK) return s;
   // default: one group per receiver layer (the copy out of a layer starts as
@@ -117,10 +151,17 @@ extern "C" hf_status hf_transfer_host(hf_plan plan, const void* h_sender_kv, voi
     int need = 0;
     for (int l = l0; l < l1; ++l) need = std::max(need, plan->max_sender_layer[l] + 1);
     if (need > copied) {
-      HF_CUDA_TRY(cudaMemcpyAsync(ds + copied * sender_layer, hs + copied * sender_layer,
-                                  (need - copied) * sender_layer, cudaMemcpyHostToDevice,
-                                  plan->s_h2d),
-                  "hf_transfer_host: sender copy");
+      if (gather) {
+        gather_sender_rows<<<2 * device_sm_count(), 256, 0, plan->s_h2d>>>(
+            static_cast<const uint4*>(h_sender_dev), reinterpret_cast<uint4*>(ds), ucol,
+            n_distinct, copied, need, plan->s_rows, static_cast<int>(row_bytes / 16));
+        HF_CUDA_TRY(cudaGetLastError(), "hf_transfer_host: sender gather");
+      } else {
+        HF_CUDA_TRY(cudaMemcpyAsync(ds + copied * sender_layer, hs + copied * sender_layer,
+                                    (need - copied) * sender_layer, cudaMemcpyHostToDevice,
+                                    plan->s_h2d),
+                    "hf_transfer_host: sender copy");
+      }
       copied = need;
     }
     cudaEvent_t ev_in = ev[2 + 2 * g], ev_out = ev[3 + 2 * g];
