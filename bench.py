@@ -360,6 +360,21 @@ def run_ours(args):
         e2e_mean = statistics.mean(per_step)
         e2e_ms = statistics.median(per_step)
         e2e_value, (e2e_ms, e2e_mean) = aggregate([e2e_ms, e2e_mean], tok.T_r, world)
+        # the same steps with the receiver cache left in device memory (the
+        # receiver model reads it there); the status word is read back
+        for it in range(n_e2e + 1):
+            if it >= 1:
+                marks[it - 1].record(stream)
+            job.s_end.copy_(h_s_end, non_blocking=True)
+            job.r_end.copy_(h_r_end, non_blocking=True)
+            job.align(stream)
+            job.make_plan(stream)
+            job.transfer_host(h_sender, None, args.e2e_groups, stream)
+            job.device_status(stream)
+        marks[n_e2e].record(stream)
+        torch.cuda.synchronize()
+        resident_ms = statistics.median(marks[i].elapsed_time(marks[i + 1]) for i in range(n_e2e))
+        _, (resident_ms,) = aggregate([resident_ms], tok.T_r, world)
         # hf_transfer_host reads only the referenced sender rows when every
         # alignment row is one sender token (here: Token Alignment, Eq. 1)
         one_token_rows = (w.align_mode in ("ta", "same_index") and w.layer_mode == "paper3"
@@ -372,7 +387,10 @@ def run_ours(args):
                "ms_per_step_mean": e2e_mean, "steps": n_e2e, "statistic": "median step",
                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
                "api": "hf_align_build + hf_plan_create + hf_transfer_host (pinned host caches)",
-               "sender_read": "referenced rows only" if one_token_rows else "whole layers"}
+               "sender_read": "referenced rows only" if one_token_rows else "whole layers",
+               "receiver_in_device_memory": {
+                   "value": tok.T_r * world / (resident_ms * 1e-3), "ms_per_step": resident_ms,
+                   "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": 4}}
         del h_sender, h_recv
 
     hbm_gbs, tflops, tflops_sust, src = peaks()

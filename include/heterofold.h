@@ -277,6 +277,9 @@ hf_status hf_transfer(hf_plan plan, const void* sender_kv, void* receiver_kv,
  * h_receiver_kv: page-locked host buffer of the receiver cache's size
  *                (contiguous or paged layout); every receiver layer is
  *                copied back whole (a paged pool's untouched blocks too).
+ *                NULL: nothing is copied back (the receiver model reads its
+ *                cache in device memory; only the sender comes from the
+ *                host).
  * n_groups:      receiver layers are processed in n_groups consecutive
  *                groups (1 .. L_r; 0 = L_r, one per layer): group g's sender
  *                layers are copied in, its layers computed on `stream`,

@@ -261,7 +261,8 @@ def transfer(plan: Plan, sender_kv, receiver_kv, stream=None) -> None:
 def transfer_host(plan: Plan, h_sender_kv, d_sender_kv, d_receiver_kv, h_receiver_kv,
                   n_groups: int = 0, stream=None) -> None:
     """hf_transfer_host: caches in page-locked host memory (torch tensors made
-    with pin_memory=True), copies overlapped with the computation."""
+    with pin_memory=True), copies overlapped with the computation;
+    h_receiver_kv None keeps the receiver cache on the device."""
     _check(lib().hf_transfer_host(plan.handle, _dptr(h_sender_kv), _dptr(d_sender_kv),
                                   _dptr(d_receiver_kv), _dptr(h_receiver_kv), int(n_groups),
                                   _stream(stream)), "hf_transfer_host")

@@ -103,7 +103,7 @@ extern "C" hf_status hf_transfer_host(hf_plan plan, const void* h_sender_kv, voi
     return HF_ERR_INVALID_ARGUMENT;
   }
   if (plan->T_r == 0) return HF_OK;
-  if (!h_sender_kv || !d_sender_kv || !d_receiver_kv || !h_receiver_kv) {
+  if (!h_sender_kv || !d_sender_kv || !d_receiver_kv) {
     set_error("hf_transfer_host: null cache pointer");
     return HF_ERR_INVALID_ARGUMENT;
   }
@@ -120,8 +120,8 @@ extern "C" hf_status hf_transfer_host(hf_plan plan, const void* h_sender_kv, voi
                       (reinterpret_cast<uintptr_t>(h_sender_dev) & 15u) == 0;
   const int32_t* ucol = reinterpret_cast<const int32_t*>(plan->ws + plan->lay.ucol);
   const int32_t* n_distinct = reinterpret_cast<const int32_t*>(plan->ws + plan->lay.n_distinct);
-  s = require_pinned(h_receiver_kv, "h_receiver_kv");
-  if (s != HF_OK) return s;
+  const bool copy_out = h_receiver_kv != nullptr;  // NULL: the cache stays on the device
+  if (copy_out && (s = require_pinned(h_receiver_kv, "h_receiver_kv")) != HF_OK) return s;
   // default: one group per receiver layer (the copy out of a layer starts as
   // soon as it is computed; measured best on a 40-layer, 32K-token transfer)
   const int G = n_groups == 0 ? d.L_r : n_groups;
@@ -169,11 +169,13 @@ extern "C" hf_status hf_transfer_host(hf_plan plan, const void* h_sender_kv, voi
     HF_CUDA_TRY(cudaStreamWaitEvent(stream, ev_in, 0), "hf_transfer_host: wait");
     s = launch_transfer(plan, d_sender_kv, d_receiver_kv, stream, l0, l1);
     if (s != HF_OK) return s;
-    HF_CUDA_TRY(cudaEventRecord(ev_out, stream), "hf_transfer_host: record");
-    HF_CUDA_TRY(cudaStreamWaitEvent(plan->s_d2h, ev_out, 0), "hf_transfer_host: wait");
-    HF_CUDA_TRY(cudaMemcpyAsync(hr + l0 * recv_layer, dr + l0 * recv_layer, (l1 - l0) * recv_layer,
-                                cudaMemcpyDeviceToHost, plan->s_d2h),
-                "hf_transfer_host: receiver copy");
+    if (copy_out) {
+      HF_CUDA_TRY(cudaEventRecord(ev_out, stream), "hf_transfer_host: record");
+      HF_CUDA_TRY(cudaStreamWaitEvent(plan->s_d2h, ev_out, 0), "hf_transfer_host: wait");
+      HF_CUDA_TRY(cudaMemcpyAsync(hr + l0 * recv_layer, dr + l0 * recv_layer,
+                                  (l1 - l0) * recv_layer, cudaMemcpyDeviceToHost, plan->s_d2h),
+                  "hf_transfer_host: receiver copy");
+    }
   }
   // `stream` is ordered after the last copy out
   HF_CUDA_TRY(cudaEventRecord(ev_done, plan->s_d2h), "hf_transfer_host: record");

@@ -52,6 +52,18 @@ def test_transfer_host_matches_device_path(name):
         assert torch.equal(h_recv, ref), (name, G)
 
 
+def test_transfer_host_can_leave_the_receiver_on_the_device():
+    c = Case(W.llama_to_ministral(800).with_(L_s=5, L_r=6), sentinel=SENTINEL).run()
+    ref = c.job.receiver.clone()
+    h_sender = torch.empty(c.sender.shape, dtype=c.sender.dtype, pin_memory=True)
+    h_sender.copy_(c.sender)
+    c.sender.zero_()
+    c.job.receiver.fill_(SENTINEL)
+    c.job.transfer_host(h_sender, None, 3)
+    torch.cuda.synchronize()
+    assert torch.equal(c.job.receiver, ref)
+
+
 def test_transfer_host_rejects_pageable_memory_and_bad_groups():
     c = Case(W.llama_to_ministral(300).with_(L_s=3, L_r=2)).run()
     pageable = torch.empty(c.sender.shape, dtype=c.sender.dtype)
