@@ -32,9 +32,8 @@ hf_status require_pinned(const void* ptr, const char* what, const void** dev_ali
 // Copies the referenced sender rows (ucol[0 .. U), U read on the device) of
 // sender layers [t0, t1), both roles, from mapped host memory into the same
 // rows of the device sender cache: 16 bytes per thread, one row's chunks on
-// consecutive threads.  Few registers and no shared memory, so its blocks
-// fit beside the transfer kernel's.
-__global__ void __launch_bounds__(256) gather_sender_rows(const uint4* __restrict__ src,
+// consecutive threads.
+__global__ void __launch_bounds__(128) gather_sender_rows(const uint4* __restrict__ src,
                                                           uint4* __restrict__ dst,
                                                           const int32_t* __restrict__ ucol,
                                                           const int32_t* __restrict__ n_distinct,
@@ -152,7 +151,9 @@ extern "C" hf_status hf_transfer_host(hf_plan plan, const void* h_sender_kv, voi
     for (int l = l0; l < l1; ++l) need = std::max(need, plan->max_sender_layer[l] + 1);
     if (need > copied) {
       if (gather) {
-        gather_sender_rows<<<2 * device_sm_count(), 256, 0, plan->s_h2d>>>(
+        // 128-thread blocks at 32 registers fit in the register file beside a
+        // transfer kernel CTA (448 x 128 registers), so the gather overlaps it
+        gather_sender_rows<<<4 * device_sm_count(), 128, 0, plan->s_h2d>>>(
             static_cast<const uint4*>(h_sender_dev), reinterpret_cast<uint4*>(ds), ucol,
             n_distinct, copied, need, plan->s_rows, static_cast<int>(row_bytes / 16));
         HF_CUDA_TRY(cudaGetLastError(), "hf_transfer_host: sender gather");
