@@ -297,12 +297,14 @@ hf_status hf_transfer_host(hf_plan plan, const void* h_sender_kv, void* d_sender
  * hf_transfer_batch — several transfer directions in one call (a
  * multi-agent round sends each message to receivers of other model
  * families; Appendix "HiddenBench Evaluation").  Direction i is
- * hf_transfer(plans[i], sender_kv[i], receiver_kv[i]); the kernels run on
- * streams of a per-device pool forked from `stream`, so each direction's
- * CTA pairs start as the previous one's retire, and `stream` is ordered
- * after all of them.  n in [0, 16]; a plan appears at most once; the
- * receiver caches must not overlap.  Asynchronous; the pool's streams are
- * created on the first call on a device.
+ * hf_transfer(plans[i], sender_kv[i], receiver_kv[i]).  When all plans
+ * share the dtype and the operand path (one-entry alignment rows with
+ * one-layer segments, or not), the directions run in one launch of the
+ * transfer kernel over all their tiles; otherwise each direction's kernel
+ * runs on a stream of a per-device pool forked from `stream` (created on
+ * the first such call on a device).  `stream` is ordered after all of them.
+ * n in [0, 16]; a plan appears at most once; the receiver caches must not
+ * overlap.  Asynchronous.
  */
 hf_status hf_transfer_batch(const hf_plan* plans, const void* const* sender_kv,
                             void* const* receiver_kv, int32_t n, hf_stream_t stream);

@@ -1,10 +1,11 @@
 // hf_transfer_batch: several transfer directions (each its own plan: model
-// pair, maps, alignment, caches) in one call.  Each direction's kernel goes
-// to its own stream of a per-device pool, forked from and joined back into
-// the caller's stream, so the persistent kernels follow one another on the
-// SMs without a host round trip: a direction's CTA pairs start as soon as
-// the previous direction's pairs retire, which fills the tail of every
-// launch (short message transfers are a few waves each).
+// pair, maps, alignment, caches) in one call.  Directions that share the
+// dtype and the operand path run in ONE launch of the persistent kernel:
+// its tiles are the concatenation of the directions' tiles and every role
+// reads its tile's direction parameters, so short transfers (a few waves
+// each) fill one another's tails.  Otherwise each direction's kernel goes to
+// its own stream of a per-device pool, forked from and joined back into the
+// caller's stream.
 #include <mutex>
 #include <string>
 
@@ -82,6 +83,8 @@ extern "C" hf_status hf_transfer_batch(const hf_plan* plans, const void* const* 
   if (n == 0) return HF_OK;
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
   if (n == 1) return launch_transfer(plans[0], sender_kv[0], receiver_kv[0], stream);
+  if (batch_compatible(plans, n))
+    return launch_transfer_batch(plans, sender_kv, receiver_kv, n, stream);
   StreamPool* pool = nullptr;
   hf_status s = get_pool(&pool);
   if (s != HF_OK) return s;

@@ -105,6 +105,11 @@ hf_status plan_build(const hf_plan_desc* desc, void* d_workspace, size_t workspa
 // One transfer-kernel launch over receiver layers [l_begin, l_end) (l_end < 0: all).
 hf_status launch_transfer(hf_plan_s* p, const void* sender, void* receiver, cudaStream_t stream,
                           int l_begin = 0, int l_end = -1);
+// Several plans in one launch: they must share the dtype and the operand
+// path (batch_compatible); n <= kMaxBatch.
+bool batch_compatible(const hf_plan_s* const* plans, int n);
+hf_status launch_transfer_batch(hf_plan_s* const* plans, const void* const* senders,
+                                void* const* receivers, int n, cudaStream_t stream);
 
 }  // namespace hf
 

@@ -396,6 +396,39 @@ __device__ __forceinline__ void build_stage_unrotated(const XferParams& P, const
   }
 }
 
+// Tiles of several transfer directions in one launch: direction d owns the
+// launch's tiles [base[d], base[d + 1]) (2 x its slots, so a slot's two
+// roles stay together), m_tiles[d] row blocks of U[d] distinct rows.
+template <int kDirs>
+struct DirTable {
+  int base[kDirs + 1];
+  int m_tiles[kDirs];
+  int U[kDirs];
+};
+
+template <int kDirs>
+__device__ __forceinline__ int build_dirs(const XferParams* Ps, int n_dir, DirTable<kDirs>* dt) {
+  int total = 0;
+  for (int d = 0; d < (kDirs == 1 ? 1 : n_dir); ++d) {
+    const int U = *Ps[d].n_distinct;
+    const int mt = (U + kPairRows - 1) / kPairRows;
+    dt->U[d] = U;
+    dt->m_tiles[d] = mt;
+    dt->base[d] = total;
+    total += 2 * Ps[d].n_l * mt * Ps[d].n_tiles_n;
+  }
+  dt->base[kDirs == 1 ? 1 : n_dir] = total;
+  return total;
+}
+
+template <int kDirs>
+__device__ __forceinline__ int dir_of(const DirTable<kDirs>& dt, int n_dir, int tile) {
+  if (kDirs == 1) return 0;
+  int d = 0;
+  while (d + 1 < n_dir && tile >= dt.base[d + 1]) ++d;
+  return d;
+}
+
 // Arrival on the leader CTA's copy of a pair barrier (`bar` is the local
 // offset): a local arrive in the leader, a relaxed remote arrive in the
 // follower.  What is announced is complete and visible before the call.
@@ -412,16 +445,16 @@ __device__ __forceinline__ void arrive_leader(uint32_t bar, int row0) {
 // layout.  A thread keeps LAG groups in flight: after committing k-block i
 // it waits for k-block i-LAG and fences it to the async proxy; then one lane
 // per warp arrives on that stage's barrier in the leader CTA of the pair.
-template <typename T, int LAG>
-__device__ __forceinline__ void gather_rows(const XferParams& P, uint8_t* sA, uint64_t* full_a,
+template <typename T, int LAG, int kDirs>
+__device__ __forceinline__ void gather_rows(const XferParams* Ps, const DirTable<kDirs>& dt,
+                                            int n_dir, uint8_t* sA, uint64_t* full_a,
                                             uint64_t* empty_a, volatile int* sAbort, int t,
-                                            int lane, int U, int row0, int total_tiles,
-                                            int tiles_per_lc, int first_tile, int tile_step) {
+                                            int lane, int row0, int total_tiles, int first_tile,
+                                            int tile_step) {
   constexpr int kBK = Elem<T>::kBK;
-  const bool by_slot = total_tiles >= 4 * tile_step;  // as in transfer_kernel
+  const bool by_slot = total_tiles >= 4 * tile_step;  // as in transfer_body
   constexpr int kPerChunk = 16 / sizeof(T);
-  const T* sender = reinterpret_cast<const T*>(P.sender);
-  const int stages = P.stages_a;
+  const int stages = Ps[0].stages_a;
   const int slab = t >> 5, rsub = lane >> 3, ch = lane & 7;
   int stage = 0;
   uint32_t phase = 0;
@@ -429,8 +462,12 @@ __device__ __forceinline__ void gather_rows(const XferParams& P, uint8_t* sA, ui
   bool ok = true;
   for (int seq = 0, tile = tile_of(0, first_tile, tile_step, by_slot); tile < total_tiles && ok;
        tile = tile_of(++seq, first_tile, tile_step, by_slot)) {
+    const int dd = dir_of(dt, n_dir, tile);
+    const XferParams& P = Ps[dd];
+    const int U = dt.U[dd];
+    const T* sender = reinterpret_cast<const T*>(P.sender);
     int lc, m, n;
-    decode_tile(tile, tiles_per_lc, P.n_tiles_n, P.l0, &lc, &m, &n);
+    decode_tile(tile - dt.base[dd], dt.m_tiles[dd] * P.n_tiles_n, P.n_tiles_n, P.l0, &lc, &m, &n);
     const int l = lc >> 1, c = lc & 1;
     // element offset of each segment's sender layer/role block, for the whole tile
     int64_t seg_base[kMaxSeg];
@@ -491,13 +528,19 @@ __device__ __forceinline__ void gather_rows(const XferParams& P, uint8_t* sA, ui
       arrive_leader(smem_addr(&full_a[(stage + stages - k) % stages]), row0);
 }
 
-template <typename T, bool kGather>
-__global__ void __launch_bounds__(kThreads, 1)
-    transfer_kernel(const __grid_constant__ CUtensorMap tmap_w, const XferParams P) {
+// The kernel body for one direction (kDirs = 1, the map and parameters are
+// kernel parameters) or several (tiles of all directions in one launch;
+// every role looks its tile's direction up and reads that direction's
+// parameters).  All directions share the dtype, the operand path and the
+// ring depths; a B stage is stage_b_stride bytes (the widest direction's).
+template <typename T, bool kGather, int kDirs>
+__device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const XferParams* Ps,
+                                              int n_dir, int stage_b_stride) {
   constexpr int kBK = Elem<T>::kBK;
+  const XferParams& P0 = Ps[0];
   extern __shared__ __align__(1024) uint8_t smem[];
   if (smem_addr(smem) & 1023u) {  // the swizzled stages need 1024-byte alignment
-    if (threadIdx.x == 0) atomicOr(P.status, HF_CHECK_INTERNAL);
+    if (threadIdx.x == 0) atomicOr(P0.status, HF_CHECK_INTERNAL);
     return;
   }
   const uint32_t rank = cluster_ctarank();  // 0: leader of the pair (issues the MMAs)
@@ -505,10 +548,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int first_tile = static_cast<int>(cluster_id_x());
   const int tile_step = static_cast<int>(nclusters_x());
   const int row0 = static_cast<int>(rank) * kBM;  // this CTA's rows within a pair tile
-  const int stages_a = P.stages_a, stages_b = P.stages_b;
-  const int half_bn = P.BN / 2;                    // B rows (receiver columns) per CTA
-  const int atom_b_bytes = half_bn * 128;
-  const int stage_b_bytes = kAtoms * atom_b_bytes;
+  const int stages_a = P0.stages_a, stages_b = P0.stages_b;
+  const int stage_b_bytes = stage_b_stride;
   uint8_t* sA = smem;
   uint8_t* sB = sA + stages_a * kStageABytes;
   float* sStg = reinterpret_cast<float*>(sB + stages_b * stage_b_bytes);
@@ -547,7 +588,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     *sAbort = 0;
     fence_barrier_init();
   }
-  if (warp == 0 && lane == 0) tma_prefetch_map(&tmap_w);
+  if (warp == 0 && lane == 0)
+    for (int d = 0; d < (kDirs == 1 ? 1 : n_dir); ++d) tma_prefetch_map(&maps[d]);
   if (warp == 1) {
     tmem_alloc_pair(smem_addr(sTmem), kTmemCols);
     tmem_relinquish_pair();
@@ -557,10 +599,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after_sync();
   const uint32_t tmem_base = *sTmem;
 
-  const int U = *P.n_distinct;
-  const int m_tiles = (U + kPairRows - 1) / kPairRows;
-  const int tiles_per_lc = m_tiles * P.n_tiles_n;
-  const int total_tiles = 2 * P.n_l * tiles_per_lc;
+  DirTable<kDirs> dt;
+  const int total_tiles = build_dirs<kDirs>(Ps, n_dir, &dt);
   const bool by_slot = total_tiles >= 4 * tile_step;
 
   if (warp == 0) {
@@ -572,8 +612,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       for (int seq = 0, tile = tile_of(0, first_tile, tile_step, by_slot); tile < total_tiles && ok;
        tile = tile_of(++seq, first_tile, tile_step, by_slot)) {
+        const int dd = dir_of(dt, n_dir, tile);
+        const XferParams& P = Ps[dd];
+        const CUtensorMap* tmap = &maps[dd];
+        const int half_bn = P.BN / 2;  // B rows (receiver columns) per CTA
+        const int atom_b_bytes = half_bn * 128;
         int lc, m, n;
-        decode_tile(tile, tiles_per_lc, P.n_tiles_n, P.l0, &lc, &m, &n);
+        decode_tile(tile - dt.base[dd], dt.m_tiles[dd] * P.n_tiles_n, P.n_tiles_n, P.l0, &lc, &m,
+                    &n);
         for (int kb = 0; kb < P.n_kb; ++kb) {
           if (!mbar_wait(smem_addr(&empty_b[stage]), phase ^ 1)) {
             raise_timeout(P, sAbort);
@@ -586,7 +632,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int a = 0; a < kAtoms; ++a)
             if (a < na)
-              tma_load_2d_pair(smem_addr(sB + stage * stage_b_bytes + a * atom_b_bytes), &tmap_w,
+              tma_load_2d_pair(smem_addr(sB + stage * stage_b_bytes + a * atom_b_bytes), tmap,
                                (kb * kAtoms + a) * kBK,
                                lc * P.d_r + n * P.BN + static_cast<int>(rank) * half_bn, fb);
           if (++stage == stages_b) {
@@ -610,9 +656,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint64_t desc_a0 = sw128_kmajor_desc(smem_addr(sA));
       const uint64_t desc_b0 = sw128_kmajor_desc(smem_addr(sB));
       const uint32_t step_a = kStageABytes >> 4, step_b = static_cast<uint32_t>(stage_b_bytes) >> 4;
-      const uint32_t atom_a = kAtomABytes >> 4, atom_b = static_cast<uint32_t>(atom_b_bytes) >> 4;
-      const uint32_t idesc = P.idesc;
-      const int n_kb = P.n_kb, last_atoms = P.last_atoms;
+      const uint32_t atom_a = kAtomABytes >> 4;
       int sa = 0, sb = 0;
       uint32_t pa = 0, pb = 0;
       int acc = 0;
@@ -620,6 +664,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       for (int seq = 0, tile = tile_of(0, first_tile, tile_step, by_slot); tile < total_tiles && ok;
        tile = tile_of(++seq, first_tile, tile_step, by_slot)) {
+        const XferParams& P = Ps[dir_of(dt, n_dir, tile)];
+        const uint32_t atom_b = static_cast<uint32_t>(P.BN / 2 * 128) >> 4;
+        const uint32_t idesc = P.idesc;
+        const int n_kb = P.n_kb, last_atoms = P.last_atoms;
         if (!mbar_wait(smem_addr(&tempty[acc]), acc_phase ^ 1)) {
           raise_timeout(P, sAbort);
           break;
@@ -674,7 +722,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_commit_pair(smem_addr(drain), 0x3);
     }
     if (lane == 0) {
-      if (!mbar_wait(smem_addr(drain), 0)) raise_timeout(P, sAbort);
+      if (!mbar_wait(smem_addr(drain), 0)) raise_timeout(P0, sAbort);
     }
     __syncwarp();
   } else if (warp < 10) {
@@ -689,17 +737,21 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int sp = warp & 3;  // TMEM lane quarter this warp may access
     const int row = sp * 32 + lane;
     const int tid_e = threadIdx.x - 64;
-    const int D = P.D_r, half = P.D_r / 2;
-    const int n_heads = P.BN / D;
-    const bool two_heads = n_heads >= 2;
-    const int n_pairs = two_heads ? n_heads / 2 : 1;
     const int ps = lane >> 2, qq = lane & 3;  // row slot 0..7, pair quad 0..3
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int seq = 0, tile = tile_of(0, first_tile, tile_step, by_slot); tile < total_tiles;
        tile = tile_of(++seq, first_tile, tile_step, by_slot)) {
+      const int dd = dir_of(dt, n_dir, tile);
+      const XferParams& P = Ps[dd];
+      const int U = dt.U[dd];
+      const int D = P.D_r, half = P.D_r / 2;
+      const int n_heads = P.BN / D;
+      const bool two_heads = n_heads >= 2;
+      const int n_pairs = two_heads ? n_heads / 2 : 1;
       int lc, m, n;
-      decode_tile(tile, tiles_per_lc, P.n_tiles_n, P.l0, &lc, &m, &n);
+      decode_tile(tile - dt.base[dd], dt.m_tiles[dd] * P.n_tiles_n, P.n_tiles_n, P.l0, &lc, &m,
+                  &n);
       const int c = lc & 1;
       if (!mbar_wait(smem_addr(&tfull[acc]), acc_phase)) {
         raise_timeout(P, sAbort);
@@ -823,12 +875,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------------------ A builders
     const int t = threadIdx.x - 320;  // 0..127
     if (kGather) {
-      switch (P.lag) {
-        case 1: gather_rows<T, 1>(P, sA, full_a, empty_a, sAbort, t, lane, U, row0, total_tiles, tiles_per_lc, first_tile, tile_step); break;
-        case 2: gather_rows<T, 2>(P, sA, full_a, empty_a, sAbort, t, lane, U, row0, total_tiles, tiles_per_lc, first_tile, tile_step); break;
-        case 3: gather_rows<T, 3>(P, sA, full_a, empty_a, sAbort, t, lane, U, row0, total_tiles, tiles_per_lc, first_tile, tile_step); break;
-        case 4: gather_rows<T, 4>(P, sA, full_a, empty_a, sAbort, t, lane, U, row0, total_tiles, tiles_per_lc, first_tile, tile_step); break;
-        default: gather_rows<T, 5>(P, sA, full_a, empty_a, sAbort, t, lane, U, row0, total_tiles, tiles_per_lc, first_tile, tile_step); break;
+      switch (P0.lag) {
+        case 1: gather_rows<T, 1, kDirs>(Ps, dt, n_dir, sA, full_a, empty_a, sAbort, t, lane, row0, total_tiles, first_tile, tile_step); break;
+        case 2: gather_rows<T, 2, kDirs>(Ps, dt, n_dir, sA, full_a, empty_a, sAbort, t, lane, row0, total_tiles, first_tile, tile_step); break;
+        case 3: gather_rows<T, 3, kDirs>(Ps, dt, n_dir, sA, full_a, empty_a, sAbort, t, lane, row0, total_tiles, first_tile, tile_step); break;
+        case 4: gather_rows<T, 4, kDirs>(Ps, dt, n_dir, sA, full_a, empty_a, sAbort, t, lane, row0, total_tiles, first_tile, tile_step); break;
+        default: gather_rows<T, 5, kDirs>(Ps, dt, n_dir, sA, full_a, empty_a, sAbort, t, lane, row0, total_tiles, first_tile, tile_step); break;
       }
     } else {
       // pooled CSR rows, blended sender layers and/or rotated sender keys:
@@ -838,11 +890,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       for (int seq = 0, tile = tile_of(0, first_tile, tile_step, by_slot); tile < total_tiles && ok;
        tile = tile_of(++seq, first_tile, tile_step, by_slot)) {
+        const int dd = dir_of(dt, n_dir, tile);
+        const XferParams& P = Ps[dd];
         int lc, m, n;
-        decode_tile(tile, tiles_per_lc, P.n_tiles_n, P.l0, &lc, &m, &n);
+        decode_tile(tile - dt.base[dd], dt.m_tiles[dd] * P.n_tiles_n, P.n_tiles_n, P.l0, &lc, &m,
+                    &n);
         const int l = lc >> 1, c = lc & 1;
         const LayerSegs segs = P.segs[l];
-        const int u = min(m * kPairRows + row0 + t, U - 1);
+        const int u = min(m * kPairRows + row0 + t, dt.U[dd] - 1);
         const int j0 = P.run_ptr[u];
         const int e0 = P.row_ptr[j0], e1 = P.row_ptr[j0 + 1];
         const bool unrot_k = P.unrot && c == 0;
@@ -896,6 +951,28 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after_sync();
     tmem_dealloc_pair(tmem_base, kTmemCols);
   }
+}
+
+template <typename T, bool kGather>
+__global__ void __launch_bounds__(kThreads, 1)
+    transfer_kernel(const __grid_constant__ CUtensorMap tmap_w,
+                    const __grid_constant__ XferParams P) {
+  transfer_body<T, kGather, 1>(&tmap_w, &P, 1, kAtoms * (P.BN / 2) * 128);
+}
+
+// Several directions in one launch (hf_transfer_batch).
+struct BatchParams {
+  CUtensorMap maps[kMaxBatch];
+  XferParams P[kMaxBatch];
+  int n_dir;
+  int stage_b_stride;
+};
+static_assert(sizeof(BatchParams) < 32000, "BatchParams must fit the kernel parameter space");
+
+template <typename T, bool kGather>
+__global__ void __launch_bounds__(kThreads, 1)
+    transfer_batch_kernel(const __grid_constant__ BatchParams B) {
+  transfer_body<T, kGather, kMaxBatch>(B.maps, B.P, B.n_dir, B.stage_b_stride);
 }
 
 // ---------------------------------------------------------------------------
@@ -966,10 +1043,11 @@ void pick_rings(int BN, int* stages_a, int* stages_b, int* lag) {
   *lag = 1;
 }
 
-template <typename T, bool kGather>
-hf_status launch_typed(const CUtensorMap& mw, const XferParams& P, int64_t max_pair_tiles,
-                       size_t smem, cudaStream_t stream) {
-  auto kern = transfer_kernel<T, kGather>;
+// Launches `kern` with clusters of two CTAs: one CTA pair per co-resident
+// cluster slot, at most one per pair tile.
+template <typename Kern, typename... Args>
+hf_status launch_pairs(Kern kern, int64_t max_pair_tiles, size_t smem, cudaStream_t stream,
+                       Args... args) {
   HF_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                    static_cast<int>(smem)),
               "set shared memory size");
@@ -992,26 +1070,28 @@ hf_status launch_typed(const CUtensorMap& mw, const XferParams& P, int64_t max_p
     clusters = std::min(clusters, active);
   clusters = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(clusters, max_pair_tiles)));
   cfg.gridDim = dim3(2 * clusters, 1, 1);
-  HF_CUDA_TRY(cudaLaunchKernelEx(&cfg, kern, mw, P), "transfer kernel launch");
+  HF_CUDA_TRY(cudaLaunchKernelEx(&cfg, kern, args...), "transfer kernel launch");
   return HF_OK;
 }
 
 }  // namespace
 
-hf_status launch_transfer(hf_plan_s* p, const void* sender, void* receiver, cudaStream_t stream,
-                          int l_begin, int l_end) {
+namespace {
+
+// The kernel parameters and map tile descriptor of one plan's launch over
+// receiver layers [l_begin, l_end); *max_pair_tiles bounds its pair tiles.
+hf_status make_xfer(hf_plan_s* p, const void* sender, void* receiver, int l_begin, int l_end,
+                    XferParams* out, CUtensorMap* map_out, int64_t* max_pair_tiles) {
   const hf_plan_desc& d = p->desc;
-  if (l_end < 0) l_end = d.L_r;
-  if (p->T_r == 0 || l_end <= l_begin) return HF_OK;
   const bool f32 = d.dtype == HF_F32;
   const int esize = f32 ? 4 : 2;
   const int bk = 128 / esize;
-  CUtensorMap mw;
+  CUtensorMap& mw = *map_out;
   hf_status s = make_map(&mw, d.d_W, f32, static_cast<uint64_t>(d.L_r) * 2 * p->d_r,
                          static_cast<uint64_t>(p->K), static_cast<uint32_t>(p->BN / 2),
                          static_cast<uint32_t>(bk), CU_TENSOR_MAP_L2_PROMOTION_L2_256B);
   if (s != HF_OK) return s;
-  XferParams P;
+  XferParams& P = *out;
   std::memset(&P, 0, sizeof(P));
   char* ws = p->ws;
   P.sender = sender;
@@ -1056,14 +1136,88 @@ hf_status launch_transfer(hf_plan_s* p, const void* sender, void* receiver, cuda
   P.knorm = d.d_knorm_w ? 1 : 0;
   P.knorm_eps = d.knorm_eps;
   P.idesc = make_idesc(f32 ? 2u : 1u, kPairRows, p->BN);
-  const size_t smem = smem_bytes(p->BN, P.stages_a, P.stages_b);
-  const int64_t max_pair_tiles =
+  *max_pair_tiles =
       2LL * P.n_l * ((p->T_r + kPairRows - 1) / kPairRows) * static_cast<int64_t>(P.n_tiles_n);
-  if (f32)
-    return p->gather ? launch_typed<float, true>(mw, P, max_pair_tiles, smem, stream)
-                     : launch_typed<float, false>(mw, P, max_pair_tiles, smem, stream);
-  return p->gather ? launch_typed<__nv_bfloat16, true>(mw, P, max_pair_tiles, smem, stream)
-                   : launch_typed<__nv_bfloat16, false>(mw, P, max_pair_tiles, smem, stream);
+  return HF_OK;
+}
+
+template <typename T, bool kGather>
+hf_status launch_batch_typed(const BatchParams& B, int64_t max_pair_tiles, size_t smem,
+                             cudaStream_t stream) {
+  return launch_pairs(transfer_batch_kernel<T, kGather>, max_pair_tiles, smem, stream, B);
+}
+
+}  // namespace
+
+hf_status launch_transfer(hf_plan_s* p, const void* sender, void* receiver, cudaStream_t stream,
+                          int l_begin, int l_end) {
+  const hf_plan_desc& d = p->desc;
+  if (l_end < 0) l_end = d.L_r;
+  if (p->T_r == 0 || l_end <= l_begin) return HF_OK;
+  XferParams P;
+  CUtensorMap mw;
+  int64_t max_pair_tiles = 0;
+  hf_status s = make_xfer(p, sender, receiver, l_begin, l_end, &P, &mw, &max_pair_tiles);
+  if (s != HF_OK) return s;
+  const size_t smem = smem_bytes(p->BN, P.stages_a, P.stages_b);
+  if (d.dtype == HF_F32)
+    return p->gather ? launch_pairs(transfer_kernel<float, true>, max_pair_tiles, smem, stream, mw, P)
+                     : launch_pairs(transfer_kernel<float, false>, max_pair_tiles, smem, stream, mw, P);
+  return p->gather
+             ? launch_pairs(transfer_kernel<__nv_bfloat16, true>, max_pair_tiles, smem, stream, mw, P)
+             : launch_pairs(transfer_kernel<__nv_bfloat16, false>, max_pair_tiles, smem, stream, mw, P);
+}
+
+bool batch_compatible(const hf_plan_s* const* plans, int n) {
+  for (int i = 1; i < n; ++i)
+    if (plans[i]->desc.dtype != plans[0]->desc.dtype || plans[i]->gather != plans[0]->gather)
+      return false;
+  return true;
+}
+
+hf_status launch_transfer_batch(hf_plan_s* const* plans, const void* const* senders,
+                                void* const* receivers, int n, cudaStream_t stream) {
+  BatchParams* B = new BatchParams();
+  std::memset(B, 0, sizeof(*B));
+  int64_t tiles = 0;
+  int max_bn = 0, k = 0;
+  for (int i = 0; i < n; ++i) {
+    hf_plan_s* p = plans[i];
+    if (p->T_r == 0) continue;
+    int64_t mt = 0;
+    const hf_status s = make_xfer(p, senders[i], receivers[i], 0, p->desc.L_r, &B->P[k],
+                                  &B->maps[k], &mt);
+    if (s != HF_OK) {
+      delete B;
+      return s;
+    }
+    tiles += mt;
+    max_bn = std::max(max_bn, p->BN);
+    ++k;
+  }
+  if (k == 0) {
+    delete B;
+    return HF_OK;
+  }
+  int sa = 0, sb = 0, lag = 0;
+  pick_rings(max_bn, &sa, &sb, &lag);
+  for (int i = 0; i < k; ++i) {
+    B->P[i].stages_a = sa;
+    B->P[i].stages_b = sb;
+    B->P[i].lag = lag;
+  }
+  B->n_dir = k;
+  B->stage_b_stride = kAtoms * (max_bn / 2) * 128;
+  const size_t smem = smem_bytes(max_bn, sa, sb);
+  hf_status s;
+  if (plans[0]->desc.dtype == HF_F32)
+    s = plans[0]->gather ? launch_batch_typed<float, true>(*B, tiles, smem, stream)
+                         : launch_batch_typed<float, false>(*B, tiles, smem, stream);
+  else
+    s = plans[0]->gather ? launch_batch_typed<__nv_bfloat16, true>(*B, tiles, smem, stream)
+                         : launch_batch_typed<__nv_bfloat16, false>(*B, tiles, smem, stream);
+  delete B;
+  return s;
 }
 
 }  // namespace hf

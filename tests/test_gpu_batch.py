@@ -1,7 +1,7 @@
 """hf_transfer_batch: the six directions of a three-agent message round
-(message spans after a context, every family pair) in one call.  Each
-direction must equal, bit for bit, its own hf_transfer (the same kernel on
-the same inputs), and match the fp64 oracle within the parity tolerance."""
+(message spans after a context, every family pair) in one launch.  Each
+direction must equal, bit for bit, its own hf_transfer (the same tiles, the
+same code), and match the fp64 oracle within the parity tolerance."""
 
 import numpy as np
 import pytest
@@ -36,6 +36,22 @@ def test_message_round_batch_matches_single_transfers_and_oracle():
     for c, ref in zip(cases, single):
         assert torch.equal(c.job.receiver, ref), c.w.name
         c.check_parity()
+
+
+def test_batch_mixing_operand_paths():
+    """Plans that differ in dtype or operand path (copied rows vs built rows)
+    go to separate launches; results equal their single transfers."""
+    ws = [W.message_round(msg_tokens=60)[0], W.tiny(),
+          W.llama_to_ministral(300).with_(L_s=3, L_r=3, align_mode="overlap_mean")]
+    cases = [Case(w, sentinel=SENTINEL).run() for w in ws]
+    single = [c.job.receiver.clone() for c in cases]
+    for c in cases:
+        c.job.receiver.fill_(SENTINEL)
+    B.transfer_batch([c.job.plan for c in cases], [c.sender for c in cases],
+                     [c.job.receiver for c in cases])
+    torch.cuda.synchronize()
+    for c, ref in zip(cases, single):
+        assert torch.equal(c.job.receiver, ref), c.w.name
 
 
 def test_batch_of_one_and_empty_batch():
