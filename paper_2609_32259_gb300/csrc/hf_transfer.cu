@@ -43,8 +43,10 @@ namespace {
 
 constexpr int kBM = 128;                 // distinct rows per CTA of a pair tile
 constexpr int kPairRows = 2 * kBM;       // distinct rows per pair tile (UMMA M = 256)
-constexpr int kThreads = 448;            // 14 warps
-constexpr int kBuilderWarps = 4;         // A tile builders: warps 10-13
+constexpr int kEpiWarps = 10;            // epilogue: warps 2-11 (8 of them read TMEM)
+constexpr int kBuilderWarps = 4;         // A tile builders: warps 12-15
+constexpr int kEpiThreads = 32 * kEpiWarps;
+constexpr int kThreads = 64 + kEpiThreads + 32 * kBuilderWarps;  // 16 warps
 constexpr int kAtoms = 2;                // 128-byte swizzle atoms (k-blocks) per pipeline stage
 constexpr int kAtomABytes = kBM * 128;   // 128 rows x 128 bytes
 constexpr int kStageABytes = kAtoms * kAtomABytes;
@@ -255,6 +257,7 @@ __device__ __forceinline__ void copy_epilogue(const XferParams& P, uint32_t ta,
     uint8_t* srow = stg + row * 256;
 #pragma unroll
     for (int k = 0; k < kHalfCols; k += 16) {
+      if (e >= 8) break;  // the two extra warps only copy
       const int col = pc0 + g * kHalfCols + k;
       uint32_t v[16];
       tmem_load_16(ta + static_cast<uint32_t>(col), v);
@@ -274,8 +277,8 @@ __device__ __forceinline__ void copy_epilogue(const XferParams& P, uint32_t ta,
             pack16(y + h * kPerChunk, (const T*)nullptr);
       }
     }
-    named_barrier_sync(1, 256);
-    for (int u = e; u < nrows; u += 8) {
+    named_barrier_sync(1, kEpiThreads);
+    for (int u = e; u < nrows; u += kEpiWarps) {
       const uint4 val = *reinterpret_cast<const uint4*>(stg + u * 256 + ((cidx ^ (u & 7)) << 4));
       const int je = srun[u + 1];
       for (int j = srun[u] + hw; j < je; j += 2) {
@@ -286,7 +289,7 @@ __device__ __forceinline__ void copy_epilogue(const XferParams& P, uint32_t ta,
                  val);
       }
     }
-    named_barrier_sync(1, 256);
+    named_barrier_sync(1, kEpiThreads);
   }
 }
 
@@ -582,7 +585,7 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(smem_addr(&tfull[a]), 1);
-      mbar_init(smem_addr(&tempty[a]), 16);  // every epilogue warp of the pair
+      mbar_init(smem_addr(&tempty[a]), 2 * kEpiWarps);  // every epilogue warp of the pair
     }
     mbar_init(smem_addr(drain), 1);
     *sAbort = 0;
@@ -725,17 +728,18 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
       if (!mbar_wait(smem_addr(drain), 0)) raise_timeout(P0, sAbort);
     }
     __syncwarp();
-  } else if (warp < 10) {
+  } else if (warp < 2 + kEpiWarps) {
     // ------------------------------------------------------------ epilogue
-    // Eight warps per CTA, for the CTA's 128 rows of the pair tile.  Step 1
-    // (per 16 rotation pairs of a head pair): warp (g, sp) reads TMEM lane
-    // quarter sp of head 2*hp+g, applies 1/r, bias and key norm, and stages
-    // fp32 rows in smem.  Step 2: the eight warps split the rows' receiver
-    // positions and write both heads, rotated.
-    const int e = warp - 2;   // 0..7: slice of the tile's receiver rows
-    const int g = e >> 2;     // head of the pair this warp stages
+    // Ten warps per CTA, for the CTA's 128 rows of the pair tile.  Step 1
+    // (per 16 rotation pairs of a head pair): warp (g, sp), e < 8, reads TMEM
+    // lane quarter sp of head 2*hp+g, applies 1/r, bias and key norm, and
+    // stages fp32 rows in smem.  Step 2: the ten warps split the rows'
+    // receiver positions and write both heads, rotated.
+    const int e = warp - 2;   // 0..9: slice of the tile's receiver rows
+    const int g = e >> 2;     // head of the pair this warp stages (e < 8)
     const int sp = warp & 3;  // TMEM lane quarter this warp may access
     const int row = sp * 32 + lane;
+    const bool stager = e < 8;
     const int tid_e = threadIdx.x - 64;
     const int ps = lane >> 2, qq = lane & 3;  // row slot 0..7, pair quad 0..3
     int acc = 0;
@@ -761,14 +765,14 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
       const int u0 = m * kPairRows + row0;
       const int nrows = min(kBM, U - u0);  // <= 0: this CTA has no rows in the tile
       if (nrows > 0) {
-        for (int i = tid_e; i <= nrows; i += 256) {
+        for (int i = tid_e; i <= nrows; i += kEpiThreads) {
           sRun[i] = P.run_ptr[u0 + i];
           sUpos[i] = i < nrows ? P.upos[u0 + i] : 0;
         }
-        named_barrier_sync(1, 256);
+        named_barrier_sync(1, kEpiThreads);
         // this warp's receiver rows [wjb, wje); lane slot ps takes rows wjb+ps, +8, ...
         const int jb = sRun[0], je = sRun[nrows];
-        const int per = (je - jb + 7) >> 3;
+        const int per = (je - jb + kEpiWarps - 1) / kEpiWarps;
         const int wjb = min(je, jb + e * per), wje = min(je, wjb + per);
         const int n_it = (wje - wjb + 7) >> 3;
         const int j0 = wjb + ps;
@@ -786,7 +790,7 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
                            reinterpret_cast<uint8_t*>(sStg), g, row, e, lane, out_lc, n * P.BN);
         } else
         for (int hp = 0; hp < n_pairs; ++hp) {
-          const bool stages_head = g == 0 || two_heads;
+          const bool stages_head = stager && (g == 0 || two_heads);
           const int tcol = (2 * hp + g) * D;            // accumulator column of this warp's head
           const int ocol_pair = n * P.BN + 2 * hp * D;  // receiver feature of the pair's first head
           float rn = 1.0f;
@@ -837,7 +841,7 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
                 *reinterpret_cast<float4*>(srow + ((k ^ (row & 7)) << 2)) =
                     make_float4(y[4 * k], y[4 * k + 1], y[4 * k + 2], y[4 * k + 3]);
             }
-            named_barrier_sync(1, 256);
+            named_barrier_sync(1, kEpiThreads);
             // step 2: rows of this warp's slice, both heads of the pair
             float f[4], C8[4], S8[4];
 #pragma unroll
@@ -861,7 +865,7 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
                 walk_step<T>(wk, j, it, sRun, sUpos, sStg, qq, two_heads, do_rope, f, C8, S8, P,
                              out_lc, ocol_pair, q, half);
             }
-            named_barrier_sync(1, 256);
+            named_barrier_sync(1, kEpiThreads);
           }
         }
       }
@@ -873,7 +877,7 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
     }
   } else {
     // ------------------------------------------------------------ A builders
-    const int t = threadIdx.x - 320;  // 0..127
+    const int t = threadIdx.x - 64 - kEpiThreads;  // 0..127
     if (kGather) {
       switch (P0.lag) {
         case 1: gather_rows<T, 1, kDirs>(Ps, dt, n_dir, sA, full_a, empty_a, sAbort, t, lane, row0, total_tiles, first_tile, tile_step); break;
