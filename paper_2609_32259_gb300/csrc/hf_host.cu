@@ -151,8 +151,9 @@ extern "C" hf_status hf_transfer_host(hf_plan plan, const void* h_sender_kv, voi
     for (int l = l0; l < l1; ++l) need = std::max(need, plan->max_sender_layer[l] + 1);
     if (need > copied) {
       if (gather) {
-        // 128-thread blocks at 32 registers fit in the register file beside a
-        // transfer kernel CTA (448 x 128 registers), so the gather overlaps it
+        // small blocks at few registers: the gather of group g + 1 runs
+        // wherever an SM frees up (the transfer kernel's CTAs hold the whole
+        // register file while they run), ahead of the group's own kernel
         gather_sender_rows<<<4 * device_sm_count(), 128, 0, plan->s_h2d>>>(
             static_cast<const uint4*>(h_sender_dev), reinterpret_cast<uint4*>(ds), ucol,
             n_distinct, copied, need, plan->s_rows, static_cast<int>(row_bytes / 16));
