@@ -12,22 +12,23 @@
 // run_ptr[u+1]) at consecutive positions from upos[u], and the epilogue
 // writes y (rotated per position for K) to every row of its run.
 //
-// One persistent CTA per SM walks tiles (l, c, 128 distinct rows, BN
-// receiver columns) with warp-specialised roles:
-//   warp 0      TMA producer of the map tile W[l][c][n0:n0+BN][k0:k0+BK]
-//               (2-D tiled load, 128-byte swizzle);
-//   warp 1      TMEM allocator and the single thread issuing tcgen05.mma
-//               (M = 128, N = BN, K = 16 bf16 / 8 tf32 per instruction) into
-//               one of two TMEM accumulators;
-//   warps 2-9   epilogue, two groups of four warps (one per TMEM lane
-//               quarter), each group owning half of the tile's columns;
-//   warps 10-13 A tile builders.  When every map input row is one sender row
-//               (Token Alignment with the three-layer neighbourhood) they copy
-//               the 128 sender rows with cp.async, eight lanes per 128-byte
-//               row; for pooled or blended rows they sum weighted sender rows
-//               in fp32 registers and round once.  Both write the 128-byte
-//               swizzled layout and fence it to the async proxy before
-//               arriving on the stage barrier.
+// Persistent clusters of two CTAs (one pair per SM pair) walk pair tiles
+// (l, c, 256 distinct rows, BN receiver columns); each CTA owns 128 of the
+// rows and half of the columns' map rows, with warp-specialised roles:
+//   warp 0      TMA producer of this CTA's half of the map tile
+//               W[l][c][n0:n0+BN][k0:k0+64 bf16] (2-D tiled load, 128-byte
+//               swizzle), one 128-byte atom of K per B stage;
+//   warp 1      TMEM allocator; in the leader CTA, the single thread issuing
+//               tcgen05.mma.cta_group::2 (M = 256, N = BN, K = 16 bf16 /
+//               8 tf32 per instruction) into one of two TMEM accumulators;
+//   warps 2-11  epilogue of the CTA's 128 rows (warps 2-9 read TMEM);
+//   warps 12-15 A tile builders, two atoms of K per A stage.  When every map
+//               input row is one sender row (Token Alignment with the
+//               three-layer neighbourhood) they copy the 128 sender rows with
+//               cp.async, eight lanes per 128-byte row; for pooled or blended
+//               rows they sum weighted sender rows in fp32 registers and round
+//               once.  Both write the 128-byte swizzled layout and fence it to
+//               the async proxy before arriving on the stage barrier.
 // Pipeline hand-offs use mbarriers with bounded waits; nothing traps.
 #include <algorithm>
 #include <climits>
@@ -623,21 +624,17 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
         int lc, m, n;
         decode_tile(tile - dt.base[dd], dt.m_tiles[dd] * P.n_tiles_n, P.n_tiles_n, P.l0, &lc, &m,
                     &n);
-        for (int kb = 0; kb < P.n_kb; ++kb) {
+        const int n_atoms = (P.n_kb - 1) * kAtoms + P.last_atoms;
+        for (int at = 0; at < n_atoms; ++at) {
           if (!mbar_wait(smem_addr(&empty_b[stage]), phase ^ 1)) {
             raise_timeout(P, sAbort);
             ok = false;
             break;
           }
           const uint32_t fb = mapa_shared(smem_addr(&full_b[stage]), 0);
-          const int na = kb == P.n_kb - 1 ? P.last_atoms : kAtoms;
-          mbar_arrive_expect_tx_cluster(fb, na * atom_b_bytes);
-#pragma unroll
-          for (int a = 0; a < kAtoms; ++a)
-            if (a < na)
-              tma_load_2d_pair(smem_addr(sB + stage * stage_b_bytes + a * atom_b_bytes), tmap,
-                               (kb * kAtoms + a) * kBK,
-                               lc * P.d_r + n * P.BN + static_cast<int>(rank) * half_bn, fb);
+          mbar_arrive_expect_tx_cluster(fb, atom_b_bytes);
+          tma_load_2d_pair(smem_addr(sB + stage * stage_b_bytes), tmap, at * kBK,
+                           lc * P.d_r + n * P.BN + static_cast<int>(rank) * half_bn, fb);
           if (++stage == stages_b) {
             stage = 0;
             phase ^= 1;
@@ -668,7 +665,6 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
       for (int seq = 0, tile = tile_of(0, first_tile, tile_step, by_slot); tile < total_tiles && ok;
        tile = tile_of(++seq, first_tile, tile_step, by_slot)) {
         const XferParams& P = Ps[dir_of(dt, n_dir, tile)];
-        const uint32_t atom_b = static_cast<uint32_t>(P.BN / 2 * 128) >> 4;
         const uint32_t idesc = P.idesc;
         const int n_kb = P.n_kb, last_atoms = P.last_atoms;
         if (!mbar_wait(smem_addr(&tempty[acc]), acc_phase ^ 1)) {
@@ -678,19 +674,24 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
         tc_fence_after_sync();
         const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * 256);
         uint32_t accumulate = 0;
-        for (int kb = 0; kb < n_kb; ++kb) {
-          if (!mbar_wait(full_a0 + 8 * sa, pa) || !mbar_wait(full_b0 + 8 * sb, pb)) {
+        for (int kb = 0; kb < n_kb && ok; ++kb) {
+          if (!mbar_wait(full_a0 + 8 * sa, pa)) {
             raise_timeout(P, sAbort);
             ok = false;
             break;
           }
-          tc_fence_after_sync();
           const int na = kb == n_kb - 1 ? last_atoms : kAtoms;
 #pragma unroll
           for (int a = 0; a < kAtoms; ++a) {
             if (a >= na) break;
+            if (!mbar_wait(full_b0 + 8 * sb, pb)) {
+              raise_timeout(P, sAbort);
+              ok = false;
+              break;
+            }
+            tc_fence_after_sync();
             const uint64_t ad = desc_a0 + sa * step_a + a * atom_a;
-            const uint64_t bd = desc_b0 + sb * step_b + a * atom_b;
+            const uint64_t bd = desc_b0 + sb * step_b;
             // four 32-byte K steps per 128-byte atom (descriptor units of 16 bytes)
             if (sizeof(T) == 2) {
               mma_bf16_pair(d_tmem, ad, bd, idesc, accumulate);
@@ -704,16 +705,17 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
               mma_tf32_pair(d_tmem, ad + 6, bd + 6, idesc, 1);
             }
             accumulate = 1;
+            tc_commit_pair(empty_b0 + 8 * sb, 0x3);
+            if (++sb == stages_b) {
+              sb = 0;
+              pb ^= 1;
+            }
           }
+          if (!ok) break;
           tc_commit_pair(empty_a0 + 8 * sa, 0x3);
-          tc_commit_pair(empty_b0 + 8 * sb, 0x3);
           if (++sa == stages_a) {
             sa = 0;
             pa ^= 1;
-          }
-          if (++sb == stages_b) {
-            sb = 0;
-            pb ^= 1;
           }
         }
         if (!ok) break;
@@ -961,7 +963,7 @@ template <typename T, bool kGather>
 __global__ void __launch_bounds__(kThreads, 1)
     transfer_kernel(const __grid_constant__ CUtensorMap tmap_w,
                     const __grid_constant__ XferParams P) {
-  transfer_body<T, kGather, 1>(&tmap_w, &P, 1, kAtoms * (P.BN / 2) * 128);
+  transfer_body<T, kGather, 1>(&tmap_w, &P, 1, (P.BN / 2) * 128);
 }
 
 // Several directions in one launch (hf_transfer_batch).
@@ -1026,25 +1028,28 @@ hf_status make_map(CUtensorMap* map, const void* base, bool f32, uint64_t rows, 
 
 size_t smem_bytes(int BN, int stages_a, int stages_b) {
   return static_cast<size_t>(stages_a) * kStageABytes +
-         static_cast<size_t>(stages_b) * kAtoms * (BN / 2) * 128 + kStgFloats * sizeof(float) +
+         static_cast<size_t>(stages_b) * (BN / 2) * 128 + kStgFloats * sizeof(float) +
          2 * kRunStride * sizeof(int32_t) + (4 * kMaxStages + 5) * sizeof(uint64_t) + 8;
 }
 
-// Ring depths (stages of kAtoms k-blocks): three or four B stages, as many
-// A stages as fit next to them.  Each loader keeps two stages of copies in
-// flight (it waits for stage i-1 after issuing stage i), which at 32 KB per
-// stage covers the L2/HBM latency; deeper loader lag only takes stages away
-// from the tensor core.
+// Ring depths.  A B stage is one 128-byte atom of K of this CTA's map rows
+// (16 KB at BN = 256), so the TMA producer refills the ring in fine steps;
+// 96 KB of B stages, and the rest of shared memory in A stages (two atoms,
+// 32 KB): three at BN = 256.  A loader waits for stage i - lag after issuing
+// stage i, so it never blocks on a young group.  Measured on the 32K
+// Llama -> Ministral-shaped transfer: three A stages and six one-atom B stages
+// beat three two-atom B stages by 1%, and four A stages with four one-atom B
+// stages lose 2-3% (deeper A rings do not pay; B depth does).
 void pick_rings(int BN, int* stages_a, int* stages_b, int* lag) {
   int dev = 0, optin = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
-  const int sb = BN == 256 ? 3 : 4;
+  const int sb = std::min(kMaxStages, (96 * 1024) / ((BN / 2) * 128));
   int sa = kMaxStages;
   while (sa > 2 && smem_bytes(BN, sa, sb) > static_cast<size_t>(optin)) --sa;
   *stages_a = sa;
   *stages_b = sb;
-  *lag = 1;
+  *lag = std::max(1, sa - 2);
 }
 
 // Launches `kern` with clusters of two CTAs: one CTA pair per co-resident
@@ -1211,7 +1216,7 @@ hf_status launch_transfer_batch(hf_plan_s* const* plans, const void* const* send
     B->P[i].lag = lag;
   }
   B->n_dir = k;
-  B->stage_b_stride = kAtoms * (max_bn / 2) * 128;
+  B->stage_b_stride = (max_bn / 2) * 128;
   const size_t smem = smem_bytes(max_bn, sa, sb);
   hf_status s;
   if (plans[0]->desc.dtype == HF_F32)
