@@ -181,58 +181,70 @@ __device__ __forceinline__ void rotate4(float4& x, float4& y, const float* c, co
   y = make_float4(y0, y1, y2, y3);
 }
 
-// The epilogue's position walk: a lane owns four rotation pairs (columns
-// q+4*qq .. +3 of the first half of each head and their partners half
-// further on) of one receiver row j at a time, for up to two heads, and
-// carries the RoPE angles of its four frequencies from row j - 8.
-struct Walk {
-  int u;       // tile row holding the current receiver row
-  int expect;  // position for which the carried angles are valid
-  float cs[4], sn[4];
-};
-
+// The epilogue's position walk for one lane: it owns four rotation pairs
+// (columns q+4*qq .. +3 of the first half of each head and their partners
+// half further on) of up to two heads, for the consecutive receiver rows
+// [jb, je) of one slice.  Shared memory is slow to answer while the tensor
+// core streams its operands, so the lane keeps the staged (unrotated) values
+// of its current distinct row in registers and reads the next row's only
+// when the walk enters its run; positions inside a run, and across runs of
+// one request, are consecutive, so the angles advance by one position per
+// row (re-anchored exactly every 16 rows and wherever the position jumps).
 template <typename T>
-__device__ __forceinline__ void walk_step(Walk& w, int j, int it, const int32_t* srun,
+__device__ __forceinline__ void walk_rows(int jb, int je, int u, const int32_t* srun,
                                           const int32_t* supos, const float* stg, int qq,
                                           bool two_heads, bool do_rope, const float* f,
-                                          const float* C8, const float* S8, const XferParams& P,
+                                          const float* C1, const float* S1, const XferParams& P,
                                           T* out_lc, int ocol, int q, int half) {
-  const int drow = P.paged ? __ldg(P.dst_row + j) : j;
-  while (srun[w.u + 1] <= j) ++w.u;
-  const int u = w.u;
-  const float* urow = stg + u * 64;
-  const int sw = u & 7;
-  float4 a0 = *reinterpret_cast<const float4*>(urow + ((qq ^ sw) << 2));
-  float4 b0 = *reinterpret_cast<const float4*>(urow + (((4 + qq) ^ sw) << 2));
-  float4 a1 = make_float4(0.f, 0.f, 0.f, 0.f), b1 = a1;
-  if (two_heads) {
-    a1 = *reinterpret_cast<const float4*>(urow + 32 + ((qq ^ sw) << 2));
-    b1 = *reinterpret_cast<const float4*>(urow + 32 + (((4 + qq) ^ sw) << 2));
-  }
-  if (do_rope) {
-    const int p = supos[u] + (j - srun[u]);
-    if (p != w.expect || (it & 15) == 0) {
-#pragma unroll
-      for (int k = 0; k < 4; ++k) rope_sincos(p, f[k], &w.sn[k], &w.cs[k]);
-    } else {  // advance every angle by eight positions
-#pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        const float t = w.cs[k] * C8[k] - w.sn[k] * S8[k];
-        w.sn[k] = w.sn[k] * C8[k] + w.cs[k] * S8[k];
-        w.cs[k] = t;
+  if (jb >= je) return;
+  float4 a0, b0, a1 = make_float4(0.f, 0.f, 0.f, 0.f), b1 = a1;
+  int uend = 0, pb = 0;  // end of the current run; position of row j is pb + j
+  int expect = INT_MIN;  // position for which cs/sn are valid
+  float cs[4] = {1.f, 1.f, 1.f, 1.f}, sn[4] = {0.f, 0.f, 0.f, 0.f};
+  --u;
+  for (int j = jb; j < je; ++j) {
+    if (j >= uend) {  // first row, or the first row of a later run
+      do {
+        ++u;
+      } while (srun[u + 1] <= j);
+      uend = srun[u + 1];
+      pb = supos[u] - srun[u];
+      const float* urow = stg + u * 64;
+      const int sw = u & 7;
+      a0 = *reinterpret_cast<const float4*>(urow + ((qq ^ sw) << 2));
+      b0 = *reinterpret_cast<const float4*>(urow + (((4 + qq) ^ sw) << 2));
+      if (two_heads) {
+        a1 = *reinterpret_cast<const float4*>(urow + 32 + ((qq ^ sw) << 2));
+        b1 = *reinterpret_cast<const float4*>(urow + 32 + (((4 + qq) ^ sw) << 2));
       }
     }
-    w.expect = p + 8;
-    rotate4(a0, b0, w.cs, w.sn);
-    if (two_heads) rotate4(a1, b1, w.cs, w.sn);
-  }
-  if (drow >= 0) {
-    T* o = out_lc + static_cast<int64_t>(drow) * P.d_r + ocol + q + 4 * qq;
-    store4(o, a0);
-    store4(o + half, b0);
-    if (two_heads) {
-      store4(o + 2 * half, a1);
-      store4(o + 3 * half, b1);
+    const int drow = P.paged ? __ldg(P.dst_row + j) : j;
+    float4 x0 = a0, y0 = b0, x1 = a1, y1 = b1;
+    if (do_rope) {
+      const int p = pb + j;
+      if (p != expect || ((j - jb) & 15) == 0) {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) rope_sincos(p, f[k], &sn[k], &cs[k]);
+      } else {  // advance every angle by one position
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const float t = cs[k] * C1[k] - sn[k] * S1[k];
+          sn[k] = sn[k] * C1[k] + cs[k] * S1[k];
+          cs[k] = t;
+        }
+      }
+      expect = p + 1;
+      rotate4(x0, y0, cs, sn);
+      if (two_heads) rotate4(x1, y1, cs, sn);
+    }
+    if (drow >= 0) {
+      T* o = out_lc + static_cast<int64_t>(drow) * P.d_r + ocol + q + 4 * qq;
+      store4(o, x0);
+      store4(o + half, y0);
+      if (two_heads) {
+        store4(o + 2 * half, x1);
+        store4(o + 3 * half, y1);
+      }
     }
   }
 }
@@ -279,16 +291,37 @@ __device__ __forceinline__ void copy_epilogue(const XferParams& P, uint32_t ta,
       }
     }
     named_barrier_sync(1, kEpiThreads);
-    for (int u = e; u < nrows; u += kEpiWarps) {
-      const uint4 val = *reinterpret_cast<const uint4*>(stg + u * 256 + ((cidx ^ (u & 7)) << 4));
-      const int je = srun[u + 1];
-      for (int j = srun[u] + hw; j < je; j += 2) {
+    // the next distinct row's staged chunk and run bounds are read while this
+    // row's receiver rows are stored (shared-memory reads are slow to answer
+    // while the tensor core streams its operands)
+    int u = e;
+    uint4 val = make_uint4(0u, 0u, 0u, 0u);
+    int js = 0, je = 0;
+    if (u < nrows) {
+      val = *reinterpret_cast<const uint4*>(stg + u * 256 + ((cidx ^ (u & 7)) << 4));
+      js = srun[u];
+      je = srun[u + 1];
+    }
+    while (u < nrows) {
+      const int un = u + kEpiWarps;
+      uint4 nval = val;
+      int njs = 0, nje = 0;
+      if (un < nrows) {
+        nval = *reinterpret_cast<const uint4*>(stg + un * 256 + ((cidx ^ (un & 7)) << 4));
+        njs = srun[un];
+        nje = srun[un + 1];
+      }
+      for (int j = js + hw; j < je; j += 2) {
         const int drow = P.paged ? __ldg(P.dst_row + j) : j;
         if (drow >= 0)
           __stcs(reinterpret_cast<uint4*>(out_lc + static_cast<int64_t>(drow) * P.d_r + ocol0 +
                                           pc0 + cidx * kPerChunk),
                  val);
       }
+      u = un;
+      val = nval;
+      js = njs;
+      je = nje;
     }
     named_barrier_sync(1, kEpiThreads);
   }
@@ -772,13 +805,14 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
           sUpos[i] = i < nrows ? P.upos[u0 + i] : 0;
         }
         named_barrier_sync(1, kEpiThreads);
-        // this warp's receiver rows [wjb, wje); lane slot ps takes rows wjb+ps, +8, ...
+        // this warp's receiver rows [wjb, wje); lane slot ps walks the
+        // consecutive rows [ljb, lje) of them
         const int jb = sRun[0], je = sRun[nrows];
         const int per = (je - jb + kEpiWarps - 1) / kEpiWarps;
         const int wjb = min(je, jb + e * per), wje = min(je, wjb + per);
-        const int n_it = (wje - wjb + 7) >> 3;
-        const int j0 = wjb + ps;
-        const int ustart = j0 < wje ? find_row(sRun, nrows, j0) : 0;
+        const int per_slot = (wje - wjb + 7) >> 3;
+        const int ljb = min(wje, wjb + ps * per_slot), lje = min(wje, ljb + per_slot);
+        const int ustart = ljb < lje ? find_row(sRun, nrows, ljb) : 0;
         const float inv_r = P.inv_r[lc];
         const float* bias = P.bias + static_cast<int64_t>(lc) * P.d_r;
         const bool do_rope = P.rope && c == 0;
@@ -845,28 +879,16 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
             }
             named_barrier_sync(1, kEpiThreads);
             // step 2: rows of this warp's slice, both heads of the pair
-            float f[4], C8[4], S8[4];
+            float f[4], C1[4], S1[4];
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
               f[k] = do_rope ? __ldg(P.inv_freq + q + 4 * qq + k) : 0.f;
-              C8[k] = 1.f;
-              S8[k] = 0.f;
-              if (do_rope) rope_sincos(8, f[k], &S8[k], &C8[k]);  // one step = eight rows
+              C1[k] = 1.f;
+              S1[k] = 0.f;
+              if (do_rope) rope_sincos(1, f[k], &S1[k], &C1[k]);  // one step = one row
             }
-            Walk wk;
-            wk.u = ustart;
-            wk.expect = INT_MIN;
-#pragma unroll
-            for (int k = 0; k < 4; ++k) {
-              wk.cs[k] = 1.f;
-              wk.sn[k] = 0.f;
-            }
-            for (int it = 0; it < n_it; ++it) {
-              const int j = j0 + 8 * it;
-              if (j < wje)
-                walk_step<T>(wk, j, it, sRun, sUpos, sStg, qq, two_heads, do_rope, f, C8, S8, P,
-                             out_lc, ocol_pair, q, half);
-            }
+            walk_rows<T>(ljb, lje, ustart, sRun, sUpos, sStg, qq, two_heads, do_rope, f, C1, S1, P,
+                         out_lc, ocol_pair, q, half);
             named_barrier_sync(1, kEpiThreads);
           }
         }
