@@ -202,7 +202,14 @@ __device__ __forceinline__ void walk_rows(int jb, int je, int u, const int32_t* 
   int expect = INT_MIN;  // position for which cs/sn are valid
   float cs[4] = {1.f, 1.f, 1.f, 1.f}, sn[4] = {0.f, 0.f, 0.f, 0.f};
   --u;
+  int dnext = P.paged ? __ldg(P.dst_row + jb) : jb;  // destination of row j, read a row ahead
   for (int j = jb; j < je; ++j) {
+    const int drow = dnext;
+    if (P.paged) {
+      if (j + 1 < je) dnext = __ldg(P.dst_row + j + 1);
+    } else {
+      dnext = j + 1;
+    }
     if (j >= uend) {  // first row, or the first row of a later run
       do {
         ++u;
@@ -218,7 +225,6 @@ __device__ __forceinline__ void walk_rows(int jb, int je, int u, const int32_t* 
         b1 = *reinterpret_cast<const float4*>(urow + 32 + (((4 + qq) ^ sw) << 2));
       }
     }
-    const int drow = P.paged ? __ldg(P.dst_row + j) : j;
     float4 x0 = a0, y0 = b0, x1 = a1, y1 = b1;
     if (do_rope) {
       const int p = pb + j;
@@ -845,6 +851,11 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
             rn = rsqrtf(ss / static_cast<float>(D) + P.knorm_eps);
           }
           for (int q = 0; q < half; q += 16) {
+            // this lane's four frequencies, loaded before step 1 so that the
+            // global read overlaps the staging
+            float f[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) f[k] = do_rope ? __ldg(P.inv_freq + q + 4 * qq + k) : 0.f;
             if (stages_head) {
               // step 1: pairs q..q+15 of head 2*hp+g for this warp's 32 rows
               uint32_t v[32];
@@ -879,10 +890,9 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
             }
             named_barrier_sync(1, kEpiThreads);
             // step 2: rows of this warp's slice, both heads of the pair
-            float f[4], C1[4], S1[4];
+            float C1[4], S1[4];
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
-              f[k] = do_rope ? __ldg(P.inv_freq + q + 4 * qq + k) : 0.f;
               C1[k] = 1.f;
               S1[k] = 0.f;
               if (do_rope) rope_sincos(1, f[k], &S1[k], &C1[k]);  // one step = one row
