@@ -2,9 +2,10 @@
 
 Each translation unit compiles in its own nvcc process, in parallel, then
 one nvcc call links the shared library.  The CUDA runtime is linked
-statically and the driver's tensor-map encoder is fetched at run time, so
-the library loads on a machine without a GPU driver (symbols can be
-inspected there; calls then fail with HF_ERR_CUDA).
+statically, cuBLAS dynamically (from the toolkit, found through an rpath),
+and the driver's tensor-map encoder is fetched at run time, so the library
+loads on a machine without a GPU driver (symbols can be inspected there;
+calls then fail with HF_ERR_CUDA).
 """
 
 from __future__ import annotations
@@ -51,6 +52,12 @@ def _stale(target: str, deps) -> bool:
     return any(os.path.getmtime(d) > t for d in deps)
 
 
+def _link_libs(exe: str):
+    """cuBLAS (hf_recolor_fit's products), found beside the toolkit's nvcc."""
+    lib = os.path.join(os.path.dirname(os.path.dirname(os.path.realpath(exe))), "lib64")
+    return ["-L" + lib, "-lcublas", "-Xlinker", "-rpath=" + lib]
+
+
 def build(verbose: bool = False, force: bool = False, ptxas_info: bool = False) -> str:
     os.makedirs(BUILD_DIR, exist_ok=True)
     headers = [os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith((".h", ".cuh"))]
@@ -76,7 +83,7 @@ def build(verbose: bool = False, force: bool = False, ptxas_info: bool = False) 
             sys.stdout.write(out)
     if force or jobs or _stale(LIB_PATH, objs):
         tmp = LIB_PATH + ".tmp"
-        _run([exe, *ARCH, "-shared", "-o", tmp, *objs])
+        _run([exe, *ARCH, "-shared", "-o", tmp, *objs, *_link_libs(exe)])
         os.replace(tmp, LIB_PATH)
     return LIB_PATH
 

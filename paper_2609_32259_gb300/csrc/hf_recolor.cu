@@ -10,13 +10,18 @@
 // Z_0 = I into (S / c)^{1/2} and (S / c)^{-1/2}; X <- X (3I - X^T X) / 2
 // turns X_0 = M / |M|_F into the orthogonal polar factor U Q^T of
 // M = U Lambda Q^T (full column rank), which is the R* of Eq. 4.
-// Offline (once per map, before folding); fp32 products on the CUDA cores.
+// Offline (once per map, before folding).  The products are plain fp32
+// GEMMs and go to cuBLAS with fp32 emulated on the bf16 tensor cores (each
+// operand split into three bf16 parts, fp32 accumulation: fp32 accuracy);
+// the statistics, centring and elementwise passes are this file's kernels.
 #include <algorithm>
 #include <cmath>
 #include <cstring>
+#include <mutex>
 #include <string>
 #include <utility>
 
+#include <cublas_v2.h>
 #include <cuda_bf16.h>
 
 #include "hf_internal.h"
@@ -24,78 +29,54 @@
 namespace hf {
 namespace {
 
-constexpr int kTM = 128, kTN = 128, kTK = 8;  // SGEMM block tile
-constexpr int kGemmThreads = 256;             // 16 x 16 threads, 8 x 8 outputs each
+constexpr int kMaxDevices = 64;
+std::mutex g_blas_mutex[kMaxDevices];
+cublasHandle_t g_blas[kMaxDevices] = {};
+
+hf_status blas_fail(cublasStatus_t st, const char* what) {
+  set_error(std::string("hf_recolor_fit: ") + what + " (cuBLAS status " +
+            std::to_string(static_cast<int>(st)) + ")");
+  return HF_ERR_CUDA;
+}
+
+// The current device's cuBLAS handle (created on first use, fp32 products
+// emulated on the tensor cores whenever possible).  Callers hold
+// g_blas_mutex[dev] while they use it.
+hf_status blas_handle(int dev, cublasHandle_t* out) {
+  if (!g_blas[dev]) {
+    cublasHandle_t h = nullptr;
+    cublasStatus_t st = cublasCreate(&h);
+    if (st != CUBLAS_STATUS_SUCCESS) return blas_fail(st, "cublasCreate");
+    st = cublasSetEmulationStrategy(h, CUBLAS_EMULATION_STRATEGY_EAGER);
+    if (st != CUBLAS_STATUS_SUCCESS) {
+      cublasDestroy(h);
+      return blas_fail(st, "cublasSetEmulationStrategy");
+    }
+    g_blas[dev] = h;
+  }
+  *out = g_blas[dev];
+  return HF_OK;
+}
 
 // C[M x N] = alpha * op(A) op(B) + beta * C, row-major C with leading
 // dimension ldc; op(A)(i, k) = A[i * a_i + k * a_k], op(B)(k, j) =
-// B[k * b_k + j * b_j] (strides express transposes).  Tiles of 128 x 128
-// with 8-deep k steps in shared memory; bounds-checked for any size.
-__global__ void __launch_bounds__(kGemmThreads) sgemm_kernel(
-    int M, int N, int K, float alpha, const float* __restrict__ A, int64_t a_i, int64_t a_k,
-    const float* __restrict__ B, int64_t b_k, int64_t b_j, float beta, float* C, int64_t ldc) {
-  __shared__ float As[kTK][kTM];
-  __shared__ float Bs[kTK][kTN];
-  const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;
-  const int i0 = blockIdx.y * kTM, j0 = blockIdx.x * kTN;
-  float acc[8][8];
-#pragma unroll
-  for (int a = 0; a < 8; ++a)
-#pragma unroll
-    for (int b = 0; b < 8; ++b) acc[a][b] = 0.f;
-  // loaders: the 1024 elements of each tile, 4 per thread; the tile index
-  // runs fastest along the operand's contiguous dimension
-  const bool a_kfast = a_k == 1, b_jfast = b_j == 1;
-  for (int k0 = 0; k0 < K; k0 += kTK) {
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      const int idx = threadIdx.x + e * kGemmThreads;
-      int ii, kk;
-      if (a_kfast) { ii = idx / kTK; kk = idx % kTK; } else { kk = idx / kTM; ii = idx % kTM; }
-      const int gi = i0 + ii, gk = k0 + kk;
-      As[kk][ii] = (gi < M && gk < K) ? A[gi * a_i + gk * a_k] : 0.f;
-      int jj, kb;
-      if (b_jfast) { kb = idx / kTN; jj = idx % kTN; } else { jj = idx / kTK; kb = idx % kTK; }
-      const int gj = j0 + jj, gk2 = k0 + kb;
-      Bs[kb][jj] = (gj < N && gk2 < K) ? B[gk2 * b_k + gj * b_j] : 0.f;
-    }
-    __syncthreads();
-#pragma unroll
-    for (int kk = 0; kk < kTK; ++kk) {
-      float a[8], b[8];
-#pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        a[q] = As[kk][ty * 8 + q];
-        b[q] = Bs[kk][tx * 8 + q];
-      }
-#pragma unroll
-      for (int p = 0; p < 8; ++p)
-#pragma unroll
-        for (int q = 0; q < 8; ++q) acc[p][q] = fmaf(a[p], b[q], acc[p][q]);
-    }
-    __syncthreads();
-  }
-#pragma unroll
-  for (int p = 0; p < 8; ++p) {
-    const int gi = i0 + ty * 8 + p;
-    if (gi >= M) continue;
-#pragma unroll
-    for (int q = 0; q < 8; ++q) {
-      const int gj = j0 + tx * 8 + q;
-      if (gj >= N) continue;
-      float* c = C + gi * ldc + gj;
-      *c = beta == 0.f ? alpha * acc[p][q] : fmaf(alpha, acc[p][q], beta * *c);
-    }
-  }
-}
-
-hf_status sgemm(cudaStream_t s, int M, int N, int K, float alpha, const float* A, int64_t a_i,
+// B[k * b_k + j * b_j], one of each operand's two strides being 1 (strides
+// express transposes).  cuBLAS is column-major: the row-major C is the
+// column-major C^T = op(B)^T op(A)^T, so B goes first.
+hf_status sgemm(cublasHandle_t h, int M, int N, int K, float alpha, const float* A, int64_t a_i,
                 int64_t a_k, const float* B, int64_t b_k, int64_t b_j, float beta, float* C,
                 int64_t ldc) {
-  dim3 grid((N + kTN - 1) / kTN, (M + kTM - 1) / kTM);
-  sgemm_kernel<<<grid, kGemmThreads, 0, s>>>(M, N, K, alpha, A, a_i, a_k, B, b_k, b_j, beta, C,
-                                             ldc);
-  HF_CUDA_TRY(cudaGetLastError(), "hf_recolor_fit: product launch");
+  // op(B)^T (N x K): column-major B with ld b_k when b_j == 1, else B^T
+  const cublasOperation_t tb = b_j == 1 ? CUBLAS_OP_N : CUBLAS_OP_T;
+  const int64_t ldb = b_j == 1 ? b_k : b_j;
+  // op(A)^T (K x M): column-major A with ld a_i when a_k == 1, else A^T
+  const cublasOperation_t ta = a_k == 1 ? CUBLAS_OP_N : CUBLAS_OP_T;
+  const int64_t lda = a_k == 1 ? a_i : a_k;
+  const cublasStatus_t st =
+      cublasGemmEx(h, tb, ta, N, M, K, &alpha, B, CUDA_R_32F, static_cast<int>(ldb), A,
+                   CUDA_R_32F, static_cast<int>(lda), &beta, C, CUDA_R_32F, static_cast<int>(ldc),
+                   CUBLAS_COMPUTE_32F_EMULATED_16BFX9, CUBLAS_GEMM_DEFAULT);
+  if (st != CUBLAS_STATUS_SUCCESS) return blas_fail(st, "product");
   return HF_OK;
 }
 
@@ -268,7 +249,7 @@ bool converged(double e, double* prev) {
 
 // Newton-Schulz square root and inverse square root of the SPD matrix S
 // (d x d): root = S^{1/2}, inv_root = S^{-1/2}.  Y, Z, T, U are d x d work.
-hf_status ns_sqrt(cudaStream_t s, const float* S, int d, float* Y, float* Z, float* T, float* U,
+hf_status ns_sqrt(cudaStream_t s, cublasHandle_t h, const float* S, int d, float* Y, float* Z, float* T, float* U,
                   float* root, float* inv_root, double* dscr, int* iters) {
   const int64_t n_el = static_cast<int64_t>(d) * d;
   const int grid = 1024;
@@ -289,7 +270,7 @@ hf_status ns_sqrt(cudaStream_t s, const float* S, int d, float* Y, float* Z, flo
   for (; it < kMaxIter; ++it) {
     // T = 1.5 I - 0.5 Z Y
     rc_affine_kernel<<<grid, 256, 0, s>>>(T, nullptr, n_el, d, 0.f, 1.5f);
-    if ((st = sgemm(s, d, d, d, -0.5f, Z, d, 1, Y, d, 1, 1.f, T, d)) != HF_OK) return st;
+    if ((st = sgemm(h, d, d, d, -0.5f, Z, d, 1, Y, d, 1, 1.f, T, d)) != HF_OK) return st;
     if (it % 4 == 3) {
       double e2 = 0.0;
       HF_CUDA_TRY(cudaMemsetAsync(dscr, 0, sizeof(double), s), "clear");
@@ -298,9 +279,9 @@ hf_status ns_sqrt(cudaStream_t s, const float* S, int d, float* Y, float* Z, flo
       if ((st = read_double(s, dscr, &e2)) != HF_OK) return st;
       if (converged(2.0 * sqrt(e2 / d), &prev)) break;
     }
-    if ((st = sgemm(s, d, d, d, 1.f, Y, d, 1, T, d, 1, 0.f, U, d)) != HF_OK) return st;  // Y T
+    if ((st = sgemm(h, d, d, d, 1.f, Y, d, 1, T, d, 1, 0.f, U, d)) != HF_OK) return st;  // Y T
     std::swap(Y, U);
-    if ((st = sgemm(s, d, d, d, 1.f, T, d, 1, Z, d, 1, 0.f, U, d)) != HF_OK) return st;  // T Z
+    if ((st = sgemm(h, d, d, d, 1.f, T, d, 1, Z, d, 1, 0.f, U, d)) != HF_OK) return st;  // T Z
     std::swap(Z, U);
   }
   *iters = it;
@@ -314,7 +295,7 @@ hf_status ns_sqrt(cudaStream_t s, const float* S, int d, float* Y, float* Z, flo
 // Orthogonal polar factor of M (dx x dy, dx >= dy, full column rank):
 // X <- X (3I - X^T X) / 2 from X_0 = M / |M|_F.  Result in *out (one of the
 // two buffers).
-hf_status ns_polar(cudaStream_t s, const float* M, int dx, int dy, float* X, float* X2,
+hf_status ns_polar(cudaStream_t s, cublasHandle_t h, const float* M, int dx, int dy, float* X, float* X2,
                    float* P, double* dscr, float** out, int* iters) {
   const int64_t n_el = static_cast<int64_t>(dx) * dy, p_el = static_cast<int64_t>(dy) * dy;
   const int grid = 1024;
@@ -332,7 +313,7 @@ hf_status ns_polar(cudaStream_t s, const float* M, int dx, int dy, float* X, flo
   double prev = 1e30;
   for (; it < kMaxIter; ++it) {
     // P = X^T X
-    if ((st = sgemm(s, dy, dy, dx, 1.f, X, 1, dy, X, dy, 1, 0.f, P, dy)) != HF_OK) return st;
+    if ((st = sgemm(h, dy, dy, dx, 1.f, X, 1, dy, X, dy, 1, 0.f, P, dy)) != HF_OK) return st;
     if (it % 4 == 3) {
       double e2 = 0.0;
       HF_CUDA_TRY(cudaMemsetAsync(dscr, 0, sizeof(double), s), "clear");
@@ -342,7 +323,7 @@ hf_status ns_polar(cudaStream_t s, const float* M, int dx, int dy, float* X, flo
     }
     // X2 = 1.5 X - 0.5 X P
     rc_affine_kernel<<<grid, 256, 0, s>>>(X2, X, n_el, dy, 1.5f, 0.f);
-    if ((st = sgemm(s, dx, dy, dy, -0.5f, X, dy, 1, P, dy, 1, 1.f, X2, dy)) != HF_OK) return st;
+    if ((st = sgemm(h, dx, dy, dy, -0.5f, X, dy, 1, P, dy, 1, 1.f, X2, dy)) != HF_OK) return st;
     std::swap(X, X2);
   }
   *iters = it;
@@ -354,7 +335,7 @@ hf_status ns_polar(cudaStream_t s, const float* M, int dx, int dy, float* X, flo
 template <typename T>
 hf_status recolor_typed(int64_t N, int dx, int dy, const void* Xv, const void* Yv, const float* w,
                         float reg, void* W_out, float* b_out, float* h_r, int32_t* h_iters,
-                        char* ws, cudaStream_t s) {
+                        char* ws, cudaStream_t s, cublasHandle_t h) {
   const Rc L = rc_layout(N, dx, dy);
   double* stats = reinterpret_cast<double*>(ws + L.stats);
   double* sx = stats;
@@ -374,43 +355,43 @@ hf_status recolor_typed(int64_t N, int dx, int dy, const void* Xv, const void* Y
   HF_CUDA_TRY(cudaGetLastError(), "hf_recolor_fit: moments launch");
   hf_status st;
   // Sigma_Z = Xc^T Xc, Sigma_Y = Yc^T Yc, Sigma_ZY = Xc^T Yc
-  if ((st = sgemm(s, dx, dx, N, 1.f, F(L.xc), 1, dx, F(L.xc), dx, 1, 0.f, F(L.sz), dx)) != HF_OK)
+  if ((st = sgemm(h, dx, dx, N, 1.f, F(L.xc), 1, dx, F(L.xc), dx, 1, 0.f, F(L.sz), dx)) != HF_OK)
     return st;
-  if ((st = sgemm(s, dy, dy, N, 1.f, F(L.yc), 1, dy, F(L.yc), dy, 1, 0.f, F(L.sy), dy)) != HF_OK)
+  if ((st = sgemm(h, dy, dy, N, 1.f, F(L.yc), 1, dy, F(L.yc), dy, 1, 0.f, F(L.sy), dy)) != HF_OK)
     return st;
-  if ((st = sgemm(s, dx, dy, N, 1.f, F(L.xc), 1, dx, F(L.yc), dy, 1, 0.f, F(L.szy), dy)) != HF_OK)
+  if ((st = sgemm(h, dx, dy, N, 1.f, F(L.xc), 1, dx, F(L.yc), dy, 1, 0.f, F(L.szy), dy)) != HF_OK)
     return st;
   if (reg > 0.f) {
     rc_ridge_kernel<<<1, 256, 0, s>>>(F(L.sz), dx, reg);
     rc_ridge_kernel<<<1, 256, 0, s>>>(F(L.sy), dy, reg);
   }
   int it1 = 0, it2 = 0, it3 = 0;
-  if ((st = ns_sqrt(s, F(L.sz), dx, F(L.p1), F(L.p2), F(L.p3), F(L.p4), F(L.p4) /*unused root*/,
+  if ((st = ns_sqrt(s, h, F(L.sz), dx, F(L.p1), F(L.p2), F(L.p3), F(L.p4), F(L.p4) /*unused root*/,
                     F(L.sz_ih), dscr, &it1)) != HF_OK)
     return st;
-  if ((st = ns_sqrt(s, F(L.sy), dy, F(L.p1), F(L.p2), F(L.p3), F(L.p4), F(L.sy_h), F(L.sy_ih),
+  if ((st = ns_sqrt(s, h, F(L.sy), dy, F(L.p1), F(L.p2), F(L.p3), F(L.p4), F(L.sy_h), F(L.sy_ih),
                     dscr, &it2)) != HF_OK)
     return st;
   // M = Sigma_Z^{-1/2} Sigma_ZY Sigma_Y^{-1/2}
-  if ((st = sgemm(s, dx, dy, dx, 1.f, F(L.sz_ih), dx, 1, F(L.szy), dy, 1, 0.f, F(L.x2), dy)) != HF_OK)
+  if ((st = sgemm(h, dx, dy, dx, 1.f, F(L.sz_ih), dx, 1, F(L.szy), dy, 1, 0.f, F(L.x2), dy)) != HF_OK)
     return st;
-  if ((st = sgemm(s, dx, dy, dy, 1.f, F(L.x2), dy, 1, F(L.sy_ih), dy, 1, 0.f, F(L.m), dy)) != HF_OK)
+  if ((st = sgemm(h, dx, dy, dy, 1.f, F(L.x2), dy, 1, F(L.sy_ih), dy, 1, 0.f, F(L.m), dy)) != HF_OK)
     return st;
   float* R = nullptr;
-  if ((st = ns_polar(s, F(L.m), dx, dy, F(L.x1), F(L.x2), F(L.xtx), dscr, &R, &it3)) != HF_OK)
+  if ((st = ns_polar(s, h, F(L.m), dx, dy, F(L.x1), F(L.x2), F(L.xtx), dscr, &R, &it3)) != HF_OK)
     return st;
   // A = Sigma_Z^{-1/2} R* Sigma_Y^{1/2}
   float* tmp = R == F(L.x1) ? F(L.x2) : F(L.x1);
-  if ((st = sgemm(s, dx, dy, dx, 1.f, F(L.sz_ih), dx, 1, R, dy, 1, 0.f, tmp, dy)) != HF_OK) return st;
-  if ((st = sgemm(s, dx, dy, dy, 1.f, tmp, dy, 1, F(L.sy_h), dy, 1, 0.f, F(L.a), dy)) != HF_OK)
+  if ((st = sgemm(h, dx, dy, dx, 1.f, F(L.sz_ih), dx, 1, R, dy, 1, 0.f, tmp, dy)) != HF_OK) return st;
+  if ((st = sgemm(h, dx, dy, dy, 1.f, tmp, dy, 1, F(L.sy_h), dy, 1, 0.f, F(L.a), dy)) != HF_OK)
     return st;
   rc_output_kernel<T><<<1024, 256, 0, s>>>(F(L.a), dx, dy, sx, sy, sw_ss, static_cast<T*>(W_out),
                                            b_out);
   HF_CUDA_TRY(cudaGetLastError(), "hf_recolor_fit: output launch");
-  double h[2];
-  HF_CUDA_TRY(cudaMemcpyAsync(h, sw_ss, sizeof(h), cudaMemcpyDeviceToHost, s), "read back");
+  double hs[2];
+  HF_CUDA_TRY(cudaMemcpyAsync(hs, sw_ss, sizeof(hs), cudaMemcpyDeviceToHost, s), "read back");
   HF_CUDA_TRY(cudaStreamSynchronize(s), "synchronize");
-  if (h_r) *h_r = static_cast<float>(std::sqrt(h[1] / (static_cast<double>(dx) * h[0])));
+  if (h_r) *h_r = static_cast<float>(std::sqrt(hs[1] / (static_cast<double>(dx) * hs[0])));
   if (h_iters) {
     h_iters[0] = it1;
     h_iters[1] = it2;
@@ -463,9 +444,23 @@ extern "C" hf_status hf_recolor_fit(hf_dtype dtype, int64_t N, int32_t d_S, int3
   }
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream_);
   char* ws = static_cast<char*>(d_workspace);
+  int dev = 0;
+  HF_CUDA_TRY(cudaGetDevice(&dev), "hf_recolor_fit: current device");
+  if (dev < 0 || dev >= kMaxDevices) {
+    set_error("hf_recolor_fit: device ordinal out of range");
+    return HF_ERR_UNSUPPORTED;
+  }
+  // one fit at a time per device uses the device's handle (the call is
+  // synchronous: it waits for its convergence checks)
+  std::lock_guard<std::mutex> lock(g_blas_mutex[dev]);
+  cublasHandle_t h = nullptr;
+  hf_status st = blas_handle(dev, &h);
+  if (st != HF_OK) return st;
+  const cublasStatus_t bs = cublasSetStream(h, s);
+  if (bs != CUBLAS_STATUS_SUCCESS) return blas_fail(bs, "cublasSetStream");
   if (dtype == HF_BF16)
     return recolor_typed<__nv_bfloat16>(N, d_S, d_R, d_X, d_Y, d_w, reg, d_W_out, d_b_out,
-                                        h_r_out, h_iters_out, ws, s);
+                                        h_r_out, h_iters_out, ws, s, h);
   return recolor_typed<float>(N, d_S, d_R, d_X, d_Y, d_w, reg, d_W_out, d_b_out, h_r_out,
-                              h_iters_out, ws, s);
+                              h_iters_out, ws, s, h);
 }
