@@ -99,27 +99,6 @@ __device__ __forceinline__ void tma_prefetch_map(const void* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(map) : "memory");
 }
 
-// 2-D tiled load of box (x, y) .. (x + box0, y + box1) into shared memory.
-__device__ __forceinline__ void tma_load_2d(uint32_t dst, const void* map, int32_t x, int32_t y,
-                                            uint32_t bar) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
-      "l"(map), "r"(x), "r"(y), "r"(bar)
-      : "memory");
-}
-
-// Gathers four rows (r0..r3) of a 2-D tensor, columns [x, x + box0), into
-// four consecutive box rows of shared memory.  The map's box is one row high.
-__device__ __forceinline__ void tma_gather4(uint32_t dst, const void* map, int32_t x, int32_t r0,
-                                            int32_t r1, int32_t r2, int32_t r3, uint32_t bar) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cta.global.tile::gather4.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%2, %3, %4, %5, %6}], [%7];" ::"r"(dst),
-      "l"(map), "r"(x), "r"(r0), "r"(r1), "r"(r2), "r"(r3), "r"(bar)
-      : "memory");
-}
-
 // ---------------------------------------------------------------------------
 // Thread-block clusters (a CTA pair sharing one tcgen05 MMA)
 // ---------------------------------------------------------------------------
@@ -174,14 +153,24 @@ __device__ __forceinline__ void mbar_arrive_expect_tx_cluster(uint32_t cluster_a
                : "memory");
 }
 
+// An L2 policy that keeps the lines a load brings in ahead of normal lines
+// when L2 evicts (for data that other CTAs read again soon).
+__device__ __forceinline__ uint64_t l2_policy_evict_last() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+
 // 2-D tiled load into this CTA's shared memory, completing on an mbarrier
-// that may be in the peer CTA of the pair (cluster address).
-__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const void* map, int32_t x, int32_t y,
-                                                 uint32_t bar_cluster) {
+// that may be in the peer CTA of the pair (cluster address), with an L2
+// cache policy for the loaded lines.
+__device__ __forceinline__ void tma_load_2d_pair_hint(uint32_t dst, const void* map, int32_t x,
+                                                      int32_t y, uint32_t bar_cluster,
+                                                      uint64_t policy) {
   asm volatile(
       "cp.async.bulk.tensor.2d.shared::cta.global.tile.mbarrier::complete_tx::bytes.cta_group::2"
-      " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
-      "l"(map), "r"(x), "r"(y), "r"(bar_cluster)
+      ".L2::cache_hint [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
+      "l"(map), "r"(x), "r"(y), "r"(bar_cluster), "l"(policy)
       : "memory");
 }
 

@@ -176,6 +176,13 @@ EDGE = {
         W.llama_to_ministral(400).with_(L_s=6, L_r=3), n_seg=3, n_terms=1, unit=True),
     "rope_table": lambda: W.llama_to_ministral(600).with_(L_s=4, L_r=3, rope_table=True,
                                                           r_pos0=(5000,)),
+    # long runs: coarse sender tokens and fine receiver tokens, so one
+    # distinct row covers ~10 receiver rows and a lane walks ~20 rows of a
+    # tile (angles carried across runs and re-anchored every 16 rows)
+    "long_runs": lambda: W.llama_to_ministral(3000).with_(L_s=4, L_r=3, mean_s=12.0, mean_r=1.2,
+                                                           r_pos0=(3000,)),
+    "long_runs_batched_paged": lambda: W.qwen25_to_llama_batched(
+        n_req=3, lo=300, hi=900, seed=21).with_(L_s=3, L_r=3, mean_s=12.0, mean_r=1.5),
     # message spans after a context (only the span's K/V is mapped)
     "message_spans_batched_paged": lambda: W.qwen25_to_llama_batched(
         n_req=3, lo=40, hi=160, seed=12).with_(L_s=4, L_r=3, span_gap=700),
