@@ -22,21 +22,44 @@ struct ScanMax {
   __device__ __forceinline__ int operator()(int a, int b) const { return a > b ? a : b; }
 };
 
+// Loads this thread's kScanItems consecutive items at i0 (identity past n):
+// two 16-byte loads when the tile is whole and the array is 16-byte aligned.
+template <typename Op>
+__device__ __forceinline__ void scan_load(const int* data, int64_t n, int64_t i0, bool vec,
+                                          int* v) {
+  if (vec && i0 + kScanItems <= n) {
+    const int4 a = *reinterpret_cast<const int4*>(data + i0);
+    const int4 b = *reinterpret_cast<const int4*>(data + i0 + 4);
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+    v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+  } else {
+#pragma unroll
+    for (int i = 0; i < kScanItems; ++i) v[i] = (i0 + i < n) ? data[i0 + i] : Op::identity();
+  }
+}
+
 // data[i] <- op(data[0..i]) for i < n, in tiles of 1024 x 8 items carried
-// across tiles.  *total (if not null) receives op over all n items (the
-// identity when n == 0).  Launch with one block of kScanThreads threads.
+// across tiles; the next tile's items are loaded while the current one is
+// scanned.  *total (if not null) receives op over all n items (the identity
+// when n == 0).  Launch with one block of kScanThreads threads.
 template <typename Op>
 __global__ void __launch_bounds__(kScanThreads) scan_inplace_kernel(int* data, int64_t n,
                                                                     int* total) {
+  static_assert(kScanItems == 8, "scan_load reads two int4 per thread");
   __shared__ int warp_incl[kScanThreads / 32];
   const Op op;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const bool vec = (reinterpret_cast<uintptr_t>(data) & 15u) == 0;
+  constexpr int64_t kTile = (int64_t)kScanThreads * kScanItems;
   int carry = Op::identity();
-  for (int64_t base = 0; base < n; base += (int64_t)kScanThreads * kScanItems) {
+  int nv[kScanItems];
+  if (n > 0) scan_load<Op>(data, n, (int64_t)tid * kScanItems, vec, nv);
+  for (int64_t base = 0; base < n; base += kTile) {
     int v[kScanItems];
-    const int64_t i0 = base + (int64_t)tid * kScanItems;
 #pragma unroll
-    for (int i = 0; i < kScanItems; ++i) v[i] = (i0 + i < n) ? data[i0 + i] : Op::identity();
+    for (int i = 0; i < kScanItems; ++i) v[i] = nv[i];
+    const int64_t i0 = base + (int64_t)tid * kScanItems;
+    if (base + kTile < n) scan_load<Op>(data, n, i0 + kTile, vec, nv);
 #pragma unroll
     for (int i = 1; i < kScanItems; ++i) v[i] = op(v[i - 1], v[i]);
     // inclusive scan of the per-thread totals within the warp
@@ -62,9 +85,16 @@ __global__ void __launch_bounds__(kScanThreads) scan_inplace_kernel(int* data, i
     __syncthreads();
     const int warp_excl = warp > 0 ? warp_incl[warp - 1] : Op::identity();
     const int excl = op(carry, op(warp_excl, lane_excl));
+    if (vec && i0 + kScanItems <= n) {
+      *reinterpret_cast<int4*>(data + i0) =
+          make_int4(op(excl, v[0]), op(excl, v[1]), op(excl, v[2]), op(excl, v[3]));
+      *reinterpret_cast<int4*>(data + i0 + 4) =
+          make_int4(op(excl, v[4]), op(excl, v[5]), op(excl, v[6]), op(excl, v[7]));
+    } else {
 #pragma unroll
-    for (int i = 0; i < kScanItems; ++i)
-      if (i0 + i < n) data[i0 + i] = op(excl, v[i]);
+      for (int i = 0; i < kScanItems; ++i)
+        if (i0 + i < n) data[i0 + i] = op(excl, v[i]);
+    }
     carry = op(carry, warp_incl[31]);
     __syncthreads();
   }
