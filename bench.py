@@ -116,7 +116,7 @@ class ClockSampler:
         except subprocess.TimeoutExpired:
             self.proc.kill()
             out, _ = self.proc.communicate()
-        sm, mx, reasons = [], [], set()
+        sm, mx, pw, reasons = [], [], [], set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         for line in out.strip().splitlines():
             f = [x.strip() for x in line.split(",")]
@@ -127,12 +127,17 @@ class ClockSampler:
                 mx.append(float(f[2]))
             except ValueError:
                 continue
+            try:
+                pw.append(float(f[3]))
+            except ValueError:
+                pass
             for n, v in zip(names, f[5:9]):
                 if v.lower().startswith("active"):
                     reasons.add(n)
         if not sm:
             return None
-        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx),
+        return {"sm_mhz": statistics.median(sm), "sm_min_mhz": min(sm), "sm_max_mhz": max(mx),
+                "power_w_median": statistics.median(pw) if pw else None,
                 "reasons": sorted(reasons), "samples": len(sm)}
 
 
@@ -341,7 +346,14 @@ def run_ours(args):
     clk = clocks.stop()
     step_ms = (t_start.elapsed_time(t_end) / args.steps if flush is None
                else statistics.mean(a.elapsed_time(bb) for a, bb in st))
-    kern_ms = statistics.mean(a.elapsed_time(bb) for a, bb in ev)
+    kern_all = [a.elapsed_time(bb) for a, bb in ev]
+    kern_ms = statistics.mean(kern_all)
+    # spread of the kernel time over the run (a power cap shows as later
+    # steps slower than the first ones)
+    q = sorted(kern_all)
+    kern_spread = {"p10": q[len(q) // 10], "p50": q[len(q) // 2], "p90": q[(9 * len(q)) // 10],
+                   "first_tenth_mean": statistics.mean(kern_all[:max(1, len(q) // 10)]),
+                   "last_tenth_mean": statistics.mean(kern_all[-max(1, len(q) // 10):])}
     value, (step_ms, kern_ms) = aggregate([step_ms, kern_ms], tok.T_r, world)
 
     # end to end through the API with host buffers
@@ -419,7 +431,8 @@ def run_ours(args):
                 "unit": "GB/s", "frac": (bytes_ / t_k / 1e9) / hbm_gbs}
     roof.update({"traffic": None, "peak_source": src, "kernel": "transfer_kernel",
                  "frac_of_sustained_peak": (flops / t_k / 1e12) / tflops_sust,
-                 "kernel_ms": kern_ms, "flop_alg": flops, "bytes_alg": bytes_,
+                 "kernel_ms": kern_ms, "kernel_ms_spread": kern_spread,
+                 "flop_alg": flops, "bytes_alg": bytes_,
                  "hbm_achieved_gbs": bytes_ / t_k / 1e9,
                  "tensor_achieved_tflops": flops / t_k / 1e12,
                  "roofline_ms": max(t_tensor, t_hbm) * 1e3})
