@@ -381,9 +381,12 @@ hf_status hf_fold(hf_dtype dtype, int32_t n_maps, int32_t d_R, int64_t K, int32_
  *       roots of Sigma_Z and Sigma_Y and by the polar factor.
  * d_workspace: hf_recolor_workspace_size bytes, 256-byte aligned.
  * Requires d_S >= d_R and N * d_S < 2^31.  Matrix roots and the polar
- * factor use Newton-Schulz iterations in fp32; the call synchronises
- * `stream` (convergence checks) and returns HF_ERR_DEVICE_CHECK if an
- * iteration does not converge (raise reg).
+ * factor use Newton-Schulz iterations in fp32; the matrix products go to
+ * cuBLAS with fp32 emulated on the tensor cores (fp32 accuracy), through a
+ * per-device handle created on the first call (calls on one device are
+ * serialised).  The call synchronises `stream` (convergence checks) and
+ * returns HF_ERR_DEVICE_CHECK if an iteration does not converge (raise
+ * reg), HF_ERR_CUDA if cuBLAS fails.
  */
 hf_status hf_recolor_workspace_size(int64_t N, int32_t d_S, int32_t d_R, size_t* bytes);
 hf_status hf_recolor_fit(hf_dtype dtype, int64_t N, int32_t d_S, int32_t d_R, const void* d_X,
