@@ -48,7 +48,7 @@ constexpr int kEpiWarps = 10;            // epilogue: warps 2-11 (8 of them read
 constexpr int kBuilderWarps = 4;         // A tile builders: warps 12-15
 constexpr int kEpiThreads = 32 * kEpiWarps;
 constexpr int kThreads = 64 + kEpiThreads + 32 * kBuilderWarps;  // 16 warps
-constexpr int kAtoms = 2;                // 128-byte swizzle atoms (k-blocks) per pipeline stage
+constexpr int kAtoms = 2;                // 128-byte swizzle atoms (k-blocks) per A stage (a B stage holds one)
 constexpr int kAtomABytes = kBM * 128;   // 128 rows x 128 bytes
 constexpr int kStageABytes = kAtoms * kAtomABytes;
 constexpr int kStgFloats = kBM * 64;     // epilogue staging: 128 rows x 2 heads x 32
@@ -81,8 +81,8 @@ struct XferParams {
   int64_t recv_rows;  // receiver rows per (layer, role) in receiver_kv
   int L_r, d_s, d_r, D_r;
   int l0, n_l;  // receiver layers [l0, l0 + n_l) of this launch
-  int n_kb, atoms_per_seg, last_atoms, BN, n_tiles_n, groups;  // n_kb: stages per tile
-  int stages_a, stages_b, lag;  // A ring, B ring, cp.async groups in flight per loader
+  int n_kb, atoms_per_seg, last_atoms, BN, n_tiles_n, groups;  // n_kb: A stages per tile
+  int stages_a, stages_b, lag;  // A ring (stages), B ring (atoms), loader groups in flight
   int rope, paged, knorm, unrot, D_s;
   float knorm_eps;
   uint32_t idesc;
