@@ -397,6 +397,20 @@ hf_status hf_recolor_fit(hf_dtype dtype, int64_t N, int32_t d_S, int32_t d_R, co
 const char* hf_status_string(hf_status status);
 const char* hf_last_error(void);
 
+/*
+ * Test hook for the kernel's bounded waits (not part of the method).
+ * hf_debug_transfer_stalled launches hf_transfer's kernel with its map
+ * producer withholding the first map atom, so the tensor-core issuer's wait
+ * for it, and then every other role's wait, runs out: the launch ends after
+ * a few seconds (each wait gives up after 2 s) with HF_CHECK_TIMEOUT set in
+ * the plan's status word (hf_plan_device_status), instead of hanging, and
+ * the CUDA context stays usable.  receiver_kv's contents are unspecified
+ * afterwards; a plan created again starts with a clear status.  Arguments as
+ * hf_transfer; HF_ERR_INVALID_ARGUMENT for a plan without receiver tokens.
+ */
+hf_status hf_debug_transfer_stalled(hf_plan plan, const void* sender_kv, void* receiver_kv,
+                                    hf_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -38,7 +38,8 @@ CHECK_BITS = {
 EXPORTED = ("hf_align_build", "hf_plan_workspace_size", "hf_plan_create", "hf_transfer",
             "hf_plan_destroy", "hf_plan_device_status", "hf_plan_distinct_rows",
             "hf_status_string", "hf_last_error", "hf_transfer_noalloc", "hf_transfer_host",
-            "hf_transfer_batch", "hf_fold", "hf_recolor_workspace_size", "hf_recolor_fit")
+            "hf_transfer_batch", "hf_fold", "hf_recolor_workspace_size", "hf_recolor_fit",
+            "hf_debug_transfer_stalled")
 
 _p = ctypes.c_void_p
 _i32p = ctypes.POINTER(ctypes.c_int32)
@@ -92,6 +93,8 @@ def lib() -> ctypes.CDLL:
         L.hf_plan_create.argtypes = [ctypes.POINTER(PlanDesc), _p, ctypes.c_size_t, _p,
                                      ctypes.POINTER(ctypes.c_void_p)]
         L.hf_transfer.argtypes = [_p, _p, _p, _p]
+        L.hf_debug_transfer_stalled.argtypes = [_p, _p, _p, _p]
+        L.hf_debug_transfer_stalled.restype = ctypes.c_int
         L.hf_plan_destroy.argtypes = [_p]
         L.hf_plan_device_status.argtypes = [_p, _p, _i32p]
         L.hf_plan_distinct_rows.argtypes = [_p, _p, _i32p]
@@ -256,6 +259,13 @@ def plan_create(desc: Desc, workspace, stream=None) -> Plan:
 def transfer(plan: Plan, sender_kv, receiver_kv, stream=None) -> None:
     _check(lib().hf_transfer(plan.handle, _dptr(sender_kv), _dptr(receiver_kv), _stream(stream)),
            "hf_transfer")
+
+
+def debug_transfer_stalled(plan: Plan, sender_kv, receiver_kv, stream=None) -> None:
+    """Test hook: a transfer launch whose first map atom never arrives (the
+    bounded waits end it with HF_CHECK_TIMEOUT in the plan's status)."""
+    _check(lib().hf_debug_transfer_stalled(plan.handle, _dptr(sender_kv), _dptr(receiver_kv),
+                                           _stream(stream)), "hf_debug_transfer_stalled")
 
 
 def transfer_host(plan: Plan, h_sender_kv, d_sender_kv, d_receiver_kv, h_receiver_kv,

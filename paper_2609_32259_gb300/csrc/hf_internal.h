@@ -103,8 +103,10 @@ hf_status launch_plan_kernels(hf_plan_s* p, const PlanTables& tables, cudaStream
 hf_status plan_build(const hf_plan_desc* desc, void* d_workspace, size_t workspace_bytes,
                      cudaStream_t stream, hf_plan_s* p, PlanTables* t);
 // One transfer-kernel launch over receiver layers [l_begin, l_end) (l_end < 0: all).
+// stall (test hook): the map producer withholds its first atom, so the
+// launch ends through the bounded waits with HF_CHECK_TIMEOUT.
 hf_status launch_transfer(hf_plan_s* p, const void* sender, void* receiver, cudaStream_t stream,
-                          int l_begin = 0, int l_end = -1);
+                          int l_begin = 0, int l_end = -1, bool stall = false);
 // Several plans in one launch: they must share the dtype and the operand
 // path (batch_compatible); n <= kMaxBatch.
 bool batch_compatible(const hf_plan_s* const* plans, int n);

@@ -84,6 +84,7 @@ struct XferParams {
   int n_kb, atoms_per_seg, last_atoms, BN, n_tiles_n, groups;  // n_kb: A stages per tile
   int stages_a, stages_b, lag;  // A ring (stages), B ring (atoms), loader groups in flight
   int rope, paged, knorm, unrot, D_s;
+  int stall;  // test hook: the map producer withholds its first atom (hf_debug_transfer_stalled)
   float knorm_eps;
   uint32_t idesc;
 };
@@ -674,10 +675,12 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
             break;
           }
           const uint32_t fb = mapa_shared(smem_addr(&full_b[stage]), 0);
-          mbar_arrive_expect_tx_cluster(fb, atom_b_bytes);
-          tma_load_2d_pair_hint(smem_addr(sB + stage * stage_b_bytes), tmap, at * kBK,
-                                lc * P.d_r + n * P.BN + static_cast<int>(rank) * half_bn, fb,
-                                pol_b);
+          if (!(P.stall && seq == 0 && at == 0)) {  // the test hook leaves this stage empty
+            mbar_arrive_expect_tx_cluster(fb, atom_b_bytes);
+            tma_load_2d_pair_hint(smem_addr(sB + stage * stage_b_bytes), tmap, at * kBK,
+                                  lc * P.d_r + n * P.BN + static_cast<int>(rank) * half_bn, fb,
+                                  pol_b);
+          }
           if (++stage == stages_b) {
             stage = 0;
             phase ^= 1;
@@ -1195,7 +1198,7 @@ hf_status launch_batch_typed(const BatchParams& B, int64_t max_pair_tiles, size_
 }  // namespace
 
 hf_status launch_transfer(hf_plan_s* p, const void* sender, void* receiver, cudaStream_t stream,
-                          int l_begin, int l_end) {
+                          int l_begin, int l_end, bool stall) {
   const hf_plan_desc& d = p->desc;
   if (l_end < 0) l_end = d.L_r;
   if (p->T_r == 0 || l_end <= l_begin) return HF_OK;
@@ -1204,6 +1207,7 @@ hf_status launch_transfer(hf_plan_s* p, const void* sender, void* receiver, cuda
   int64_t max_pair_tiles = 0;
   hf_status s = make_xfer(p, sender, receiver, l_begin, l_end, &P, &mw, &max_pair_tiles);
   if (s != HF_OK) return s;
+  P.stall = stall ? 1 : 0;
   const size_t smem = smem_bytes(p->BN, P.stages_a, P.stages_b);
   if (d.dtype == HF_F32)
     return p->gather ? launch_pairs(transfer_kernel<float, true>, max_pair_tiles, smem, stream, mw, P)
@@ -1283,4 +1287,19 @@ extern "C" hf_status hf_transfer(hf_plan plan, const void* sender_kv, void* rece
     return HF_ERR_INVALID_ARGUMENT;
   }
   return hf::launch_transfer(plan, sender_kv, receiver_kv, reinterpret_cast<cudaStream_t>(stream));
+}
+
+extern "C" hf_status hf_debug_transfer_stalled(hf_plan plan, const void* sender_kv,
+                                               void* receiver_kv, hf_stream_t stream) {
+  if (!plan || plan->T_r == 0 || !sender_kv || !receiver_kv) {
+    hf::set_error("hf_debug_transfer_stalled: needs a plan with receiver tokens and both caches");
+    return HF_ERR_INVALID_ARGUMENT;
+  }
+  if ((reinterpret_cast<uintptr_t>(sender_kv) | reinterpret_cast<uintptr_t>(receiver_kv) |
+       reinterpret_cast<uintptr_t>(plan->desc.d_W)) & 15u) {
+    hf::set_error("hf_debug_transfer_stalled: caches and maps must be 16-byte aligned");
+    return HF_ERR_INVALID_ARGUMENT;
+  }
+  return hf::launch_transfer(plan, sender_kv, receiver_kv, reinterpret_cast<cudaStream_t>(stream),
+                             0, -1, true);
 }

@@ -159,3 +159,10 @@ def test_rotated_sender_workspace_holds_sender_positions(B):
     a = B.plan_workspace_size(_desc(B, s_tok_ptr=[0, 50000]))
     b = B.plan_workspace_size(_desc(B, s_tok_ptr=[0, 50000], sender_k_rotated=True, theta_s=1e4))
     assert b - a >= 4 * 50000 - 256
+
+
+def test_debug_stalled_transfer_rejects_empty_plan(B):
+    # the bounded-wait test hook validates on the host before any launch
+    with pytest.raises(B.HFError) as e:
+        B.debug_transfer_stalled(B.Plan(None, None, None), None, None)
+    assert e.value.status == B.HF_ERR_INVALID_ARGUMENT
