@@ -183,6 +183,15 @@ EDGE = {
                                                            r_pos0=(3000,)),
     "long_runs_batched_paged": lambda: W.qwen25_to_llama_batched(
         n_req=3, lo=300, hi=900, seed=21).with_(L_s=3, L_r=3, mean_s=12.0, mean_r=1.5),
+    # an empty request between two others (no tokens, no blocks)
+    "empty_request_paged": lambda: W.qwen25_to_llama_batched(
+        n_req=3, lo=100, hi=400, seed=31).with_(L_s=3, L_r=3, r_tokens=(300, 0, 211)),
+    # fp32 caches and maps (tf32 MMA) with a paged receiver cache
+    "batched_paged_f32": lambda: W.qwen25_to_llama_batched(
+        n_req=3, lo=50, hi=300, seed=32).with_(L_s=3, L_r=3, dtype="f32"),
+    # key norm on long runs (the norm is per distinct row, the rotation per position)
+    "knorm_long_runs": lambda: W.llama_to_ministral(2000).with_(
+        L_s=4, L_r=3, knorm=True, mean_s=12.0, mean_r=1.3, r_pos0=(777,)),
     # message spans after a context (only the span's K/V is mapped)
     "message_spans_batched_paged": lambda: W.qwen25_to_llama_batched(
         n_req=3, lo=40, hi=160, seed=12).with_(L_s=4, L_r=3, span_gap=700),
