@@ -92,13 +92,23 @@ extern "C" hf_status hf_transfer_batch(const hf_plan* plans, const void* const* 
   // recorded and waited on within this call, under the lock.
   std::lock_guard<std::mutex> lock(g_pool_mutex);
   HF_CUDA_TRY(cudaEventRecord(pool->fork, stream), "hf_transfer_batch: record");
-  for (int i = 0; i < n; ++i) {
-    HF_CUDA_TRY(cudaStreamWaitEvent(pool->streams[i], pool->fork, 0), "hf_transfer_batch: wait");
+  // Directions already launched are joined back into `stream` even when a
+  // later one fails, so the caller's stream never runs ahead of kernels that
+  // still use its caches.
+  int launched = 0;
+  for (int i = 0; i < n && s == HF_OK; ++i) {
+    cudaError_t e = cudaStreamWaitEvent(pool->streams[i], pool->fork, 0);
+    if (e != cudaSuccess) {
+      s = cuda_fail(e, "hf_transfer_batch: wait");
+      break;
+    }
     s = launch_transfer(plans[i], sender_kv[i], receiver_kv[i], pool->streams[i]);
-    if (s != HF_OK) return s;
-    HF_CUDA_TRY(cudaEventRecord(pool->join[i], pool->streams[i]), "hf_transfer_batch: record");
+    launched = i + 1;  // a failed launch may still have queued nothing; joining it is harmless
   }
-  for (int i = 0; i < n; ++i)
-    HF_CUDA_TRY(cudaStreamWaitEvent(stream, pool->join[i], 0), "hf_transfer_batch: wait");
-  return HF_OK;
+  for (int i = 0; i < launched; ++i) {
+    cudaError_t e = cudaEventRecord(pool->join[i], pool->streams[i]);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(stream, pool->join[i], 0);
+    if (e != cudaSuccess && s == HF_OK) s = cuda_fail(e, "hf_transfer_batch: join");
+  }
+  return s;
 }

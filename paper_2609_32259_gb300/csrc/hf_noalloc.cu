@@ -63,6 +63,17 @@ extern "C" hf_status hf_transfer_noalloc(const hf_plan_desc* desc, const void* s
               " bytes (about 340K receiver tokens); use hf_plan_create with a workspace");
     return HF_ERR_UNSUPPORTED;
   }
+  // the cache checks come before any work is queued: a rejected call leaves
+  // the shared scratch untouched (desc and its r_tok_ptr were checked above)
+  if (desc->r_tok_ptr[desc->n_req] > 0 && (!sender_kv || !receiver_kv)) {
+    set_error("hf_transfer_noalloc: null cache pointer");
+    return HF_ERR_INVALID_ARGUMENT;
+  }
+  if ((reinterpret_cast<uintptr_t>(sender_kv) | reinterpret_cast<uintptr_t>(receiver_kv) |
+       reinterpret_cast<uintptr_t>(desc->d_W)) & 15u) {
+    set_error("hf_transfer_noalloc: caches and maps must be 16-byte aligned");
+    return HF_ERR_INVALID_ARGUMENT;
+  }
   void* ws = nullptr;
   s = scratch_for_current_device(&ws);
   if (s != HF_OK) return s;
@@ -72,14 +83,5 @@ extern "C" hf_status hf_transfer_noalloc(const hf_plan_desc* desc, const void* s
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   s = plan_build(desc, ws, kNoAllocScratchBytes, st, &plan, &tables);
   if (s != HF_OK) return s;
-  if (plan.T_r > 0 && (!sender_kv || !receiver_kv)) {
-    set_error("hf_transfer_noalloc: null cache pointer");
-    return HF_ERR_INVALID_ARGUMENT;
-  }
-  if ((reinterpret_cast<uintptr_t>(sender_kv) | reinterpret_cast<uintptr_t>(receiver_kv) |
-       reinterpret_cast<uintptr_t>(desc->d_W)) & 15u) {
-    set_error("hf_transfer_noalloc: caches and maps must be 16-byte aligned");
-    return HF_ERR_INVALID_ARGUMENT;
-  }
   return launch_transfer(&plan, sender_kv, receiver_kv, st);
 }

@@ -229,7 +229,10 @@ __global__ void plan_runs_kernel(RowArgs a) {
     if (starts) {
       const int32_t u = incl - 1;
       d.run_ptr[u] = static_cast<int32_t>(j);
-      int32_t k = a.col[a.row_ptr[j]];
+      // an empty row (flagged by plan_rows_kernel) has no column to read:
+      // row_ptr[j] may be the end of the caller's col array
+      const int32_t e0 = a.row_ptr[j];
+      int32_t k = a.row_ptr[j + 1] > e0 ? a.col[e0] : 0;
       if (k < 0 || k >= a.T_s) k = 0;  // flagged by plan_rows_kernel
       d.ucol[u] = a.span ? d.srow[k] : k;  // the sender-cache row
       d.upos[u] = d.pos[j];

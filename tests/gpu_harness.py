@@ -128,9 +128,14 @@ class Case:
                           sender_row_of=self.sender_row_of)
 
     def check_parity(self, layers=None, rows=None, rel_tol=REL_FRO_TOL, abs_tol=MAX_ABS_TOL):
+        """Every (layer, role) of `layers` on `rows` against the oracle; the
+        per-(layer, role) errors are kept in self.errors (largest max-abs
+        first in report())."""
         layers = list(range(self.w.L_r)) if layers is None else list(layers)
         rows = np.arange(self.tok.T_r) if rows is None else np.asarray(rows, dtype=np.int64)
         worst = {"rel_fro": 0.0, "max_abs": 0.0}
+        if not hasattr(self, "errors"):
+            self.errors = {}
         assert self.job.device_status() == 0
         for l in layers:
             ref = self.oracle([l], rows)
@@ -141,9 +146,20 @@ class Case:
                 mx = float(np.abs(diff).max()) if diff.size else 0.0
                 worst["rel_fro"] = max(worst["rel_fro"], rel)
                 worst["max_abs"] = max(worst["max_abs"], mx)
+                old = self.errors.get((ll, c), (0.0, 0.0, 0))
+                self.errors[(ll, c)] = (max(old[0], rel), max(old[1], mx), old[2] + diff.size)
                 assert rel <= rel_tol, (ll, c, rel)
                 assert mx <= abs_tol, (ll, c, mx)
         return worst
+
+    def report(self, top=4):
+        """One line: the workload, outputs compared, and the (layer, role)
+        pairs with the largest max-abs error."""
+        items = sorted(self.errors.items(), key=lambda kv: -kv[1][1])
+        n = sum(v[2] for v in self.errors.values())
+        worst = ", ".join(f"l{l}{'KV'[c]} max_abs={v[1]:.4g} rel_fro={v[0]:.3g}"
+                          for (l, c), v in items[:top])
+        return f"{self.w.name} {self.w.align_mode}+{self.w.layer_mode}: {n} outputs; {worst}"
 
 
 def sampled_rows(tok, n, seed=0):
@@ -156,3 +172,51 @@ def sampled_rows(tok, n, seed=0):
         if b > a:
             rows.update({a, b - 1, min(a + 1, b - 1)})
     return np.array(sorted(rows), dtype=np.int64)
+
+
+def run_boundary_rows(csr, r_tok_ptr, max_runs=None, seed=0):
+    """First and last receiver row of every run of identical alignment rows
+    (the rows where the kernel's epilogue starts or ends a distinct row's
+    expansion), plus each request's first and last rows; with max_runs, of
+    that many seeded runs only."""
+    rp = np.asarray(csr.row_ptr, np.int64)
+    col = np.asarray(csr.col, np.int64)
+    w = np.asarray(csr.w, np.float64)
+    T = len(rp) - 1
+    starts = np.zeros(T, bool)
+    for q in range(len(r_tok_ptr) - 1):
+        a = int(r_tok_ptr[q])
+        if a < int(r_tok_ptr[q + 1]):
+            starts[a] = True
+    one = np.all(rp[1:] - rp[:-1] == 1)
+    if one:  # one entry per row: a run starts where the column or weight changes
+        first = col[rp[:-1]]
+        wt = w[rp[:-1]]
+        starts[1:] |= (first[1:] != first[:-1]) | (wt[1:] != wt[:-1])
+    else:
+        for j in range(1, T):
+            a0, a1, b0, b1 = rp[j - 1], rp[j], rp[j], rp[j + 1]
+            if (a1 - a0 != b1 - b0 or not np.array_equal(col[a0:a1], col[b0:b1])
+                    or not np.array_equal(w[a0:a1], w[b0:b1])):
+                starts[j] = True
+    first_rows = np.nonzero(starts)[0]
+    last_rows = np.concatenate([first_rows[1:] - 1, [T - 1]]) if T else first_rows
+    if max_runs is not None and len(first_rows) > max_runs:
+        pick = np.random.default_rng(seed).choice(len(first_rows), max_runs, replace=False)
+        first_rows, last_rows = first_rows[pick], last_rows[pick]
+    return np.unique(np.concatenate([first_rows, last_rows]))
+
+
+def section8c_rows(tok, csr, n_random=4096, seed=0, max_runs=4096):
+    """The sampled rows of a long transfer: the first and last rows of the
+    runs of identical alignment rows (of max_runs seeded runs when there are
+    more), each request's first and last rows (the rows before the first
+    shared boundary open the first run), and n_random seeded rows."""
+    rows = set(run_boundary_rows(csr, tok.r_tok_ptr, max_runs, seed).tolist())
+    rows.update(sampled_rows(tok, n_random, seed).tolist())
+    return np.array(sorted(rows), dtype=np.int64)
+
+
+def whole_layers(L_r):
+    """First, last and two middle receiver layers."""
+    return sorted({0, L_r // 3, (2 * L_r) // 3, L_r - 1})
