@@ -64,12 +64,14 @@ def workload(name):
         "llama_to_ministral_32k": lambda: W.llama_to_ministral(32768),
         "llama_to_qwen25_4k": lambda: W.llama_to_qwen25(4096),
         "qwen25_to_llama_batched_paged": W.qwen25_to_llama_batched,
+        "qwen25_to_llama_kv_ridge_4k": lambda: W.qwen25_to_llama_kv_ridge(4096),
         "tiny": W.tiny,
     }
     w = None
     for prefix, make in (("ministral_to_llama_", W.ministral_to_llama),
                          ("llama_to_ministral_", W.llama_to_ministral),
-                         ("llama_to_qwen25_", W.llama_to_qwen25)):
+                         ("llama_to_qwen25_", W.llama_to_qwen25),
+                         ("qwen25_to_llama_kv_ridge_", W.qwen25_to_llama_kv_ridge)):
         if name.startswith(prefix) and name[len(prefix):].isdigit():
             w = make(int(name[len(prefix):]))
     if w is None:
@@ -187,8 +189,12 @@ def algorithmic_work(w, tok, U, n_distinct_cols):
     e = 2 if w.dtype == "bf16" else 4
     flops = 2.0 * 2 * w.L_r * U * w.K * w.d_r
     T_r = tok.T_r
+    # sender layers the layer table reads (all of them for Eq. 1 and the
+    # interpolation on these depth pairs; the selected ones for an explicit table)
+    n_layers = (len({t for seg_l in w.seg_layer for seg in seg_l for t in seg})
+                if w.layer_mode == "explicit" else w.L_s)
     bytes_ = (2 * w.L_r * T_r * w.d_r * e            # receiver cache
-              + w.L_s * 2 * n_distinct_cols * w.d_s * e  # sender rows
+              + n_layers * 2 * n_distinct_cols * w.d_s * e  # sender rows
               + 2 * w.L_r * w.K * w.d_r * e          # maps
               + 2 * w.L_r * w.d_r * 4                # bias
               + T_r * 4 * 6)                         # CSR + run / position / row metadata
@@ -219,16 +225,26 @@ class OracleSample:
         self.A = Wm.float().cpu().numpy().transpose(0, 1, 3, 2)
         self.b = b.cpu().numpy()
         self.r = r
-        self.segs = O.layer_segments(w.layer_mode, w.L_s, w.L_r)
+        if w.layer_mode == "explicit":
+            self.segs = O.explicit_segments(w.seg_layer, np.asarray(w.seg_w, np.float32))
+        else:
+            self.segs = O.layer_segments(w.layer_mode, w.L_s, w.L_r)
         self.pos = O.receiver_positions(tok.r_tok_ptr)[j0:j0 + n_rows]
         self.inv = O.rope_inv_freq(w.theta_r, w.D_r)
         self.w = w
         self.n_rows = n_rows
 
     def run(self):
+        w = self.w
+        if w.kv_ridge:  # the per-head maps of the KV Ridge apply
+            sel = [[t[0] for t in seg] for seg in w.seg_layer]
+            Wh = [[[self.A[l][c][:, h * w.D_r:(h + 1) * w.D_r] for h in range(w.H_r)]
+                   for c in range(2)] for l in range(w.L_r)]
+            bh = self.b.reshape(w.L_r, 2, w.H_r, w.D_r)
+            return self.O.kv_ridge_transfer(self.sender, self.csr, sel, Wh, bh, H_r=w.H_r,
+                                            D_r=w.D_r, pos=self.pos, inv_freq_r=self.inv)
         return self.O.transfer(self.sender, self.csr, self.segs, self.A, self.b, self.r,
-                               H_r=self.w.H_r, D_r=self.w.D_r, pos=self.pos,
-                               inv_freq_r=self.inv)
+                               H_r=w.H_r, D_r=w.D_r, pos=self.pos, inv_freq_r=self.inv)
 
 
 def blas_threads():

@@ -85,9 +85,14 @@ typedef enum {
   /* One segment: the linear interpolation of sender layers floor(p) and
      floor(p)+1 at p = l (L_S-1)/(L_R-1) (zero-based l): K = d_S. */
   HF_LAYER_INTERP = 1,
-  /* A caller-given table with the structure of Eq. 2: n_seg segments per
-     receiver layer, segment s = sum over its n_terms terms of
-     h_seg_w * (sender layer h_seg_layer): K = n_seg d_S. */
+  /* A caller-given table with the structure of Eq. 2: n_seg (1 .. 8)
+     segments per receiver layer, segment s = sum over its n_terms terms of
+     h_seg_w * (sender layer h_seg_layer): K = n_seg d_S.  The KV Ridge
+     comparison system (Appendix A baseline details, Appendix F mapper size)
+     is this mode with its k = 8 selected sender layers as eight one-layer
+     segments of weight 1, its per-head maps stacked into one dense
+     [8 d_S, d_R] map per layer and role (each head's map reads all KV heads
+     of the eight layers) and r = 1. */
   HF_LAYER_EXPLICIT = 2
 } hf_layer_mode;
 
@@ -218,10 +223,22 @@ typedef struct {
   int64_t sender_rows;
 
   /* HF_LAYER_EXPLICIT only: host arrays [L_r][n_seg][n_terms]. */
-  int32_t n_seg;                /* 1 .. 3 segments per receiver layer */
+  int32_t n_seg;                /* 1 .. 8 segments per receiver layer */
   int32_t n_terms;              /* 1 .. 2 sender layers per segment */
   const int32_t* h_seg_layer;   /* zero-based sender layers, in [0, L_s) */
   const float* h_seg_w;         /* finite weights */
+
+  /* bf16 plans whose map input rows are computed rather than copied
+     (overlap mean pooling, blended layers, weighted explicit segments,
+     rotated sender keys): 0 (default) carries each computed row to the
+     tensor core as a pair of bf16 rows, the rounded value and its rounding
+     residual, both against the same map rows, so the product sees ~16
+     mantissa bits of the fp32 row (about twice the tensor-core work on
+     those rows; the error is the output rounding alone); 1 rounds the row
+     once to bf16 (faster; adds a relative error of about 2^-9 per input
+     feature, which at 1e9 outputs can exceed 2e-2 absolute).  Ignored for
+     copied rows and fp32 plans. */
+  int32_t round_built_operands;
 } hf_plan_desc;
 
 typedef struct hf_plan_s* hf_plan;

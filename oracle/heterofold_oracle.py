@@ -32,6 +32,11 @@ What it computes (arxiv 2609.32259, "HeteroFold"):
 * The output-aware low-rank correction, Eq. 7: y_hat = y0 + (y0 B) G with
   y0 = (x / r) A + b, and its folding, Eq. 9: A_final = A (I + B G),
   b_final = b (I + B G).
+* The KV Ridge + TA apply (Appendix A, baseline details; Section 4 setup;
+  Appendix F, mapper size): each receiver layer reads k = 8 selected sender
+  layers, and each receiver KV head has its own ridge map from all KV heads
+  of those layers (their concatenation) to that head's features; with TA the
+  token correspondence is Token Alignment, otherwise same-index pairing.
 * The folded inference map, Eq. 9: Phi(x) = (x / r) A_final + b_final,
   one map per receiver layer and role, reshaped to receiver KV heads; keys
   then get the receiver's key normalisation and RoPE at receiver positions
@@ -452,6 +457,55 @@ def transfer(sender, csr: CSR, segments, A, b, r, *, H_r: int, D_r: int,
             if c == ROLE_K:
                 if knorm_g is not None:
                     y = key_norm(y, knorm_g, knorm_eps)
+                y = rope(y, np.asarray(pos)[rows], inv_freq_r)
+            out[(l, c)] = y
+    return out
+
+
+# ---------------------------------------------------------------------------
+# KV Ridge + TA apply (Appendix A baseline details, Appendix F mapper size)
+# ---------------------------------------------------------------------------
+
+KV_RIDGE_K = 8  # sender layers per receiver layer (the method's default k)
+
+
+def kv_ridge_segments(selected) -> List[List[List[Tuple[int, float]]]]:
+    """KV Ridge's layer routing: receiver layer l reads the sender layers
+    selected[l] (k of them, chosen offline by calibration R^2), each as one
+    segment of weight 1, concatenated in the given order."""
+    return [[[(int(t), 1.0)] for t in sel] for sel in selected]
+
+
+def kv_ridge_transfer(sender, csr: CSR, selected, W_heads, b_heads, *, H_r: int, D_r: int,
+                      pos: np.ndarray, inv_freq_r: np.ndarray,
+                      layers: Optional[Iterable[int]] = None,
+                      rows: Optional[np.ndarray] = None,
+                      roles: Iterable[int] = (ROLE_K, ROLE_V)) -> Dict[Tuple[int, int], np.ndarray]:
+    """The receiver cache entries of the KV Ridge apply.
+
+    For receiver layer l, role c and receiver KV head h:
+        y_h = x W_heads[l][c][h] + b_heads[l][c][h],
+    x the concatenation of every KV head of the selected sender layers
+    (kv_ridge_segments(selected)[l], Eq. 2's layout) at the aligned sender
+    token; W_heads[l][c][h] is [k * d_S, D_r] and b_heads[l][c][h] is [D_r].
+    A ridge map is a plain least-squares affine map: there is no Eq. 3
+    normaliser.  Keys then get RoPE at their receiver positions, as in
+    transfer().  Returns {(l, c): [n_rows, H_r, D_r] float64}."""
+    rows = np.arange(csr.n_rows) if rows is None else np.asarray(rows, dtype=np.int64)
+    segments = kv_ridge_segments(selected)
+    layers = range(len(segments)) if layers is None else layers
+    out: Dict[Tuple[int, int], np.ndarray] = {}
+    for l in layers:
+        for c in roles:
+            x = map_input(sender, csr, segments[l], c, rows)
+            y = np.empty((len(rows), H_r, D_r))
+            for h in range(H_r):
+                Wh = np.asarray(W_heads[l][c][h], dtype=np.float64)
+                if Wh.shape != (x.shape[1], D_r):
+                    raise ValueError(f"head map shape {Wh.shape} does not match input width "
+                                     f"{x.shape[1]} and D_r {D_r}")
+                y[:, h, :] = x @ Wh + np.asarray(b_heads[l][c][h], dtype=np.float64)
+            if c == ROLE_K:
                 y = rope(y, np.asarray(pos)[rows], inv_freq_r)
             out[(l, c)] = y
     return out

@@ -67,6 +67,7 @@ class PlanDesc(ctypes.Structure):
         ("s_row0", _i32p), ("sender_rows", ctypes.c_int64),
         ("n_seg", ctypes.c_int32), ("n_terms", ctypes.c_int32),
         ("h_seg_layer", _i32p), ("h_seg_w", _f32p),
+        ("round_built_operands", ctypes.c_int32),
     ]
 
 
@@ -182,7 +183,8 @@ class Desc:
                  r_pos0=None, d_knorm_w=None, knorm_eps=1e-6, paged=False, block_size=16,
                  n_blocks=0, max_blocks_per_req=0, d_block_table=None, inv_freq_r=None,
                  sender_k_rotated=False, theta_s=0.0, inv_freq_s=None, s_pos0=None,
-                 seg_layer=None, seg_w=None, s_row0=None, sender_rows=0):
+                 seg_layer=None, seg_w=None, s_row0=None, sender_rows=0,
+                 round_built_operands=False):
         self._s = _host_i32(s_tok_ptr)
         self._r = _host_i32(r_tok_ptr)
         self._pos0 = None if r_pos0 is None else _host_i32(r_pos0)
@@ -218,7 +220,8 @@ class Desc:
             sender_rows=int(sender_rows),
             n_seg=n_seg, n_terms=n_terms,
             h_seg_layer=_as_i32p(self._segl) if self._segl is not None else None,
-            h_seg_w=_f32_or_null(self._segw))
+            h_seg_w=_f32_or_null(self._segw),
+            round_built_operands=int(bool(round_built_operands)))
 
 
 def plan_workspace_size(desc: Desc) -> int:

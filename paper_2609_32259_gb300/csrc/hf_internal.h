@@ -13,7 +13,8 @@ namespace hf {
 
 constexpr int kMaxReq = 1024;        // requests per call
 constexpr int kMaxLayersR = 128;     // receiver layers
-constexpr int kMaxSeg = 3;           // map input segments per receiver layer
+constexpr int kMaxSeg = 8;           // map input segments per receiver layer (Eq. 1: 3;
+                                     // KV Ridge's layer routing: 8)
 constexpr int kMaxTerms = 2;         // sender layers blended into one segment
 constexpr int kMaxHeadDim = 256;
 constexpr int kMaxBatch = 16;        // directions per hf_transfer_batch call
@@ -53,11 +54,12 @@ struct WorkspaceLayout {
 
 WorkspaceLayout workspace_layout(const hf_plan_desc& d);
 
-// Constant tables copied into the workspace by the plan kernel (passed by
-// value as a kernel parameter, so plan creation issues no host copies).
-struct PlanTables {
+// Constant tables copied into the workspace by the plan kernels.  They are
+// passed by value as kernel parameters, so plan creation issues no host
+// copies; the layer table goes to a kernel of its own because one launch's
+// parameters are limited to 32 KB.
+struct PlanConsts {
   int32_t L_r, D_r, D_s, n_req;
-  LayerSegs segs[kMaxLayersR];
   float inv_r[2 * kMaxLayersR];
   float inv_freq[kMaxHeadDim / 2];
   float inv_freq_s[kMaxHeadDim / 2];
@@ -67,7 +69,16 @@ struct PlanTables {
   int32_t s_pos0[kMaxReq];
   int32_t s_row0[kMaxReq];
 };
-static_assert(sizeof(PlanTables) < 32000, "PlanTables must fit the kernel parameter space");
+struct SegTables {
+  int32_t L_r;
+  LayerSegs segs[kMaxLayersR];
+};
+struct PlanTables {
+  PlanConsts c;
+  SegTables s;
+};
+static_assert(sizeof(PlanConsts) < 32000, "PlanConsts must fit the kernel parameter space");
+static_assert(sizeof(SegTables) < 32000, "SegTables must fit the kernel parameter space");
 
 }  // namespace hf
 
@@ -77,6 +88,7 @@ struct hf_plan_s {
   int64_t T_s, T_r, nnz_hint;
   int BN, groups, stages;
   bool gather;  // every map input row is a single unweighted sender row
+  bool split;   // computed bf16 operand rows go to the tensor core as value + residual
   bool rope;    // receiver keys get RoPE
   bool unrot;   // sender keys carry RoPE and are rotated back in the builder
   bool span;    // aligned sender tokens are spans inside a longer sender cache

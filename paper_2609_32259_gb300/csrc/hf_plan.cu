@@ -124,13 +124,12 @@ PlanDev plan_dev(const hf_plan_s* p) {
 }
 
 // Copies the constant tables into the workspace and clears the counters.
-__global__ void plan_init_kernel(PlanTables t, PlanDev d) {
+__global__ void plan_init_kernel(PlanConsts t, PlanDev d) {
   const int tid = threadIdx.x;
   if (tid == 0) {
     *d.status = 0;
     *d.n_distinct = 0;
   }
-  for (int i = tid; i < t.L_r; i += blockDim.x) d.segs[i] = t.segs[i];
   for (int i = tid; i < 2 * t.L_r; i += blockDim.x) d.inv_r[i] = t.inv_r[i];
   for (int i = tid; i < t.D_r / 2; i += blockDim.x) d.inv_freq[i] = t.inv_freq[i];
   for (int i = tid; i <= t.n_req; i += blockDim.x) d.r_tok_ptr[i] = t.r_tok_ptr[i];
@@ -139,6 +138,11 @@ __global__ void plan_init_kernel(PlanTables t, PlanDev d) {
   for (int i = tid; i <= t.n_req; i += blockDim.x) d.s_tok_ptr[i] = t.s_tok_ptr[i];
   for (int i = tid; i < t.n_req; i += blockDim.x) d.s_pos0[i] = t.s_pos0[i];
   for (int i = tid; i < t.n_req; i += blockDim.x) d.s_row0[i] = t.s_row0[i];
+}
+
+// Copies the layer table into the workspace.
+__global__ void plan_segs_kernel(SegTables t, LayerSegs* segs) {
+  for (int i = threadIdx.x; i < t.L_r; i += blockDim.x) segs[i] = t.segs[i];
 }
 
 // Per aligned sender token: its RoPE position (sender_k_rotated), the
@@ -315,7 +319,7 @@ hf_status validate(const hf_plan_desc* d) {
       d->layer_mode != HF_LAYER_EXPLICIT)
     return bad("unknown layer mode");
   if (d->layer_mode == HF_LAYER_EXPLICIT) {
-    if (d->n_seg < 1 || d->n_seg > kMaxSeg) return bad("explicit layer table: n_seg must be 1..3");
+    if (d->n_seg < 1 || d->n_seg > kMaxSeg) return bad("explicit layer table: n_seg must be 1..8");
     if (d->n_terms < 1 || d->n_terms > kMaxTerms)
       return bad("explicit layer table: n_terms must be 1..2");
     if (!d->h_seg_layer || !d->h_seg_w) return bad("explicit layer table: null arrays");
@@ -367,6 +371,8 @@ hf_status validate(const hf_plan_desc* d) {
       return unsup("sender_k_rotated: D_s/2 must be a multiple of 8 (bf16) or 4 (fp32), D_s must "
                    "divide 128 (bf16) or 64 (fp32), d_S a multiple of 128 (bf16) or 64 (fp32)");
   }
+  if (d->round_built_operands != 0 && d->round_built_operands != 1)
+    return bad("round_built_operands must be 0 or 1");
   if (d->paged) {
     if (d->block_size < 1 || d->n_blocks < 1 || d->max_blocks_per_req < 1 || !d->d_block_table)
       return bad("paged layout needs block_size, n_blocks, max_blocks_per_req, d_block_table");
@@ -392,7 +398,8 @@ hf_status validate(const hf_plan_desc* d) {
 
 hf_status launch_plan_kernels(hf_plan_s* p, const PlanTables& tables, cudaStream_t stream) {
   const PlanDev d = plan_dev(p);
-  plan_init_kernel<<<1, 256, 0, stream>>>(tables, d);
+  plan_init_kernel<<<1, 256, 0, stream>>>(tables.c, d);
+  plan_segs_kernel<<<1, 128, 0, stream>>>(tables.s, d.segs);
   HF_CUDA_TRY(cudaGetLastError(), "plan init launch");
   if (p->T_r == 0) return HF_OK;
   RowArgs a;
@@ -476,6 +483,7 @@ hf_status plan_build(const hf_plan_desc* desc, void* d_workspace, size_t workspa
   p->unrot = desc->sender_k_rotated == 1;
   p->rope = desc->theta_r > 0.0 || desc->h_inv_freq_r != nullptr;
   p->gather = one_layer_segments && desc->align_mode != HF_ALIGN_OVERLAP_MEAN && !p->unrot;
+  p->split = !p->gather && desc->dtype == HF_BF16 && desc->round_built_operands == 0;
   p->ws = static_cast<char*>(d_workspace);
   p->ws_bytes = workspace_bytes;
   p->lay = lay;
@@ -492,35 +500,38 @@ hf_status plan_build(const hf_plan_desc* desc, void* d_workspace, size_t workspa
   p->desc.h_seg_w = nullptr;
 
   std::memset(t, 0, sizeof(*t));
-  t->L_r = desc->L_r;
-  t->D_r = desc->D_r;
-  t->D_s = p->unrot ? desc->D_s : 0;
-  t->n_req = desc->n_req;
-  build_layer_table(*desc, t->segs);
+  PlanConsts* c = &t->c;
+  c->L_r = desc->L_r;
+  c->D_r = desc->D_r;
+  c->D_s = p->unrot ? desc->D_s : 0;
+  c->n_req = desc->n_req;
+  t->s.L_r = desc->L_r;
+  build_layer_table(*desc, t->s.segs);
   for (int l = 0; l < desc->L_r; ++l) {
+    const LayerSegs& sg = t->s.segs[l];
     int mx = 0;
-    for (int k = 0; k < t->segs[l].n_seg; ++k)
-      for (int i = 0; i < t->segs[l].n_terms[k]; ++i) mx = std::max(mx, t->segs[l].layer[k][i]);
+    for (int k = 0; k < sg.n_seg; ++k)
+      for (int i = 0; i < sg.n_terms[k]; ++i) mx = std::max(mx, sg.layer[k][i]);
     p->max_sender_layer[l] = mx;
   }
-  for (int i = 0; i < 2 * desc->L_r; ++i) t->inv_r[i] = static_cast<float>(1.0 / desc->h_r[i]);
+  for (int i = 0; i < 2 * desc->L_r; ++i) c->inv_r[i] = static_cast<float>(1.0 / desc->h_r[i]);
   // inv_freq_i = fp32(theta^(-2i/D)) evaluated in double precision
   // (or the caller's table)
   for (int i = 0; i < desc->D_r / 2; ++i)
-    t->inv_freq[i] = desc->h_inv_freq_r ? desc->h_inv_freq_r[i]
+    c->inv_freq[i] = desc->h_inv_freq_r ? desc->h_inv_freq_r[i]
                      : desc->theta_r > 0.0
                          ? static_cast<float>(std::pow(desc->theta_r, -(2.0 * i) / desc->D_r))
                          : 0.0f;
   if (p->unrot)
     for (int i = 0; i < desc->D_s / 2; ++i)
-      t->inv_freq_s[i] = desc->h_inv_freq_s
+      c->inv_freq_s[i] = desc->h_inv_freq_s
                              ? desc->h_inv_freq_s[i]
                              : static_cast<float>(std::pow(desc->theta_s, -(2.0 * i) / desc->D_s));
-  for (int q = 0; q <= desc->n_req; ++q) t->r_tok_ptr[q] = desc->r_tok_ptr[q];
-  for (int q = 0; q < desc->n_req; ++q) t->r_pos0[q] = desc->r_pos0 ? desc->r_pos0[q] : 0;
-  for (int q = 0; q <= desc->n_req; ++q) t->s_tok_ptr[q] = desc->s_tok_ptr[q];
-  for (int q = 0; q < desc->n_req; ++q) t->s_pos0[q] = desc->s_pos0 ? desc->s_pos0[q] : 0;
-  for (int q = 0; q < desc->n_req; ++q) t->s_row0[q] = desc->s_row0 ? desc->s_row0[q] : 0;
+  for (int q = 0; q <= desc->n_req; ++q) c->r_tok_ptr[q] = desc->r_tok_ptr[q];
+  for (int q = 0; q < desc->n_req; ++q) c->r_pos0[q] = desc->r_pos0 ? desc->r_pos0[q] : 0;
+  for (int q = 0; q <= desc->n_req; ++q) c->s_tok_ptr[q] = desc->s_tok_ptr[q];
+  for (int q = 0; q < desc->n_req; ++q) c->s_pos0[q] = desc->s_pos0 ? desc->s_pos0[q] : 0;
+  for (int q = 0; q < desc->n_req; ++q) c->s_row0[q] = desc->s_row0 ? desc->s_row0[q] : 0;
   return launch_plan_kernels(p, *t, stream);
 }
 

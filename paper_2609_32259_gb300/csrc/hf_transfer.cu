@@ -82,6 +82,10 @@ struct XferParams {
   int L_r, d_s, d_r, D_r;
   int l0, n_l;  // receiver layers [l0, l0 + n_l) of this launch
   int n_kb, atoms_per_seg, last_atoms, BN, n_tiles_n, groups;  // n_kb: A stages per tile
+  // split: each A stage holds one map atom of K as two bf16 atoms, the
+  // rounded operand and its rounding residual, multiplied by the same B atom
+  // (atoms_per_stage = 1); otherwise kAtoms atoms of K per A stage
+  int split, atoms_per_stage, n_batoms;  // n_batoms: B atoms (map atoms of K) per tile
   int stages_a, stages_b, lag;  // A ring (stages), B ring (atoms), loader groups in flight
   int rope, paged, knorm, unrot, D_s;
   int stall;  // test hook: the map producer withholds its first atom (hf_debug_transfer_stalled)
@@ -158,6 +162,41 @@ __device__ __forceinline__ uint4 pack16(const float* a, const __nv_bfloat16*) {
 __device__ __forceinline__ uint4 pack16(const float* a, const float*) {
   return make_uint4(__float_as_uint(a[0]), __float_as_uint(a[1]), __float_as_uint(a[2]),
                     __float_as_uint(a[3]));
+}
+
+// 8 fp32 values as bf16 (round to nearest) in *hi, and in *lo the bf16
+// rounding of what that rounding lost (exact in fp32): hi + lo carries each
+// value to about 16 mantissa bits.
+__device__ __forceinline__ void pack16_split(const float* a, uint4* hi, uint4* lo) {
+  uint32_t h[4], r[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const __nv_bfloat162 b = __floats2bfloat162_rn(a[2 * i], a[2 * i + 1]);
+    const float2 bf = __bfloat1622float2(b);
+    const __nv_bfloat162 d = __floats2bfloat162_rn(a[2 * i] - bf.x, a[2 * i + 1] - bf.y);
+    h[i] = *reinterpret_cast<const uint32_t*>(&b);
+    r[i] = *reinterpret_cast<const uint32_t*>(&d);
+  }
+  *hi = make_uint4(h[0], h[1], h[2], h[3]);
+  *lo = make_uint4(r[0], r[1], r[2], r[3]);
+}
+
+// Writes 16 bytes of fp32 results of operand row t, chunk ch, into an A atom
+// (rounded once), or into the value atom and the residual atom (split).
+template <typename T>
+__device__ __forceinline__ void put_chunk(const float* a, uint8_t* atom, uint8_t* lo_atom, int t,
+                                          int ch) {
+  const int off = t * 128 + ((ch ^ (t & 7)) << 4);
+  if constexpr (sizeof(T) == 2) {
+    if (lo_atom) {
+      uint4 hi, lo;
+      pack16_split(a, &hi, &lo);
+      *reinterpret_cast<uint4*>(atom + off) = hi;
+      *reinterpret_cast<uint4*>(lo_atom + off) = lo;
+      return;
+    }
+  }
+  *reinterpret_cast<uint4*>(atom + off) = pack16(a, (const T*)nullptr);
 }
 
 // Receiver-cache stores are streaming stores (st.global.cs, evict first):
@@ -347,10 +386,12 @@ __device__ __forceinline__ int find_row(const int32_t* srun, int nrows, int j) {
 // One 128-byte atom of operand row t for the builder path: features
 // [kin*kBK, (kin+1)*kBK) of segment `seg`, i.e. sum over the segment's
 // sender layers (weight om) and the row's CSR entries (weight w) of the
-// sender rows, accumulated in fp32 and rounded once into the swizzled layout.
+// sender rows, accumulated in fp32 and written into the swizzled layout,
+// rounded once, or as value + residual atoms when lo_atom is given.
 template <typename T>
 __device__ __forceinline__ void build_atom(const XferParams& P, const LayerSegs& segs, int seg,
-                                           int kin, int c, int e0, int e1, uint8_t* atom, int t) {
+                                           int kin, int c, int e0, int e1, uint8_t* atom,
+                                           uint8_t* lo_atom, int t) {
   constexpr int kBK = Elem<T>::kBK;
   constexpr int kPerChunk = 16 / sizeof(T);
   const T* sender = reinterpret_cast<const T*>(P.sender);
@@ -374,11 +415,64 @@ __device__ __forceinline__ void build_atom(const XferParams& P, const LayerSegs&
       for (int k2 = 0; k2 < 8; ++k2) accum16(x[k2], wt, acc + k2 * kPerChunk, (const T*)nullptr);
     }
   }
-  uint8_t* dst = atom + t * 128;
 #pragma unroll
-  for (int k2 = 0; k2 < 8; ++k2)
-    *reinterpret_cast<uint4*>(dst + ((k2 ^ (t & 7)) << 4)) =
-        pack16(acc + k2 * kPerChunk, (const T*)nullptr);
+  for (int k2 = 0; k2 < 8; ++k2) put_chunk<T>(acc + k2 * kPerChunk, atom, lo_atom, t, k2);
+}
+
+// One atom of operand row t when the sender keys carry RoPE (split operands):
+// each sender row is rotated back at its own sender position before the CSR
+// and layer weights are applied.  Feature i of a head pairs with i + D_s/2
+// (first half: x cos + y sin) or i - D_s/2 (second half: x cos - y sin), the
+// angle pos * inv_freq_s_{i mod D_s/2}; a 16-byte chunk never straddles the
+// halves (D_s/2 is a multiple of the chunk).  The angle uses the same
+// exact-product reduction as the epilogue.
+template <typename T>
+__device__ __forceinline__ void build_atom_unrotated(const XferParams& P, const LayerSegs& segs,
+                                                     int seg, int kin, int c, int e0, int e1,
+                                                     uint8_t* atom, uint8_t* lo_atom, int t) {
+  constexpr int kBK = Elem<T>::kBK;
+  constexpr int kPerChunk = 16 / sizeof(T);
+  const T* sender = reinterpret_cast<const T*>(P.sender);
+  const int hs = P.D_s / 2;
+#pragma unroll 1
+  for (int ch = 0; ch < kBK / kPerChunk; ++ch) {
+    const int el = kin * kBK + ch * kPerChunk;  // feature within the segment
+    const int i = el % P.D_s;
+    const bool first = i < hs;
+    const int partner = first ? el + hs : el - hs;
+    const int fi = first ? i : i - hs;
+    float f[kPerChunk], acc[kPerChunk];
+#pragma unroll
+    for (int q = 0; q < kPerChunk; ++q) {
+      f[q] = __ldg(P.inv_freq_s + fi + q);
+      acc[q] = 0.f;
+    }
+    for (int ti = 0; ti < segs.n_terms[seg]; ++ti) {
+      const int tl = segs.layer[seg][ti];
+      const float om = segs.w[seg][ti];
+      const T* base = sender + (static_cast<int64_t>(tl * 2 + c) * P.s_rows) * P.d_s;
+      for (int e = e0; e < e1; ++e) {
+        const int k = P.col[e];
+        if (k < 0 || k >= P.T_s) continue;  // flagged at plan creation
+        const float wt = om * P.w[e];
+        const int64_t kr = P.srow ? __ldg(P.srow + k) : k;
+        const T* row = base + kr * P.d_s;
+        float x[kPerChunk], y[kPerChunk];
+#pragma unroll
+        for (int q = 0; q < kPerChunk; ++q) x[q] = y[q] = 0.f;
+        accum16(__ldg(reinterpret_cast<const uint4*>(row + el)), 1.f, x, (const T*)nullptr);
+        accum16(__ldg(reinterpret_cast<const uint4*>(row + partner)), 1.f, y, (const T*)nullptr);
+        const int p = __ldg(P.spos + k);
+#pragma unroll
+        for (int q = 0; q < kPerChunk; ++q) {
+          float sn, cs;
+          rope_sincos(p, f[q], &sn, &cs);
+          acc[q] = fmaf(wt, first ? fmaf(x[q], cs, y[q] * sn) : fmaf(x[q], cs, -y[q] * sn), acc[q]);
+        }
+      }
+    }
+    put_chunk<T>(acc, atom, lo_atom, t, ch);
+  }
 }
 
 // One stage (kAtoms atoms = whole heads of one segment) of operand row t
@@ -513,11 +607,15 @@ __device__ __forceinline__ void gather_rows(const XferParams* Ps, const DirTable
     int lc, m, n;
     decode_tile(tile - dt.base[dd], dt.m_tiles[dd] * P.n_tiles_n, P.n_tiles_n, P.l0, &lc, &m, &n);
     const int l = lc >> 1, c = lc & 1;
-    // element offset of each segment's sender layer/role block, for the whole tile
-    int64_t seg_base[kMaxSeg];
-#pragma unroll
-    for (int s2 = 0; s2 < kMaxSeg; ++s2)
-      seg_base[s2] = (static_cast<int64_t>(P.segs[l].layer[s2][0] * 2 + c) * P.s_rows) * P.d_s;
+    // element offset of segment s2's sender layer/role block; the current
+    // segment's is in sbase and the next one's is loaded a segment ahead
+    const LayerSegs* lsegs = P.segs + l;
+    const int n_seg = __ldg(&lsegs->n_seg);
+    auto seg_base = [&](int s2) -> int64_t {
+      return (static_cast<int64_t>(__ldg(&lsegs->layer[s2][0]) * 2 + c) * P.s_rows) * P.d_s;
+    };
+    int64_t sbase = seg_base(0);
+    int64_t snext = n_seg > 1 ? seg_base(1) : 0;
     int64_t roff[8];
     uint32_t doff[8];
 #pragma unroll
@@ -539,13 +637,14 @@ __device__ __forceinline__ void gather_rows(const XferParams* Ps, const DirTable
 #pragma unroll
       for (int a = 0; a < kAtoms; ++a) {
         if (a < na) {
-          const int64_t sbase = seg == 0 ? seg_base[0] : (seg == 1 ? seg_base[1] : seg_base[2]);
           const T* base = sender + sbase + kin * kBK;
 #pragma unroll
           for (int i = 0; i < 8; ++i) cp_async_16(sa + a * kAtomABytes + doff[i], base + roff[i]);
           if (++kin == P.atoms_per_seg) {
             kin = 0;
             ++seg;
+            sbase = snext;
+            if (seg + 1 < n_seg) snext = seg_base(seg + 1);
           }
         }
       }
@@ -667,7 +766,7 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
         int lc, m, n;
         decode_tile(tile - dt.base[dd], dt.m_tiles[dd] * P.n_tiles_n, P.n_tiles_n, P.l0, &lc, &m,
                     &n);
-        const int n_atoms = (P.n_kb - 1) * kAtoms + P.last_atoms;
+        const int n_atoms = P.n_batoms;
         for (int at = 0; at < n_atoms; ++at) {
           if (!mbar_wait(smem_addr(&empty_b[stage]), phase ^ 1)) {
             raise_timeout(P, sAbort);
@@ -712,7 +811,8 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
        tile = tile_of(++seq, first_tile, tile_step, by_slot)) {
         const XferParams& P = Ps[dir_of(dt, n_dir, tile)];
         const uint32_t idesc = P.idesc;
-        const int n_kb = P.n_kb, last_atoms = P.last_atoms;
+        const int n_kb = P.n_kb, last_atoms = P.last_atoms, per_stage = P.atoms_per_stage;
+        const bool split = P.split != 0;
         if (!mbar_wait(smem_addr(&tempty[acc]), acc_phase ^ 1)) {
           raise_timeout(P, sAbort);
           break;
@@ -726,7 +826,7 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
             ok = false;
             break;
           }
-          const int na = kb == n_kb - 1 ? last_atoms : kAtoms;
+          const int na = kb == n_kb - 1 ? last_atoms : per_stage;
 #pragma unroll
           for (int a = 0; a < kAtoms; ++a) {
             if (a >= na) break;
@@ -744,6 +844,13 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
               mma_bf16_pair(d_tmem, ad + 2, bd + 2, idesc, 1);
               mma_bf16_pair(d_tmem, ad + 4, bd + 4, idesc, 1);
               mma_bf16_pair(d_tmem, ad + 6, bd + 6, idesc, 1);
+              if (split) {  // the residual atom against the same map atom
+                const uint64_t lo = ad + atom_a;
+                mma_bf16_pair(d_tmem, lo, bd, idesc, 1);
+                mma_bf16_pair(d_tmem, lo + 2, bd + 2, idesc, 1);
+                mma_bf16_pair(d_tmem, lo + 4, bd + 4, idesc, 1);
+                mma_bf16_pair(d_tmem, lo + 6, bd + 6, idesc, 1);
+              }
             } else {
               mma_tf32_pair(d_tmem, ad, bd, idesc, accumulate);
               mma_tf32_pair(d_tmem, ad + 2, bd + 2, idesc, 1);
@@ -954,7 +1061,17 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
             break;
           }
           uint8_t* st = sA + stage * kStageABytes;
-          if (unrot_k) {
+          if (P.split) {
+            // one map atom of K: the value atom and its residual atom
+            if (unrot_k)
+              build_atom_unrotated<T>(P, segs, seg, kin, c, e0, e1, st, st + kAtomABytes, t);
+            else
+              build_atom<T>(P, segs, seg, kin, c, e0, e1, st, st + kAtomABytes, t);
+            if (++kin == P.atoms_per_seg) {
+              kin = 0;
+              ++seg;
+            }
+          } else if (unrot_k) {
             // the stage is whole heads of one segment (checked at plan creation)
             build_stage_unrotated<T>(P, segs, seg, kin, c, e0, e1, st, t);
             kin += kAtoms;
@@ -965,7 +1082,7 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
           } else {
             const int na = kb == P.n_kb - 1 ? P.last_atoms : kAtoms;
             for (int a = 0; a < na; ++a) {
-              build_atom<T>(P, segs, seg, kin, c, e0, e1, st + a * kAtomABytes, t);
+              build_atom<T>(P, segs, seg, kin, c, e0, e1, st + a * kAtomABytes, nullptr, t);
               if (++kin == P.atoms_per_seg) {
                 kin = 0;
                 ++seg;
@@ -1169,8 +1286,11 @@ hf_status make_xfer(hf_plan_s* p, const void* sender, void* receiver, int l_begi
   P.d_r = p->d_r;
   P.D_r = d.D_r;
   const int n_atoms = p->K / bk;  // 128-byte k-blocks per output row
-  P.n_kb = (n_atoms + kAtoms - 1) / kAtoms;
-  P.last_atoms = n_atoms - kAtoms * (P.n_kb - 1);
+  P.split = p->split ? 1 : 0;
+  P.atoms_per_stage = p->split ? 1 : kAtoms;
+  P.n_batoms = n_atoms;
+  P.n_kb = (n_atoms + P.atoms_per_stage - 1) / P.atoms_per_stage;
+  P.last_atoms = n_atoms - P.atoms_per_stage * (P.n_kb - 1);
   P.atoms_per_seg = p->d_s / bk;
   P.BN = p->BN;
   P.n_tiles_n = p->d_r / p->BN;
@@ -1219,7 +1339,8 @@ hf_status launch_transfer(hf_plan_s* p, const void* sender, void* receiver, cuda
 
 bool batch_compatible(const hf_plan_s* const* plans, int n) {
   for (int i = 1; i < n; ++i)
-    if (plans[i]->desc.dtype != plans[0]->desc.dtype || plans[i]->gather != plans[0]->gather)
+    if (plans[i]->desc.dtype != plans[0]->desc.dtype || plans[i]->gather != plans[0]->gather ||
+        plans[i]->split != plans[0]->split)
       return false;
   return true;
 }

@@ -23,7 +23,11 @@ which are available offline:
   the root-mean-square channel scale of that role times U(0.9, 1.1), so the
   mapped features have roughly unit variance;
 * paged cache: 16-token blocks, a pool with 10% spare blocks and a seeded
-  random permutation as the block table.
+  random permutation as the block table;
+* KV Ridge apply: per receiver layer the 8 sender layers with the smallest
+  |t - p| + U(0, 3) (p the proportional depth; a stand-in for the
+  calibrated R^2 ranking), maps drawn as above and divided by the scale r
+  would have had, with r = 1 (ridge maps have no normaliser).
 """
 
 from __future__ import annotations
@@ -69,6 +73,7 @@ class Workload:
     s_pos0: Optional[Tuple[int, ...]] = None
     rope_table: bool = False           # receiver RoPE from a caller table (inv_freq_r_table)
     span_gap: int = 0                  # message spans: cache rows before each request's span
+    kv_ridge: bool = False             # KV Ridge apply: explicit k-layer table, maps without r
 
     @property
     def d_s(self) -> int:
@@ -136,6 +141,34 @@ def ministral_to_llama(T_r: int) -> Workload:
     return Workload(f"ministral_to_llama8b_{T_r}", L_s=40, H_s=8, D_s=128, L_r=32, H_r=8,
                     D_r=128, theta_s=1e8, theta_r=500000.0, r_tokens=(T_r,),
                     mean_s=3.6, mean_r=4.0, seed=4)
+
+
+def kv_ridge_selection(L_s: int, L_r: int, k: int = 8, seed: int = 0):
+    """A stand-in for KV Ridge's calibrated layer selection (k sender layers
+    per receiver layer, ranked by calibration R^2, which favours layers near
+    the proportional depth): the k sender layers with the smallest
+    |t - p| + U(0, 3), p = l (L_s - 1)/(L_r - 1), in ascending order."""
+    rng = np.random.default_rng([seed, 1010])
+    out = []
+    for l in range(L_r):
+        p = l * (L_s - 1) / (L_r - 1) if L_r > 1 else 0.0
+        score = np.abs(np.arange(L_s) - p) + rng.uniform(0.0, 3.0, size=L_s)
+        out.append(tuple(sorted(int(t) for t in np.argsort(score, kind="stable")[:k])))
+    return tuple(out)
+
+
+def qwen25_to_llama_kv_ridge(T_r: int = 4096, k: int = 8, align_mode: str = "ta") -> Workload:
+    """KV Ridge + TA apply on the Qwen2.5-7B-shaped -> Llama-3.1-8B-shaped
+    direction: k = 8 selected sender layers per receiver layer, one dense
+    [k d_S, d_R] map per layer and role (the per-head maps stacked), no
+    Eq. 3 normaliser."""
+    sel = kv_ridge_selection(28, 32, k, seed=13)
+    layers = tuple(tuple((t,) for t in s) for s in sel)
+    weights = tuple(tuple((1.0,) for _ in s) for s in sel)
+    return Workload(f"qwen25_7b_to_llama8b_kv_ridge{k}_{T_r}", L_s=28, H_s=4, D_s=128, L_r=32,
+                    H_r=8, D_r=128, theta_s=1e6, theta_r=500000.0, r_tokens=(T_r,),
+                    mean_s=3.6, mean_r=4.0, seed=13, align_mode=align_mode,
+                    layer_mode="explicit", seg_layer=layers, seg_w=weights, kv_ridge=True)
 
 
 SWEEP_TOKENS = (256, 512, 1024, 4096, 16384, 32768, 65536, 131072)
@@ -269,19 +302,26 @@ def sender_kv(w: Workload, T_s: int, device="cpu") -> torch.Tensor:
 
 def maps(w: Workload, device="cpu"):
     """Folded maps: W [L_r, 2, d_r, K] (= A_final transposed, workload
-    dtype), bias [L_r, 2, d_r] fp32, r [L_r, 2] fp32 (host numpy)."""
+    dtype), bias [L_r, 2, d_r] fp32, r [L_r, 2] fp32 (host numpy).
+
+    KV Ridge workloads have no normaliser: their maps come out of the same
+    draw divided by the scale r would have had (so the outputs keep unit
+    variance) and r is 1."""
+    rng = np.random.default_rng([w.seed, 505])
+    sc = channel_scales(w).astype(np.float64)
+    rms_role = np.sqrt(np.mean(sc ** 2, axis=(0, 2)))  # per role
+    r = (rms_role[None, :] * rng.uniform(0.9, 1.1, size=(w.L_r, 2))).astype(np.float32)
     g = torch.Generator(device=device)
     g.manual_seed(int(w.seed) * 1000 + 404)
     std = 1.0 / math.sqrt(w.K)
     W = torch.empty((w.L_r, 2, w.d_r, w.K), dtype=w.torch_dtype, device=device)
     for l in range(w.L_r):
         for c in range(2):
-            W[l, c] = (torch.randn((w.d_r, w.K), generator=g, device=device) * std).to(w.torch_dtype)
+            scale = std / float(r[l, c]) if w.kv_ridge else std
+            W[l, c] = (torch.randn((w.d_r, w.K), generator=g, device=device) * scale).to(w.torch_dtype)
     b = torch.randn((w.L_r, 2, w.d_r), generator=g, device=device, dtype=torch.float32) * 0.1
-    rng = np.random.default_rng([w.seed, 505])
-    sc = channel_scales(w).astype(np.float64)
-    rms_role = np.sqrt(np.mean(sc ** 2, axis=(0, 2)))  # per role
-    r = (rms_role[None, :] * rng.uniform(0.9, 1.1, size=(w.L_r, 2))).astype(np.float32)
+    if w.kv_ridge:
+        r = np.ones((w.L_r, 2), np.float32)
     return W, b, r
 
 

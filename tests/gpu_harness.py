@@ -59,8 +59,35 @@ class MapFetcher:
         return MapFetcher._L(self.W[l])
 
 
+class HeadMapFetcher:
+    """W_h[l][c][h] = the per-head map of receiver head h: columns
+    h D_r .. (h+1) D_r - 1 of A = W[l][c]^T, as fp64 numpy."""
+
+    def __init__(self, Wm: torch.Tensor, H_r: int, D_r: int):
+        self.W, self.H, self.D = Wm, H_r, D_r
+
+    def __getitem__(self, l):
+        W, D = self.W, self.D
+
+        class _LC:
+            def __getitem__(_, c):
+                A = W[l][c].float().cpu().numpy().T
+                return [A[:, h * D:(h + 1) * D] for h in range(A.shape[1] // D)]
+        return _LC()
+
+
+class HeadBiasFetcher:
+    """b_h[l][c][h] = the bias of receiver head h, fp64 numpy."""
+
+    def __init__(self, b: torch.Tensor, H_r: int, D_r: int):
+        self.b = b.double().cpu().numpy().reshape(b.shape[0], 2, H_r, D_r)
+
+    def __getitem__(self, l):
+        return self.b[l]
+
+
 class Case:
-    def __init__(self, w: W.Workload, device="cuda", sentinel=None):
+    def __init__(self, w: W.Workload, device="cuda", sentinel=None, **desc_options):
         self.w = w
         self.dev = torch.device(device)
         self.tok = W.tokens(w)
@@ -71,7 +98,8 @@ class Case:
         self.r_pos0 = W.r_pos0(w)
         self.job = pipeline.job_from_workload(w, self.tok, self.sender, self.Wm, self.b, self.r,
                                               paged=self.paged, knorm_w=self.knorm_w,
-                                              r_pos0=self.r_pos0, device=self.dev)
+                                              r_pos0=self.r_pos0, device=self.dev,
+                                              **desc_options)
         if sentinel is not None:
             self.job.receiver.fill_(sentinel)
         self.csr = O.alignment_csr(w.align_mode, self.tok.s_tok_ptr, self.tok.r_tok_ptr,
@@ -120,6 +148,14 @@ class Case:
         return y.reshape(len(rows), self.w.H_r, self.w.D_r)
 
     def oracle(self, layers, rows, roles=(0, 1)):
+        if self.w.kv_ridge:  # the per-head formulation, against the stacked map on the GPU
+            selected = [[t[0] for t in seg] for seg in self.w.seg_layer]
+            return O.kv_ridge_transfer(RowFetcher(self.sender), self.csr, selected,
+                                       HeadMapFetcher(self.Wm, self.w.H_r, self.w.D_r),
+                                       HeadBiasFetcher(self.b, self.w.H_r, self.w.D_r),
+                                       H_r=self.w.H_r, D_r=self.w.D_r, pos=self.pos,
+                                       inv_freq_r=self.inv_freq_r, layers=layers, rows=rows,
+                                       roles=roles)
         return O.transfer(RowFetcher(self.sender), self.csr, self.segs, MapFetcher(self.Wm),
                           self.b.cpu().numpy(), self.r, H_r=self.w.H_r, D_r=self.w.D_r,
                           pos=self.pos, inv_freq_r=self.inv_freq_r,

@@ -212,6 +212,26 @@ def check_mapper_size_table_f():
         assert sum(2 * (len(s) * int(ds) * int(dr) + int(dr)) for s in segs) == n
 
 
+def check_mapper_size_table_f_kv_ridge():
+    """Appendix F's Table, KV Ridge column: per receiver layer, role and
+    receiver head, one map from the concatenated KV heads of k = 8 sender
+    layers (8 H_S D_S inputs) to D_R outputs, plus a D_R bias.  Maps that
+    read only the matching sender head (block-diagonal) would store H_S times
+    fewer parameters and miss every entry of the column."""
+    g = _read_golden("mapper_size_table_f_kv_ridge.txt")
+    for row in g["_rows"]:
+        _, _, _Ls, Lr, Hs, Ds, Hr, Dr, millions = row
+        Lr, Hs, Ds, Hr, Dr = int(Lr), int(Hs), int(Ds), int(Hr), int(Dr)
+        k = O.KV_RIDGE_K
+        per_head = k * Hs * Ds * Dr + Dr
+        n = 2 * Lr * Hr * per_head
+        assert round(n / 1e6) == int(millions), (row, n)
+        # the same count as one stacked [k d_S, d_R] map per layer and role
+        assert O.mapper_parameter_count(Lr, Hs * Ds, Hr * Dr, n_seg=k) == n
+        block_diag = 2 * Lr * Hr * (k * Ds * Dr + Dr)
+        assert round(block_diag / 1e6) != int(millions)
+
+
 # ---------------------------------------------------------------------------
 # RoPE and key norm
 # ---------------------------------------------------------------------------
@@ -490,6 +510,73 @@ def check_explicit_segments():
     assert np.allclose(y.reshape(len(rows), -1), ref1)
 
 
+def _kv_ridge_problem(seed, align_mode, L_s=5, L_r=3, H_s=2, D_s=4, H_r=2, D_r=4, k=3):
+    P = _tiny_problem(seed, align_mode, O.LAYER_PAPER3, L_s=L_s, L_r=L_r, H_s=H_s, D_s=D_s,
+                      H_r=H_r, D_r=D_r)
+    rng = np.random.default_rng(seed + 100)
+    sel = [sorted(rng.choice(L_s, size=k, replace=False).tolist()) for _ in range(L_r)]
+    Kin = k * H_s * D_s
+    Wh = rng.normal(size=(L_r, 2, H_r, Kin, D_r)) / math.sqrt(Kin)
+    bh = rng.normal(size=(L_r, 2, H_r, D_r)) * 0.1
+    return P, sel, Wh, bh
+
+
+def check_kv_ridge_brute_force():
+    """The KV Ridge apply element by element with Python loops: receiver head
+    h of layer l, role c at receiver row j is sum over the selected sender
+    layers s, every sender feature f (all heads) of the aligned token, of
+    x[s][f] * W_h[s * d_S + f][d], plus the head's bias; keys rotated."""
+    for seed, am in [(30, O.ALIGN_TA), (31, O.ALIGN_SAME_INDEX), (32, O.ALIGN_OVERLAP_MEAN)]:
+        P, sel, Wh, bh = _kv_ridge_problem(seed, am)
+        sender, csr, d_s = P["sender"], P["csr"], P["d_s"]
+        H_r, D_r, inv, pos = P["H_r"], P["D_r"], P["inv"], P["pos"]
+        got = O.kv_ridge_transfer(sender, csr, sel, Wh, bh, H_r=H_r, D_r=D_r, pos=pos,
+                                  inv_freq_r=inv)
+        for l in range(len(sel)):
+            for c in (0, 1):
+                for j in range(csr.n_rows):
+                    y = np.zeros((H_r, D_r))
+                    for h in range(H_r):
+                        for d in range(D_r):
+                            acc = bh[l, c, h, d]
+                            for si, t in enumerate(sel[l]):
+                                for e in range(csr.row_ptr[j], csr.row_ptr[j + 1]):
+                                    for f in range(d_s):
+                                        acc += (csr.w[e] * sender[t, c, csr.col[e], f]
+                                                * Wh[l, c, h, si * d_s + f, d])
+                            y[h, d] = acc
+                    if c == 0:
+                        half = D_r // 2
+                        z = y.copy()
+                        for i in range(half):
+                            a = pos[j] * inv[i]
+                            z[:, i] = y[:, i] * math.cos(a) - y[:, i + half] * math.sin(a)
+                            z[:, i + half] = y[:, i + half] * math.cos(a) + y[:, i] * math.sin(a)
+                        y = z
+                    assert np.allclose(got[(l, c)][j], y, rtol=1e-10, atol=1e-10), (seed, l, c, j)
+
+
+def check_kv_ridge_equals_stacked_map():
+    """The per-head maps stacked column-wise (head-major, h * D_R + d) are one
+    dense [k d_S, d_R] map: the KV Ridge apply equals transfer() with the
+    k one-layer segments, that map, the stacked biases and r = 1."""
+    for seed, am in [(33, O.ALIGN_TA), (34, O.ALIGN_OVERLAP_MEAN)]:
+        P, sel, Wh, bh = _kv_ridge_problem(seed, am, L_s=9, L_r=4, k=8)
+        H_r, D_r = P["H_r"], P["D_r"]
+        L_r = len(sel)
+        A = np.concatenate([Wh[:, :, h] for h in range(H_r)], axis=-1)  # [L_r, 2, K, d_R]
+        b = bh.reshape(L_r, 2, H_r * D_r)
+        ridge = O.kv_ridge_transfer(P["sender"], P["csr"], sel, Wh, bh, H_r=H_r, D_r=D_r,
+                                    pos=P["pos"], inv_freq_r=P["inv"])
+        segs = O.kv_ridge_segments(sel)
+        assert all(len(sg) == 8 and all(len(t) == 1 and t[0][1] == 1.0 for t in sg)
+                   for sg in segs)
+        dense = O.transfer(P["sender"], P["csr"], segs, A, b, np.ones((L_r, 2)), H_r=H_r,
+                           D_r=D_r, pos=P["pos"], inv_freq_r=P["inv"])
+        for key in ridge:
+            assert np.allclose(ridge[key], dense[key], rtol=1e-12, atol=1e-12), (seed, key)
+
+
 def check_identity_map_reproduces_input():
     """Same depth, same tokenisation, A = [0; I; 0] (the middle block reads
     sender layer pi(l) = l), b = 0, r = 1: V is the sender V, K is the sender K
@@ -759,7 +846,8 @@ ALL_CHECKS = [
     check_ta_worked_example, check_ta_literal_shared_boundary, check_ta_brute_force,
     check_ta_identity, check_same_index, check_overlap_brute_force, check_csr_batching,
     check_layer_alignment_closed_form, check_layer_alignment_hand_tables,
-    check_layer_interpolation, check_mapper_size_table_f,
+    check_layer_interpolation, check_mapper_size_table_f, check_mapper_size_table_f_kv_ridge,
+    check_kv_ridge_brute_force, check_kv_ridge_equals_stacked_map,
     check_rope_two_dim_rotation, check_rope_complex_form, check_rope_relative_position,
     check_rope_inverse, check_inv_freq, check_key_norm,
     check_transfer_brute_force, check_transfer_brute_force_rotated_sender,

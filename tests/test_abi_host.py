@@ -64,7 +64,7 @@ def _desc(B, **over):
     (dict(paged=True, block_size=16, n_blocks=0), 1),  # paged layout incomplete
     (dict(d_W=None), 1),
     # optional fields
-    (dict(layer_mode="explicit", seg_layer=np.zeros((6, 4, 1)), seg_w=1.0), 1),   # n_seg > 3
+    (dict(layer_mode="explicit", seg_layer=np.zeros((6, 9, 1)), seg_w=1.0), 1),   # n_seg > 8
     (dict(layer_mode="explicit", seg_layer=np.zeros((6, 2, 3)), seg_w=1.0), 1),   # n_terms > 2
     (dict(layer_mode="explicit", seg_layer=np.full((6, 2, 1), 4), seg_w=1.0), 1),  # layer >= L_s
     (dict(layer_mode="explicit", seg_layer=np.zeros((6, 1, 2)), seg_w=np.nan), 1),

@@ -103,6 +103,28 @@ def test_ministral_to_llama_sweep(T_r):
         c.check_parity(rows=sampled_rows(c.tok, 512, seed=T_r))
 
 
+# ---------------------------------------------------------------- KV Ridge apply
+# KV Ridge + TA (the paper's comparison system, Appendix A): eight selected
+# sender layers per receiver layer, one dense [8 d_S, d_R] map per layer and
+# role (the per-head maps stacked), no normaliser.  The kernel runs it as an
+# explicit eight-segment layer table; the oracle applies the per-head maps.
+def test_kv_ridge_ta_qwen25_to_llama_4k():
+    c = Case(W.qwen25_to_llama_kv_ridge(4096)).run()
+    c.check_csr()
+    assert c.job.plan is not None
+    c.check_parity(layers=whole_layers(c.w.L_r))
+    c.check_parity(rows=sampled_rows(c.tok, 1024, seed=8))
+    print(c.report())
+
+
+def test_kv_ridge_same_index_small():
+    """KV Ridge without TA pairs sender token i with receiver token i."""
+    c = Case(W.qwen25_to_llama_kv_ridge(700, align_mode="same_index").with_(r_tokens=(700,))
+             ).run()
+    c.check_csr()
+    c.check_parity(layers=[0, 7, 31])
+
+
 # ---------------------------------------------------------------- alignment CSR
 @pytest.mark.parametrize("mode", ["ta", "overlap_mean", "same_index"])
 @pytest.mark.parametrize("make", [lambda: W.llama_to_qwen25(4096), W.qwen25_to_llama_batched,
@@ -188,6 +210,10 @@ EDGE = {
     "interp_ta_bf16": lambda: W.llama_to_ministral(600).with_(L_s=5, L_r=7, layer_mode="interp"),
     "overlap_paper_bf16": lambda: W.llama_to_ministral(600).with_(L_s=5, L_r=4,
                                                                   align_mode="overlap_mean"),
+    # an eight-segment table with weights in [-1, 1]: eight computed segments
+    "explicit_eight_segments_built": lambda: _explicit(
+        W.qwen25_to_llama_kv_ridge(500).with_(L_s=9, L_r=3, kv_ridge=False), n_seg=8,
+        n_terms=1),
     "ta_paper_f32": lambda: W.llama_to_ministral(400).with_(L_s=4, L_r=3, dtype="f32"),
     "same_index": lambda: W.llama_to_ministral(500).with_(L_s=4, L_r=3, align_mode="same_index"),
     "d128_one_head": lambda: W.llama_to_ministral(333).with_(L_s=3, L_r=2, H_r=1, D_r=128),
@@ -242,6 +268,16 @@ def _explicit(w, n_seg, n_terms, unit=False):
 @pytest.mark.parametrize("name", sorted(EDGE))
 def test_edge_case(name):
     c = Case(EDGE[name]()).run()
+    c.check_csr()
+    c.check_parity()
+
+
+# Computed operand rows rounded once to bf16 (round_built_operands = 1):
+# the faster path, inside the tolerance at these sizes.
+@pytest.mark.parametrize("name", ["overlap_paper_bf16", "interp_ta_bf16", "rotated_sender_ta",
+                                  "rotated_sender_batched_paged", "explicit_two_terms"])
+def test_edge_case_rounded_operands(name):
+    c = Case(EDGE[name](), round_built_operands=True).run()
     c.check_csr()
     c.check_parity()
 

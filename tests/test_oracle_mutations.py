@@ -207,7 +207,28 @@ def _transfer_times_r(sender, csr, segments, A, b, r, **kw):
     return _orig_transfer(sender, csr, segments, A, b, r2, **kw)
 
 
+def _kv_ridge_segments_reversed(selected):
+    # wrong: the selected layers concatenated in reverse order
+    return [[[(int(t), 1.0)] for t in reversed(list(sel))] for sel in selected]
+
+
+_kv_ridge_ok = O.kv_ridge_transfer
+
+
+def _kv_ridge_rotates_values(sender, csr, selected, W_heads, b_heads, *, H_r, D_r, pos,
+                             inv_freq_r, **kw):
+    out = _kv_ridge_ok(sender, csr, selected, W_heads, b_heads, H_r=H_r, D_r=D_r, pos=pos,
+                       inv_freq_r=inv_freq_r, **kw)
+    rows = np.arange(csr.n_rows) if kw.get("rows") is None else np.asarray(kw["rows"])
+    for (l, c), y in out.items():
+        if c == O.ROLE_V:
+            out[(l, c)] = O.rope(y, np.asarray(pos)[rows], inv_freq_r)
+    return out
+
+
 MUTATIONS = {
+    "kv_ridge_segments_reversed": ("kv_ridge_segments", _kv_ridge_segments_reversed),
+    "kv_ridge_rotates_values": ("kv_ridge_transfer", _kv_ridge_rotates_values),
     "ta_any_sender_boundary": ("token_alignment", _ta_any_sender_boundary),
     "ta_next_boundary": ("token_alignment", _ta_next_boundary),
     "depth_floor": ("proportional_depth", _depth_floor),
