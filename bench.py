@@ -40,6 +40,8 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--round-built-operands", action="store_true",
+                    help="computed operand rows rounded once to bf16 (no value + residual pair)")
     return ap.parse_args()
 
 
@@ -247,6 +249,17 @@ class OracleSample:
                                H_r=w.H_r, D_r=w.D_r, pos=self.pos, inv_freq_r=self.inv)
 
 
+def _copied_operands(w):
+    """Every map input row is a copy of one sender row: one-entry alignment
+    rows, segments of one sender layer of weight 1, keys without RoPE."""
+    if w.align_mode == "overlap_mean" or w.layer_mode == "interp" or w.sender_k_rotated:
+        return False
+    if w.layer_mode == "explicit":
+        return all(len(terms) == 1 and float(terms[0]) == 1.0
+                   for layer in w.seg_w for terms in layer)
+    return True
+
+
 def blas_threads():
     for k in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
         v = os.environ.get(k)
@@ -335,7 +348,8 @@ def run_ours(args):
     sender = W.sender_kv(w, W.sender_cache_rows(w, tok), dev)
     Wm, b, r = W.maps(w, dev)
     paged = W.paged_layout(w, tok) if w.paged else None
-    job = pipeline.job_from_workload(w, tok, sender, Wm, b, r, paged=paged, device=dev)
+    job = pipeline.job_from_workload(w, tok, sender, Wm, b, r, paged=paged, device=dev,
+                                     round_built_operands=args.round_built_operands)
     stream = torch.cuda.current_stream(dev)
 
     for _ in range(max(3, args.warmup)):
@@ -515,6 +529,10 @@ def run_ours(args):
                    "distinct_rows": U, "sender": f"{w.L_s}x{w.H_s}x{w.D_s}",
                    "receiver": f"{w.L_r}x{w.H_r}x{w.D_r}",
                    "mode": f"{w.align_mode}+{w.layer_mode}",
+                   "operands": ("copied sender rows" if _copied_operands(w)
+                                else "computed rows rounded once to bf16"
+                                if args.round_built_operands or w.dtype != "bf16"
+                                else "computed rows as bf16 value + residual"),
                    "l2": ("inputs larger than L2 (no flush)" if flush is None else
                           "256 MB L2 flush write between steps (outside the timed events)"),
                    "parallelism": "replicas" if world > 1 else "single"},

@@ -398,12 +398,12 @@ hf_status hf_fold(hf_dtype dtype, int32_t n_maps, int32_t d_R, int64_t K, int32_
  *       roots of Sigma_Z and Sigma_Y and by the polar factor.
  * d_workspace: hf_recolor_workspace_size bytes, 256-byte aligned.
  * Requires d_S >= d_R and N * d_S < 2^31.  Matrix roots and the polar
- * factor use Newton-Schulz iterations in fp32; the matrix products go to
- * cuBLAS with fp32 emulated on the tensor cores (fp32 accuracy), through a
- * per-device handle created on the first call (calls on one device are
- * serialised).  The call synchronises `stream` (convergence checks) and
- * returns HF_ERR_DEVICE_CHECK if an iteration does not converge (raise
- * reg), HF_ERR_CUDA if cuBLAS fails.
+ * factor use Newton-Schulz iterations in fp32; the matrix products run on
+ * this library's tcgen05 kernel in fp32 accuracy (each fp32 operand split
+ * exactly into three bf16 parts, the six largest partial products summed in
+ * an fp32 tensor-memory accumulator).  The call synchronises `stream`
+ * (convergence checks) and returns HF_ERR_DEVICE_CHECK if an iteration does
+ * not converge (raise reg) or a product kernel's wait ran out.
  */
 hf_status hf_recolor_workspace_size(int64_t N, int32_t d_S, int32_t d_R, size_t* bytes);
 hf_status hf_recolor_fit(hf_dtype dtype, int64_t N, int32_t d_S, int32_t d_R, const void* d_X,
@@ -427,6 +427,24 @@ const char* hf_last_error(void);
  */
 hf_status hf_debug_transfer_stalled(hf_plan plan, const void* sender_kv, void* receiver_kv,
                                     hf_stream_t stream);
+
+/*
+ * Test hook for the fp32 product kernel behind hf_recolor_fit (not part of
+ * the method): C[M x N] = alpha op(A) op(B) + beta C on the tensor cores in
+ * fp32 accuracy (each operand split exactly into three bf16 parts, the six
+ * largest partial products summed in fp32).  Row-major C with leading
+ * dimension ldc >= N; op(A)(i, k) = d_A[i * a_i + k * a_k] (i < M, k < K),
+ * op(B)(k, j) = d_B[k * b_k + j * b_j] (j < N): strides express transposes.
+ * d_workspace: hf_debug_matmul_workspace_size bytes, 256-byte aligned.
+ * h_err (or NULL): synchronises `stream` and returns the kernel's error word
+ * (0: clean; nonzero: a pipeline wait ran out).  Asynchronous otherwise.
+ */
+hf_status hf_debug_matmul_workspace_size(int32_t M, int32_t N, int32_t K, size_t* bytes);
+hf_status hf_debug_matmul_f32(int32_t M, int32_t N, int32_t K, float alpha, const float* d_A,
+                              int64_t a_i, int64_t a_k, const float* d_B, int64_t b_k,
+                              int64_t b_j, float beta, float* d_C, int64_t ldc,
+                              void* d_workspace, size_t workspace_bytes, int32_t* h_err,
+                              hf_stream_t stream);
 
 #ifdef __cplusplus
 }

@@ -39,7 +39,8 @@ EXPORTED = ("hf_align_build", "hf_plan_workspace_size", "hf_plan_create", "hf_tr
             "hf_plan_destroy", "hf_plan_device_status", "hf_plan_distinct_rows",
             "hf_status_string", "hf_last_error", "hf_transfer_noalloc", "hf_transfer_host",
             "hf_transfer_batch", "hf_fold", "hf_recolor_workspace_size", "hf_recolor_fit",
-            "hf_debug_transfer_stalled")
+            "hf_debug_transfer_stalled", "hf_debug_matmul_workspace_size",
+            "hf_debug_matmul_f32")
 
 _p = ctypes.c_void_p
 _i32p = ctypes.POINTER(ctypes.c_int32)
@@ -115,6 +116,14 @@ def lib() -> ctypes.CDLL:
                                      _p, _p, _p, ctypes.c_float, _p, _p, _f32p, _i32p, _p,
                                      ctypes.c_size_t, _p]
         L.hf_recolor_fit.restype = ctypes.c_int
+        L.hf_debug_matmul_workspace_size.argtypes = [ctypes.c_int32, ctypes.c_int32,
+                                                     ctypes.c_int32, ctypes.POINTER(ctypes.c_size_t)]
+        L.hf_debug_matmul_workspace_size.restype = ctypes.c_int
+        L.hf_debug_matmul_f32.argtypes = [ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
+                                          ctypes.c_float, _p, ctypes.c_int64, ctypes.c_int64, _p,
+                                          ctypes.c_int64, ctypes.c_int64, ctypes.c_float, _p,
+                                          ctypes.c_int64, _p, ctypes.c_size_t, _i32p, _p]
+        L.hf_debug_matmul_f32.restype = ctypes.c_int
         L.hf_status_string.argtypes = [ctypes.c_int]
         L.hf_status_string.restype = ctypes.c_char_p
         L.hf_last_error.argtypes = []
@@ -351,3 +360,22 @@ def status_string(status: int) -> str:
 
 def decode_check_bits(bits: int):
     return [name for b, name in CHECK_BITS.items() if bits & b]
+
+
+def debug_matmul_f32(A, a_strides, B, b_strides, C, M, N, K, alpha=1.0, beta=0.0,
+                     stream=None) -> int:
+    """Test hook: C = alpha op(A) op(B) + beta C through hf_debug_matmul_f32;
+    a_strides = (a_i, a_k), b_strides = (b_k, b_j) in elements; returns the
+    kernel's error word (0 = clean)."""
+    import torch
+    n = ctypes.c_size_t(0)
+    _check(lib().hf_debug_matmul_workspace_size(int(M), int(N), int(K), ctypes.byref(n)),
+           "hf_debug_matmul_workspace_size")
+    ws = torch.empty(int(n.value), dtype=torch.uint8, device=C.device)
+    err = np.zeros(1, np.int32)
+    _check(lib().hf_debug_matmul_f32(int(M), int(N), int(K), float(alpha), _dptr(A),
+                                     int(a_strides[0]), int(a_strides[1]), _dptr(B),
+                                     int(b_strides[0]), int(b_strides[1]), float(beta), _dptr(C),
+                                     int(C.stride(0)), _dptr(ws), int(n.value), _as_i32p(err),
+                                     _stream(stream)), "hf_debug_matmul_f32")
+    return int(err[0])

@@ -2,8 +2,8 @@
 
 Each translation unit compiles in its own nvcc process, in parallel, then
 one nvcc call links the shared library.  The CUDA runtime is linked
-statically, cuBLAS dynamically (from the toolkit, found through an rpath),
-and the driver's tensor-map encoder is fetched at run time, so the library
+statically and the driver's tensor-map encoder is fetched at run time (no
+other library is linked: every kernel is this library's own), so the library
 loads on a machine without a GPU driver (symbols can be inspected there;
 calls then fail with HF_ERR_CUDA).
 """
@@ -25,7 +25,7 @@ LIB_NAME = "libheterofold.so"
 LIB_PATH = os.path.join(PKG_DIR, LIB_NAME)
 
 SOURCES = ["hf_align.cu", "hf_plan.cu", "hf_transfer.cu", "hf_noalloc.cu", "hf_host.cu",
-           "hf_batch.cu", "hf_fold.cu", "hf_recolor.cu"]
+           "hf_batch.cu", "hf_fold.cu", "hf_recolor.cu", "hf_gemm.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",
          "--expt-relaxed-constexpr"]
@@ -50,12 +50,6 @@ def _stale(target: str, deps) -> bool:
         return True
     t = os.path.getmtime(target)
     return any(os.path.getmtime(d) > t for d in deps)
-
-
-def _link_libs(exe: str):
-    """cuBLAS (hf_recolor_fit's products), found beside the toolkit's nvcc."""
-    lib = os.path.join(os.path.dirname(os.path.dirname(os.path.realpath(exe))), "lib64")
-    return ["-L" + lib, "-lcublas", "-Xlinker", "-rpath=" + lib]
 
 
 def build(verbose: bool = False, force: bool = False, ptxas_info: bool = False) -> str:
@@ -83,7 +77,7 @@ def build(verbose: bool = False, force: bool = False, ptxas_info: bool = False) 
             sys.stdout.write(out)
     if force or jobs or _stale(LIB_PATH, objs):
         tmp = LIB_PATH + ".tmp"
-        _run([exe, *ARCH, "-shared", "-o", tmp, *objs, *_link_libs(exe)])
+        _run([exe, *ARCH, "-shared", "-o", tmp, *objs])
         os.replace(tmp, LIB_PATH)
     return LIB_PATH
 

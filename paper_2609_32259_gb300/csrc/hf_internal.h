@@ -125,6 +125,27 @@ bool batch_compatible(const hf_plan_s* const* plans, int n);
 hf_status launch_transfer_batch(hf_plan_s* const* plans, const void* const* senders,
                                 void* const* receivers, int n, cudaStream_t stream);
 
+// Device buffers of gemm_f32 (part of hf_recolor_fit's workspace): the bf16
+// planes of both operands, split-K partials, and an error word (set when a
+// pipeline wait of the product kernel ran out).
+struct GemmWork {
+  void* planes_a;
+  size_t planes_a_bytes;
+  void* planes_b;
+  size_t planes_b_bytes;
+  float* partial;
+  size_t partial_bytes;
+  int32_t* err;
+};
+// Bytes of the three bf16 planes of an operand with `rows` rows and K columns.
+size_t gemm_planes_bytes(int64_t rows, int64_t K);
+// C[M x N] = alpha op(A) op(B) + beta C (row-major C, leading dimension ldc),
+// op(A)(i, k) = A[i * a_i + k * a_k], op(B)(k, j) = B[k * b_k + j * b_j], in
+// fp32 accuracy on the tensor cores (hf_gemm.cu).  Asynchronous on s.
+hf_status gemm_f32(cudaStream_t s, const GemmWork& wk, int M, int N, int K, float alpha,
+                   const float* A, int64_t a_i, int64_t a_k, const float* B, int64_t b_k,
+                   int64_t b_j, float beta, float* C, int64_t ldc);
+
 }  // namespace hf
 
 #define HF_CUDA_TRY(expr, what)                      \

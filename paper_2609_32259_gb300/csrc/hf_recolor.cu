@@ -10,18 +10,17 @@
 // Z_0 = I into (S / c)^{1/2} and (S / c)^{-1/2}; X <- X (3I - X^T X) / 2
 // turns X_0 = M / |M|_F into the orthogonal polar factor U Q^T of
 // M = U Lambda Q^T (full column rank), which is the R* of Eq. 4.
-// Offline (once per map, before folding).  The products are plain fp32
-// GEMMs and go to cuBLAS with fp32 emulated on the bf16 tensor cores (each
-// operand split into three bf16 parts, fp32 accumulation: fp32 accuracy);
-// the statistics, centring and elementwise passes are this file's kernels.
+// Offline (once per map, before folding).  The products are fp32 GEMMs on
+// this library's tcgen05 kernel (hf_gemm.cu: each operand split exactly into
+// three bf16 parts, six partial products in an fp32 accumulator: fp32
+// accuracy); the statistics, centring and elementwise passes are this file's
+// kernels.
 #include <algorithm>
 #include <cmath>
 #include <cstring>
-#include <mutex>
 #include <string>
 #include <utility>
 
-#include <cublas_v2.h>
 #include <cuda_bf16.h>
 
 #include "hf_internal.h"
@@ -29,54 +28,29 @@
 namespace hf {
 namespace {
 
-constexpr int kMaxDevices = 64;
-std::mutex g_blas_mutex[kMaxDevices];
-cublasHandle_t g_blas[kMaxDevices] = {};
+// The moments' products run over the samples in chunks of this many, so the
+// bf16 planes of their operands stay a bounded part of the workspace.
+constexpr int64_t kMomentChunk = 8192;
+// Split-K partials: room for every SM pair's 256 x 256 tile twice over.
+constexpr size_t kPartialBytes = static_cast<size_t>(2) * 96 * 65536 * sizeof(float);
 
-hf_status blas_fail(cublasStatus_t st, const char* what) {
-  set_error(std::string("hf_recolor_fit: ") + what + " (cuBLAS status " +
-            std::to_string(static_cast<int>(st)) + ")");
-  return HF_ERR_CUDA;
+hf_status sgemm(const GemmWork& h, cudaStream_t s, int M, int N, int K, float alpha,
+                const float* A, int64_t a_i, int64_t a_k, const float* B, int64_t b_k,
+                int64_t b_j, float beta, float* C, int64_t ldc) {
+  return gemm_f32(s, h, M, N, K, alpha, A, a_i, a_k, B, b_k, b_j, beta, C, ldc);
 }
 
-// The current device's cuBLAS handle (created on first use, fp32 products
-// emulated on the tensor cores whenever possible).  Callers hold
-// g_blas_mutex[dev] while they use it.
-hf_status blas_handle(int dev, cublasHandle_t* out) {
-  if (!g_blas[dev]) {
-    cublasHandle_t h = nullptr;
-    cublasStatus_t st = cublasCreate(&h);
-    if (st != CUBLAS_STATUS_SUCCESS) return blas_fail(st, "cublasCreate");
-    st = cublasSetEmulationStrategy(h, CUBLAS_EMULATION_STRATEGY_EAGER);
-    if (st != CUBLAS_STATUS_SUCCESS) {
-      cublasDestroy(h);
-      return blas_fail(st, "cublasSetEmulationStrategy");
-    }
-    g_blas[dev] = h;
+// A product over the sample axis (K = N samples) in chunks of kMomentChunk:
+// C = alpha sum_chunks op(A_c) op(B_c).
+hf_status moment_product(const GemmWork& h, cudaStream_t s, int M, int N, int64_t K,
+                         const float* A, int64_t a_i, int64_t a_k, const float* B, int64_t b_k,
+                         int64_t b_j, float* C, int64_t ldc) {
+  for (int64_t k0 = 0; k0 < K; k0 += kMomentChunk) {
+    const int kc = static_cast<int>(std::min<int64_t>(kMomentChunk, K - k0));
+    const hf_status st = sgemm(h, s, M, N, kc, 1.f, A + k0 * a_k, a_i, a_k, B + k0 * b_k, b_k,
+                               b_j, k0 == 0 ? 0.f : 1.f, C, ldc);
+    if (st != HF_OK) return st;
   }
-  *out = g_blas[dev];
-  return HF_OK;
-}
-
-// C[M x N] = alpha * op(A) op(B) + beta * C, row-major C with leading
-// dimension ldc; op(A)(i, k) = A[i * a_i + k * a_k], op(B)(k, j) =
-// B[k * b_k + j * b_j], one of each operand's two strides being 1 (strides
-// express transposes).  cuBLAS is column-major: the row-major C is the
-// column-major C^T = op(B)^T op(A)^T, so B goes first.
-hf_status sgemm(cublasHandle_t h, int M, int N, int K, float alpha, const float* A, int64_t a_i,
-                int64_t a_k, const float* B, int64_t b_k, int64_t b_j, float beta, float* C,
-                int64_t ldc) {
-  // op(B)^T (N x K): column-major B with ld b_k when b_j == 1, else B^T
-  const cublasOperation_t tb = b_j == 1 ? CUBLAS_OP_N : CUBLAS_OP_T;
-  const int64_t ldb = b_j == 1 ? b_k : b_j;
-  // op(A)^T (K x M): column-major A with ld a_i when a_k == 1, else A^T
-  const cublasOperation_t ta = a_k == 1 ? CUBLAS_OP_N : CUBLAS_OP_T;
-  const int64_t lda = a_k == 1 ? a_i : a_k;
-  const cublasStatus_t st =
-      cublasGemmEx(h, tb, ta, N, M, K, &alpha, B, CUDA_R_32F, static_cast<int>(ldb), A,
-                   CUDA_R_32F, static_cast<int>(lda), &beta, C, CUDA_R_32F, static_cast<int>(ldc),
-                   CUBLAS_COMPUTE_32F_EMULATED_16BFX9, CUBLAS_GEMM_DEFAULT);
-  if (st != CUBLAS_STATUS_SUCCESS) return blas_fail(st, "product");
   return HF_OK;
 }
 
@@ -194,7 +168,8 @@ __global__ void rc_output_kernel(const float* A, int dx, int dy, const double* s
 
 struct Rc {
   size_t stats, mu, xc, yc, sz, sy, szy, p1, p2, p3, p4, sz_ih, sy_ih, sy_h, m, x1, x2, xtx, a,
-      total;
+      planes_a, planes_b, partial, err, total;
+  size_t planes_bytes;
 };
 
 Rc rc_layout(int64_t N, int dx, int dy) {
@@ -226,6 +201,14 @@ Rc rc_layout(int64_t N, int dx, int dy) {
   L.x2 = take(f * dx * dy);
   L.xtx = take(f * dy * dy);
   L.a = take(f * dx * dy);
+  // bf16 planes of the products' operands: rows up to max(d_S, d_R), K up
+  // to max(d_S, one chunk of samples)
+  const int64_t kmax = std::max<int64_t>(dx, std::min<int64_t>(N, kMomentChunk));
+  L.planes_bytes = gemm_planes_bytes(static_cast<int64_t>(dmax), kmax);
+  L.planes_a = take(L.planes_bytes);
+  L.planes_b = take(L.planes_bytes);
+  L.partial = take(kPartialBytes);
+  L.err = take(sizeof(int32_t));
   L.total = off;
   return L;
 }
@@ -249,7 +232,7 @@ bool converged(double e, double* prev) {
 
 // Newton-Schulz square root and inverse square root of the SPD matrix S
 // (d x d): root = S^{1/2}, inv_root = S^{-1/2}.  Y, Z, T, U are d x d work.
-hf_status ns_sqrt(cudaStream_t s, cublasHandle_t h, const float* S, int d, float* Y, float* Z, float* T, float* U,
+hf_status ns_sqrt(cudaStream_t s, const GemmWork& h, const float* S, int d, float* Y, float* Z, float* T, float* U,
                   float* root, float* inv_root, double* dscr, int* iters) {
   const int64_t n_el = static_cast<int64_t>(d) * d;
   const int grid = 1024;
@@ -270,7 +253,7 @@ hf_status ns_sqrt(cudaStream_t s, cublasHandle_t h, const float* S, int d, float
   for (; it < kMaxIter; ++it) {
     // T = 1.5 I - 0.5 Z Y
     rc_affine_kernel<<<grid, 256, 0, s>>>(T, nullptr, n_el, d, 0.f, 1.5f);
-    if ((st = sgemm(h, d, d, d, -0.5f, Z, d, 1, Y, d, 1, 1.f, T, d)) != HF_OK) return st;
+    if ((st = sgemm(h, s, d, d, d, -0.5f, Z, d, 1, Y, d, 1, 1.f, T, d)) != HF_OK) return st;
     if (it % 4 == 3) {
       double e2 = 0.0;
       HF_CUDA_TRY(cudaMemsetAsync(dscr, 0, sizeof(double), s), "clear");
@@ -279,9 +262,9 @@ hf_status ns_sqrt(cudaStream_t s, cublasHandle_t h, const float* S, int d, float
       if ((st = read_double(s, dscr, &e2)) != HF_OK) return st;
       if (converged(2.0 * sqrt(e2 / d), &prev)) break;
     }
-    if ((st = sgemm(h, d, d, d, 1.f, Y, d, 1, T, d, 1, 0.f, U, d)) != HF_OK) return st;  // Y T
+    if ((st = sgemm(h, s, d, d, d, 1.f, Y, d, 1, T, d, 1, 0.f, U, d)) != HF_OK) return st;  // Y T
     std::swap(Y, U);
-    if ((st = sgemm(h, d, d, d, 1.f, T, d, 1, Z, d, 1, 0.f, U, d)) != HF_OK) return st;  // T Z
+    if ((st = sgemm(h, s, d, d, d, 1.f, T, d, 1, Z, d, 1, 0.f, U, d)) != HF_OK) return st;  // T Z
     std::swap(Z, U);
   }
   *iters = it;
@@ -295,7 +278,7 @@ hf_status ns_sqrt(cudaStream_t s, cublasHandle_t h, const float* S, int d, float
 // Orthogonal polar factor of M (dx x dy, dx >= dy, full column rank):
 // X <- X (3I - X^T X) / 2 from X_0 = M / |M|_F.  Result in *out (one of the
 // two buffers).
-hf_status ns_polar(cudaStream_t s, cublasHandle_t h, const float* M, int dx, int dy, float* X, float* X2,
+hf_status ns_polar(cudaStream_t s, const GemmWork& h, const float* M, int dx, int dy, float* X, float* X2,
                    float* P, double* dscr, float** out, int* iters) {
   const int64_t n_el = static_cast<int64_t>(dx) * dy, p_el = static_cast<int64_t>(dy) * dy;
   const int grid = 1024;
@@ -313,7 +296,7 @@ hf_status ns_polar(cudaStream_t s, cublasHandle_t h, const float* M, int dx, int
   double prev = 1e30;
   for (; it < kMaxIter; ++it) {
     // P = X^T X
-    if ((st = sgemm(h, dy, dy, dx, 1.f, X, 1, dy, X, dy, 1, 0.f, P, dy)) != HF_OK) return st;
+    if ((st = sgemm(h, s, dy, dy, dx, 1.f, X, 1, dy, X, dy, 1, 0.f, P, dy)) != HF_OK) return st;
     if (it % 4 == 3) {
       double e2 = 0.0;
       HF_CUDA_TRY(cudaMemsetAsync(dscr, 0, sizeof(double), s), "clear");
@@ -323,7 +306,7 @@ hf_status ns_polar(cudaStream_t s, cublasHandle_t h, const float* M, int dx, int
     }
     // X2 = 1.5 X - 0.5 X P
     rc_affine_kernel<<<grid, 256, 0, s>>>(X2, X, n_el, dy, 1.5f, 0.f);
-    if ((st = sgemm(h, dx, dy, dy, -0.5f, X, dy, 1, P, dy, 1, 1.f, X2, dy)) != HF_OK) return st;
+    if ((st = sgemm(h, s, dx, dy, dy, -0.5f, X, dy, 1, P, dy, 1, 1.f, X2, dy)) != HF_OK) return st;
     std::swap(X, X2);
   }
   *iters = it;
@@ -335,7 +318,7 @@ hf_status ns_polar(cudaStream_t s, cublasHandle_t h, const float* M, int dx, int
 template <typename T>
 hf_status recolor_typed(int64_t N, int dx, int dy, const void* Xv, const void* Yv, const float* w,
                         float reg, void* W_out, float* b_out, float* h_r, int32_t* h_iters,
-                        char* ws, cudaStream_t s, cublasHandle_t h) {
+                        char* ws, cudaStream_t s) {
   const Rc L = rc_layout(N, dx, dy);
   double* stats = reinterpret_cast<double*>(ws + L.stats);
   double* sx = stats;
@@ -345,6 +328,14 @@ hf_status recolor_typed(int64_t N, int dx, int dy, const void* Xv, const void* Y
   auto F = [&](size_t off) { return reinterpret_cast<float*>(ws + off); };
   const T* X = static_cast<const T*>(Xv);
   const T* Y = static_cast<const T*>(Yv);
+  GemmWork h;
+  h.planes_a = ws + L.planes_a;
+  h.planes_b = ws + L.planes_b;
+  h.planes_a_bytes = h.planes_b_bytes = L.planes_bytes;
+  h.partial = F(L.partial);
+  h.partial_bytes = kPartialBytes;
+  h.err = reinterpret_cast<int32_t*>(ws + L.err);
+  HF_CUDA_TRY(cudaMemsetAsync(h.err, 0, sizeof(int32_t), s), "clear");
   HF_CUDA_TRY(cudaMemsetAsync(stats, 0, sizeof(double) * (dx + dy + 4), s), "clear");
   const int d = dx + dy;
   dim3 sgrid((d + 255) / 256, static_cast<unsigned>(std::min<int64_t>(N, 256)));
@@ -355,11 +346,11 @@ hf_status recolor_typed(int64_t N, int dx, int dy, const void* Xv, const void* Y
   HF_CUDA_TRY(cudaGetLastError(), "hf_recolor_fit: moments launch");
   hf_status st;
   // Sigma_Z = Xc^T Xc, Sigma_Y = Yc^T Yc, Sigma_ZY = Xc^T Yc
-  if ((st = sgemm(h, dx, dx, N, 1.f, F(L.xc), 1, dx, F(L.xc), dx, 1, 0.f, F(L.sz), dx)) != HF_OK)
+  if ((st = moment_product(h, s, dx, dx, N, F(L.xc), 1, dx, F(L.xc), dx, 1, F(L.sz), dx)) != HF_OK)
     return st;
-  if ((st = sgemm(h, dy, dy, N, 1.f, F(L.yc), 1, dy, F(L.yc), dy, 1, 0.f, F(L.sy), dy)) != HF_OK)
+  if ((st = moment_product(h, s, dy, dy, N, F(L.yc), 1, dy, F(L.yc), dy, 1, F(L.sy), dy)) != HF_OK)
     return st;
-  if ((st = sgemm(h, dx, dy, N, 1.f, F(L.xc), 1, dx, F(L.yc), dy, 1, 0.f, F(L.szy), dy)) != HF_OK)
+  if ((st = moment_product(h, s, dx, dy, N, F(L.xc), 1, dx, F(L.yc), dy, 1, F(L.szy), dy)) != HF_OK)
     return st;
   if (reg > 0.f) {
     rc_ridge_kernel<<<1, 256, 0, s>>>(F(L.sz), dx, reg);
@@ -373,24 +364,31 @@ hf_status recolor_typed(int64_t N, int dx, int dy, const void* Xv, const void* Y
                     dscr, &it2)) != HF_OK)
     return st;
   // M = Sigma_Z^{-1/2} Sigma_ZY Sigma_Y^{-1/2}
-  if ((st = sgemm(h, dx, dy, dx, 1.f, F(L.sz_ih), dx, 1, F(L.szy), dy, 1, 0.f, F(L.x2), dy)) != HF_OK)
+  if ((st = sgemm(h, s, dx, dy, dx, 1.f, F(L.sz_ih), dx, 1, F(L.szy), dy, 1, 0.f, F(L.x2), dy)) != HF_OK)
     return st;
-  if ((st = sgemm(h, dx, dy, dy, 1.f, F(L.x2), dy, 1, F(L.sy_ih), dy, 1, 0.f, F(L.m), dy)) != HF_OK)
+  if ((st = sgemm(h, s, dx, dy, dy, 1.f, F(L.x2), dy, 1, F(L.sy_ih), dy, 1, 0.f, F(L.m), dy)) != HF_OK)
     return st;
   float* R = nullptr;
   if ((st = ns_polar(s, h, F(L.m), dx, dy, F(L.x1), F(L.x2), F(L.xtx), dscr, &R, &it3)) != HF_OK)
     return st;
   // A = Sigma_Z^{-1/2} R* Sigma_Y^{1/2}
   float* tmp = R == F(L.x1) ? F(L.x2) : F(L.x1);
-  if ((st = sgemm(h, dx, dy, dx, 1.f, F(L.sz_ih), dx, 1, R, dy, 1, 0.f, tmp, dy)) != HF_OK) return st;
-  if ((st = sgemm(h, dx, dy, dy, 1.f, tmp, dy, 1, F(L.sy_h), dy, 1, 0.f, F(L.a), dy)) != HF_OK)
+  if ((st = sgemm(h, s, dx, dy, dx, 1.f, F(L.sz_ih), dx, 1, R, dy, 1, 0.f, tmp, dy)) != HF_OK) return st;
+  if ((st = sgemm(h, s, dx, dy, dy, 1.f, tmp, dy, 1, F(L.sy_h), dy, 1, 0.f, F(L.a), dy)) != HF_OK)
     return st;
   rc_output_kernel<T><<<1024, 256, 0, s>>>(F(L.a), dx, dy, sx, sy, sw_ss, static_cast<T*>(W_out),
                                            b_out);
   HF_CUDA_TRY(cudaGetLastError(), "hf_recolor_fit: output launch");
   double hs[2];
+  int32_t gemm_err = 0;
   HF_CUDA_TRY(cudaMemcpyAsync(hs, sw_ss, sizeof(hs), cudaMemcpyDeviceToHost, s), "read back");
+  HF_CUDA_TRY(cudaMemcpyAsync(&gemm_err, h.err, sizeof(gemm_err), cudaMemcpyDeviceToHost, s),
+              "read back");
   HF_CUDA_TRY(cudaStreamSynchronize(s), "synchronize");
+  if (gemm_err != 0) {
+    set_error("hf_recolor_fit: a product kernel's pipeline wait ran out (internal error)");
+    return HF_ERR_DEVICE_CHECK;
+  }
   if (h_r) *h_r = static_cast<float>(std::sqrt(hs[1] / (static_cast<double>(dx) * hs[0])));
   if (h_iters) {
     h_iters[0] = it1;
@@ -444,23 +442,9 @@ extern "C" hf_status hf_recolor_fit(hf_dtype dtype, int64_t N, int32_t d_S, int3
   }
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream_);
   char* ws = static_cast<char*>(d_workspace);
-  int dev = 0;
-  HF_CUDA_TRY(cudaGetDevice(&dev), "hf_recolor_fit: current device");
-  if (dev < 0 || dev >= kMaxDevices) {
-    set_error("hf_recolor_fit: device ordinal out of range");
-    return HF_ERR_UNSUPPORTED;
-  }
-  // one fit at a time per device uses the device's handle (the call is
-  // synchronous: it waits for its convergence checks)
-  std::lock_guard<std::mutex> lock(g_blas_mutex[dev]);
-  cublasHandle_t h = nullptr;
-  hf_status st = blas_handle(dev, &h);
-  if (st != HF_OK) return st;
-  const cublasStatus_t bs = cublasSetStream(h, s);
-  if (bs != CUBLAS_STATUS_SUCCESS) return blas_fail(bs, "cublasSetStream");
   if (dtype == HF_BF16)
     return recolor_typed<__nv_bfloat16>(N, d_S, d_R, d_X, d_Y, d_w, reg, d_W_out, d_b_out,
-                                        h_r_out, h_iters_out, ws, s, h);
+                                        h_r_out, h_iters_out, ws, s);
   return recolor_typed<float>(N, d_S, d_R, d_X, d_Y, d_w, reg, d_W_out, d_b_out, h_r_out,
-                              h_iters_out, ws, s, h);
+                              h_iters_out, ws, s);
 }

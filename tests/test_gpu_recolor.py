@@ -73,3 +73,33 @@ def test_recolor_recovers_an_exact_rotation():
 def test_recolor_rejects_bad_shapes():
     with pytest.raises(B.HFError):
         B.recolor_workspace_size(100, 64, 128)   # d_S < d_R
+
+
+def test_recolor_at_the_benchmarked_shape():
+    """One map of the 32K Llama -> Ministral-shaped direction: 32,768 weighted
+    sample pairs, d_S = 3 x 1,024 (Eq. 2 input), d_R = 1,024, bf16 inputs,
+    reg 1e-3 (the bench's workload): every Newton-Schulz iteration count the
+    bench runs, against the oracle's fp64 eigendecompositions and SVD."""
+    N, d_s, d_r = 32768, 3072, 1024
+    g = torch.Generator(device="cuda").manual_seed(12)
+    X = (torch.randn((N, d_s), generator=g, device="cuda")
+         @ (torch.randn((d_s, d_s), generator=g, device="cuda") / d_s ** 0.5)).to(torch.bfloat16)
+    A_true = torch.randn((d_s, d_r), generator=g, device="cuda") / d_s ** 0.5
+    Y = (X.float() @ A_true + 0.5 * torch.randn((N, d_r), generator=g, device="cuda")
+         ).to(torch.bfloat16)
+    w = torch.rand((N,), generator=g, device="cuda") + 0.5
+    ws = torch.empty(B.recolor_workspace_size(N, d_s, d_r), dtype=torch.uint8, device="cuda")
+    W_out = torch.empty((d_r, d_s), dtype=torch.bfloat16, device="cuda")
+    b_out = torch.empty((d_r,), dtype=torch.float32, device="cuda")
+    r, its = B.recolor_fit("bf16", X, Y, w, W_out, b_out, ws, reg=1e-3, return_iters=True)
+    A = W_out.double().cpu().numpy().T
+    b = b_out.double().cpu().numpy()
+    Xn, Yn, wn = X.double().cpu().numpy(), Y.double().cpu().numpy(), w.double().cpu().numpy()
+    A_ref, b_ref, r_ref = O.recolor(Xn, Yn, wn, reg=1e-3)
+    assert abs(r - r_ref) <= 1e-5 * r_ref
+    assert all(0 < k < 80 for k in its), its
+    rel = np.linalg.norm(A - A_ref) / np.linalg.norm(A_ref)
+    assert rel <= 6e-3, rel   # bf16 rounding of A_final dominates (2^-9 relative)
+    relb = np.linalg.norm(b - b_ref) / max(np.linalg.norm(b_ref), 1.0)
+    assert relb <= 6e-3, relb
+    print(f"recolor 32768 x 3072 -> 1024: iterations {its}, rel A {rel:.2e}, rel b {relb:.2e}")
