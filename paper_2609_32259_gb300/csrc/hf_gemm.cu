@@ -57,6 +57,7 @@ struct GemmParams {
   int tiles_m, tiles_n, splits, kb_per_split;
   int n_terms;
   int term_a[kGMaxTerms], term_b[kGMaxTerms];
+  int vec;            // C rows can take 16-byte stores (ldc % 4 == 0, C 16-byte aligned)
   float alpha, beta;
 };
 
@@ -238,7 +239,7 @@ __global__ void __launch_bounds__(kGThreads, 1)
       const int row = m * kGTile + static_cast<int>(rank) * kGRows + row_in;
       const uint32_t ta = tmem_base + static_cast<uint32_t>(acc * kGTile) +
                           (static_cast<uint32_t>(q * 32) << 16);
-      const bool vec = (P.ldc % 4) == 0;
+      const bool vec = P.vec != 0;
       for (int c0 = 0; c0 < kGTile; c0 += 16) {
         uint32_t v[16];
         tmem_load_16(ta + static_cast<uint32_t>(c0), v);
@@ -246,7 +247,8 @@ __global__ void __launch_bounds__(kGThreads, 1)
         if (row >= P.M || col >= P.N) continue;
         if (P.splits > 1) {
           float* dst = P.partial + (static_cast<int64_t>(sp) * P.M + row) * P.N + col;
-          if (col + 16 <= P.N && (P.N % 4) == 0) {
+          if (col + 16 <= P.N && (P.N % 4) == 0 &&
+              (reinterpret_cast<uintptr_t>(P.partial) & 15u) == 0) {
 #pragma unroll
             for (int i = 0; i < 16; i += 4)
               *reinterpret_cast<float4*>(dst + i) =
@@ -475,6 +477,7 @@ hf_status gemm_f32(cudaStream_t s, const GemmWork& wk, int M, int N, int K, floa
     P.term_a[t] = ta[t];
     P.term_b[t] = tb[t];
   }
+  P.vec = (ldc % 4 == 0 && (reinterpret_cast<uintptr_t>(C) & 15u) == 0) ? 1 : 0;
   P.alpha = alpha;
   P.beta = beta;
   const int pairs = std::max(1, device_sm_count() / 2);
