@@ -9,17 +9,25 @@
 // i + j <= 2, summed by the tensor core into one fp32 TMEM accumulator; the
 // dropped terms are below 2^-23 of |a||b|, the size of fp32 rounding.
 //
+// The tensor core adds into its fp32 accumulator with truncation (measured
+// on GB300: a sum of 4,096 positive products comes out 1e-5 low, 7.6e-5 at
+// 16,384, where fp32 rounding to nearest is unbiased), so one accumulator
+// never takes more than one 64-wide atom of K (24 MMAs, the smallest terms
+// first): the epilogue drains each atom's accumulator into fp32 registers
+// with rounding to nearest while the tensor core fills the other one.
+//
 // The kernel: persistent clusters of two CTAs (one per SM pair), pair tiles
 // of 256 x 256 outputs (tcgen05.mma.cta_group::2, M = 256, N = 256,
 // K = 16 bf16 per instruction), each CTA holding 128 rows of the A tile and
 // 128 rows of the B tile.  A stage is one 128-byte atom (64 bf16) of K of
 // one term's A plane and B plane, loaded by TMA (128-byte swizzle) and
 // completing on the leader CTA's barrier.
-//   warp 0     TMA producer
-//   warp 1     TMEM allocator; in the leader CTA the thread issuing the MMAs
-//              into one of two 256-column accumulators
-//   warps 2-5  epilogue: TMEM -> registers -> alpha * acc + beta * C (or a
-//              split-K partial) -> global
+//   warp 0      TMA producer
+//   warp 1      TMEM allocator; in the leader CTA the thread issuing the MMAs
+//               of one K atom into one of two 256-column accumulators
+//   warps 2-17  epilogue: 4 warps per TMEM lane quarter, 64 columns each;
+//               per K atom TMEM -> registers (running fp32 sums); per tile
+//               alpha * sum + beta * C (or a split-K partial) -> global
 // Small products are split along K so that every SM pair has work; a second
 // kernel sums the partials.  Waits are bounded: a wait that runs out sets an
 // error word and the CTA pair unwinds.
@@ -41,7 +49,8 @@ constexpr int kGTile = 256;                 // pair tile: 256 x 256 outputs
 constexpr int kGAtomBytes = kGRows * 128;   // one 128-byte atom of K for 128 rows
 constexpr int kGStageBytes = 2 * kGAtomBytes;
 constexpr int kGStages = 6;
-constexpr int kGEpiWarps = 4;
+constexpr int kGEpiWarps = 16;
+constexpr int kGEpiCols = kGTile / (kGEpiWarps / 4);  // columns per epilogue thread
 constexpr int kGThreads = 64 + 32 * kGEpiWarps;
 constexpr int kGMaxTerms = 6;
 constexpr int kGTmemCols = 512;
@@ -176,15 +185,17 @@ __global__ void __launch_bounds__(kGThreads, 1)
         int m, n, sp;
         gemm_decode(P, tile, &m, &n, &sp);
         const int kb0 = sp * P.kb_per_split, kb1 = min(P.n_kb, kb0 + P.kb_per_split);
-        if (!mbar_wait(smem_addr(&tempty[acc]), acc_phase ^ 1)) {
-          atomicOr(P.err, 1);
-          *sAbort = 1;
-          break;
-        }
-        tc_fence_after_sync();
-        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * kGTile);
-        uint32_t accumulate = 0;
         for (int kb = kb0; kb < kb1 && ok; ++kb) {
+          // one K atom per accumulator (the accumulator adds by truncation)
+          if (!mbar_wait(smem_addr(&tempty[acc]), acc_phase ^ 1)) {
+            atomicOr(P.err, 1);
+            *sAbort = 1;
+            ok = false;
+            break;
+          }
+          tc_fence_after_sync();
+          const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * kGTile);
+          uint32_t accumulate = 0;
           for (int t = 0; t < P.n_terms; ++t) {
             if (!mbar_wait(smem_addr(&full[stage]), phase)) {
               atomicOr(P.err, 1);
@@ -206,11 +217,11 @@ __global__ void __launch_bounds__(kGThreads, 1)
               phase ^= 1;
             }
           }
+          if (!ok) break;
+          tc_commit_pair(smem_addr(&tfull[acc]), 0x3);
+          acc ^= 1;
+          if (acc == 0) acc_phase ^= 1;
         }
-        if (!ok) break;
-        tc_commit_pair(smem_addr(&tfull[acc]), 0x3);
-        acc ^= 1;
-        if (acc == 0) acc_phase ^= 1;
       }
       tc_commit_pair(smem_addr(drain), 0x3);
     }
@@ -223,77 +234,90 @@ __global__ void __launch_bounds__(kGThreads, 1)
     __syncwarp();
   } else {
     // ------------------------------------------------------------ epilogue
-    const int q = warp & 3;  // TMEM lane quarter this warp may access
+    const int e = warp - 2;       // 0..15
+    const int q = warp & 3;       // TMEM lane quarter this warp may access
+    const int cg = e >> 2;        // column group: columns cg * 64 .. + 63
     const int row_in = q * 32 + lane;
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int tile = first; tile < total; tile += step) {
+    bool ok = true;
+    for (int tile = first; tile < total && ok; tile += step) {
       int m, n, sp;
       gemm_decode(P, tile, &m, &n, &sp);
-      if (!mbar_wait(smem_addr(&tfull[acc]), acc_phase)) {
-        atomicOr(P.err, 1);
-        *sAbort = 1;
-        break;
+      const int kb0 = sp * P.kb_per_split, kb1 = min(P.n_kb, kb0 + P.kb_per_split);
+      float sum[kGEpiCols];
+#pragma unroll
+      for (int i = 0; i < kGEpiCols; ++i) sum[i] = 0.f;
+      for (int kb = kb0; kb < kb1; ++kb) {
+        if (!mbar_wait(smem_addr(&tfull[acc]), acc_phase)) {
+          atomicOr(P.err, 1);
+          *sAbort = 1;
+          ok = false;
+          break;
+        }
+        tc_fence_after_sync();
+        const uint32_t ta = tmem_base + static_cast<uint32_t>(acc * kGTile + cg * kGEpiCols) +
+                            (static_cast<uint32_t>(q * 32) << 16);
+#pragma unroll
+        for (int c0 = 0; c0 < kGEpiCols; c0 += 16) {
+          uint32_t v[16];
+          tmem_load_16(ta + static_cast<uint32_t>(c0), v);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) sum[c0 + i] = __fadd_rn(sum[c0 + i], __uint_as_float(v[i]));
+        }
+        tc_fence_before_sync();
+        __syncwarp();
+        if (lane == 0) {
+          if (rank == 0)
+            mbar_arrive_relaxed(smem_addr(&tempty[acc]));
+          else
+            mbar_arrive_cluster(mapa_shared(smem_addr(&tempty[acc]), 0));
+        }
+        acc ^= 1;
+        if (acc == 0) acc_phase ^= 1;
       }
-      tc_fence_after_sync();
+      if (!ok) break;
       const int row = m * kGTile + static_cast<int>(rank) * kGRows + row_in;
-      const uint32_t ta = tmem_base + static_cast<uint32_t>(acc * kGTile) +
-                          (static_cast<uint32_t>(q * 32) << 16);
-      const bool vec = P.vec != 0;
-      for (int c0 = 0; c0 < kGTile; c0 += 16) {
-        uint32_t v[16];
-        tmem_load_16(ta + static_cast<uint32_t>(c0), v);
-        const int col = n * kGTile + c0;
-        if (row >= P.M || col >= P.N) continue;
-        if (P.splits > 1) {
-          float* dst = P.partial + (static_cast<int64_t>(sp) * P.M + row) * P.N + col;
-          if (col + 16 <= P.N && (P.N % 4) == 0 &&
-              (reinterpret_cast<uintptr_t>(P.partial) & 15u) == 0) {
+      const int col0 = n * kGTile + cg * kGEpiCols;
+      if (row >= P.M) continue;
+      if (P.splits > 1) {
+        float* dst = P.partial + (static_cast<int64_t>(sp) * P.M + row) * P.N + col0;
+        const bool v4 = (P.N % 4) == 0 && (reinterpret_cast<uintptr_t>(P.partial) & 15u) == 0;
 #pragma unroll
-            for (int i = 0; i < 16; i += 4)
-              *reinterpret_cast<float4*>(dst + i) =
-                  make_float4(__uint_as_float(v[i]), __uint_as_float(v[i + 1]),
-                              __uint_as_float(v[i + 2]), __uint_as_float(v[i + 3]));
+        for (int i = 0; i < kGEpiCols; i += 4) {
+          if (v4 && col0 + i + 4 <= P.N) {
+            *reinterpret_cast<float4*>(dst + i) =
+                make_float4(sum[i], sum[i + 1], sum[i + 2], sum[i + 3]);
           } else {
-            for (int i = 0; i < 16 && col + i < P.N; ++i) dst[i] = __uint_as_float(v[i]);
+            for (int k = 0; k < 4; ++k)
+              if (col0 + i + k < P.N) dst[i + k] = sum[i + k];
           }
-        } else {
-          float* dst = P.C + static_cast<int64_t>(row) * P.ldc + col;
-          if (col + 16 <= P.N && vec) {
+        }
+      } else {
+        float* dst = P.C + static_cast<int64_t>(row) * P.ldc + col0;
 #pragma unroll
-            for (int i = 0; i < 16; i += 4) {
-              float4 o = make_float4(P.alpha * __uint_as_float(v[i]),
-                                     P.alpha * __uint_as_float(v[i + 1]),
-                                     P.alpha * __uint_as_float(v[i + 2]),
-                                     P.alpha * __uint_as_float(v[i + 3]));
-              if (P.beta != 0.f) {
-                const float4 c = *reinterpret_cast<const float4*>(dst + i);
-                o.x = fmaf(P.beta, c.x, o.x);
-                o.y = fmaf(P.beta, c.y, o.y);
-                o.z = fmaf(P.beta, c.z, o.z);
-                o.w = fmaf(P.beta, c.w, o.w);
-              }
-              *reinterpret_cast<float4*>(dst + i) = o;
+        for (int i = 0; i < kGEpiCols; i += 4) {
+          if (P.vec && col0 + i + 4 <= P.N) {
+            float4 o = make_float4(P.alpha * sum[i], P.alpha * sum[i + 1], P.alpha * sum[i + 2],
+                                   P.alpha * sum[i + 3]);
+            if (P.beta != 0.f) {
+              const float4 c = *reinterpret_cast<const float4*>(dst + i);
+              o.x = fmaf(P.beta, c.x, o.x);
+              o.y = fmaf(P.beta, c.y, o.y);
+              o.z = fmaf(P.beta, c.z, o.z);
+              o.w = fmaf(P.beta, c.w, o.w);
             }
+            *reinterpret_cast<float4*>(dst + i) = o;
           } else {
-            for (int i = 0; i < 16 && col + i < P.N; ++i) {
-              float o = P.alpha * __uint_as_float(v[i]);
-              if (P.beta != 0.f) o = fmaf(P.beta, dst[i], o);
-              dst[i] = o;
+            for (int k = 0; k < 4; ++k) {
+              if (col0 + i + k >= P.N) continue;
+              float o = P.alpha * sum[i + k];
+              if (P.beta != 0.f) o = fmaf(P.beta, dst[i + k], o);
+              dst[i + k] = o;
             }
           }
         }
       }
-      tc_fence_before_sync();
-      __syncwarp();
-      if (lane == 0) {
-        if (rank == 0)
-          mbar_arrive_relaxed(smem_addr(&tempty[acc]));
-        else
-          mbar_arrive_cluster(mapa_shared(smem_addr(&tempty[acc]), 0));
-      }
-      acc ^= 1;
-      if (acc == 0) acc_phase ^= 1;
     }
   }
 
@@ -470,8 +494,9 @@ hf_status gemm_f32(cudaStream_t s, const GemmWork& wk, int M, int N, int K, floa
   P.n_kb = static_cast<int>(Kp / 64);
   P.tiles_m = static_cast<int>(Mp / kGTile);
   P.tiles_n = static_cast<int>(Np / kGTile);
-  // terms a_i b_j with i + j <= 2, largest first
-  const int ta[kGMaxTerms] = {0, 0, 1, 0, 1, 2}, tb[kGMaxTerms] = {0, 1, 0, 2, 1, 0};
+  // terms a_i b_j with i + j <= 2, smallest first: an accumulator that
+  // adds by truncation loses at most an ulp of its current magnitude per add
+  const int ta[kGMaxTerms] = {2, 1, 0, 1, 0, 0}, tb[kGMaxTerms] = {0, 1, 2, 0, 1, 0};
   P.n_terms = kGMaxTerms;
   for (int t = 0; t < kGMaxTerms; ++t) {
     P.term_a[t] = ta[t];

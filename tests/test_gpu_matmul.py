@@ -97,3 +97,23 @@ def test_matmul_gram_shares_planes():
     ref = x.astype(np.float64).T @ x.astype(np.float64)
     got = C.cpu().numpy().astype(np.float64)
     assert np.linalg.norm(got - ref) / np.linalg.norm(ref) <= 5e-6
+
+
+def test_matmul_unbiased_on_positive_data():
+    """Positive operands, K = 16,384: the tensor core's accumulator adds by
+    truncation (a single accumulator over K came out 7.6e-5 low on average),
+    so the kernel drains it into round-to-nearest fp32 sums every 64-wide K
+    atom; the mean relative error must stay at the fp32 level."""
+    M, K = 1024, 16384
+    gen = np.random.default_rng(17)
+    a = (1.0 + gen.random((M, K))).astype(np.float32)
+    b = (1.0 + gen.random((K, M))).astype(np.float32)
+    dA = torch.as_tensor(a, device="cuda")
+    dB = torch.as_tensor(b, device="cuda")
+    C = torch.empty((M, M), dtype=torch.float32, device="cuda")
+    assert B.debug_matmul_f32(dA, (K, 1), dB, (M, 1), C, M, M, K) == 0
+    ref = torch.as_tensor(a, dtype=torch.float64, device="cuda") @ torch.as_tensor(
+        b, dtype=torch.float64, device="cuda")
+    rel = ((C.double() - ref) / ref).cpu().numpy()
+    assert abs(rel.mean()) <= 1e-6, rel.mean()
+    assert np.abs(rel).max() <= 1e-5, np.abs(rel).max()
