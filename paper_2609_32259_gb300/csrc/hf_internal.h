@@ -89,6 +89,7 @@ struct hf_plan_s {
   int BN, groups, stages;
   bool gather;  // every map input row is a single unweighted sender row
   bool split;   // computed bf16 operand rows go to the tensor core as value + residual
+  bool staged;  // split rows of one entry each: raw sender atoms staged by cp.async
   bool rope;    // receiver keys get RoPE
   bool unrot;   // sender keys carry RoPE and are rotated back in the builder
   bool span;    // aligned sender tokens are spans inside a longer sender cache

@@ -124,7 +124,10 @@ PlanDev plan_dev(const hf_plan_s* p) {
 }
 
 // Copies the constant tables into the workspace and clears the counters.
-__global__ void plan_init_kernel(PlanConsts t, PlanDev d) {
+// The tables stay in the kernel parameter space (__grid_constant__): indexing
+// a by-value parameter with a thread-dependent index would make every
+// thread copy the whole table to local memory first.
+__global__ void plan_init_kernel(const __grid_constant__ PlanConsts t, PlanDev d) {
   const int tid = threadIdx.x;
   if (tid == 0) {
     *d.status = 0;
@@ -140,9 +143,13 @@ __global__ void plan_init_kernel(PlanConsts t, PlanDev d) {
   for (int i = tid; i < t.n_req; i += blockDim.x) d.s_row0[i] = t.s_row0[i];
 }
 
-// Copies the layer table into the workspace.
-__global__ void plan_segs_kernel(SegTables t, LayerSegs* segs) {
-  for (int i = threadIdx.x; i < t.L_r; i += blockDim.x) segs[i] = t.segs[i];
+// Copies the layer table into the workspace, one 32-bit word per thread step.
+__global__ void plan_segs_kernel(const __grid_constant__ SegTables t, LayerSegs* segs) {
+  static_assert(sizeof(LayerSegs) % 4 == 0, "LayerSegs is copied as 32-bit words");
+  const uint32_t* src = reinterpret_cast<const uint32_t*>(t.segs);
+  uint32_t* dst = reinterpret_cast<uint32_t*>(segs);
+  const int n = t.L_r * static_cast<int>(sizeof(LayerSegs) / 4);
+  for (int i = threadIdx.x; i < n; i += blockDim.x) dst[i] = src[i];
 }
 
 // Per aligned sender token: its RoPE position (sender_k_rotated), the
@@ -484,6 +491,10 @@ hf_status plan_build(const hf_plan_desc* desc, void* d_workspace, size_t workspa
   p->rope = desc->theta_r > 0.0 || desc->h_inv_freq_r != nullptr;
   p->gather = one_layer_segments && desc->align_mode != HF_ALIGN_OVERLAP_MEAN && !p->unrot;
   p->split = !p->gather && desc->dtype == HF_BF16 && desc->round_built_operands == 0;
+  // one-entry rows (Token Alignment, same-index) have at most two (term,
+  // entry) pairs per segment, both staged by cp.async; pooled rows have more,
+  // whose direct loads stall the warp anyway (measured slower staged)
+  p->staged = p->split && !p->unrot && desc->align_mode != HF_ALIGN_OVERLAP_MEAN;
   p->ws = static_cast<char*>(d_workspace);
   p->ws_bytes = workspace_bytes;
   p->lay = lay;

@@ -86,6 +86,7 @@ struct XferParams {
   // rounded operand and its rounding residual, multiplied by the same B atom
   // (atoms_per_stage = 1); otherwise kAtoms atoms of K per A stage
   int split, atoms_per_stage, n_batoms;  // n_batoms: B atoms (map atoms of K) per tile
+  int staged;  // split one-entry rows built by build_rows_staged
   int stages_a, stages_b, lag;  // A ring (stages), B ring (atoms), loader groups in flight
   int rope, paged, knorm, unrot, D_s;
   int stall;  // test hook: the map producer withholds its first atom (hf_debug_transfer_stalled)
@@ -671,6 +672,193 @@ __device__ __forceinline__ void gather_rows(const XferParams* Ps, const DirTable
       arrive_leader(smem_addr(&full_a[(stage + stages - k) % stages]), row0);
 }
 
+// Computed A rows in split mode without rotated keys (pooled rows, blended
+// or weighted layers), staged: a stage is one map atom of K.  The loader
+// copies the first two raw (term, entry) sender atoms of every row into the
+// stage's two atom slots with cp.async, eight lanes per 128-byte row as in
+// gather_rows, and keeps LAG stages in flight; once a stage's copies have
+// landed, thread t of the warp finishes row 32 slab + t (finish_staged_row):
+// it combines the two staged atoms and any further (term, entry) pairs
+// (loaded directly) in fp32 with their weights, and overwrites the slots
+// with the bf16 value and its rounding residual.  The first two pairs of a
+// row are (term 0, entry 0) and (term 1, entry 0) for two-term segments,
+// (term 0, entries 0 and 1) otherwise, so blended one-entry rows need no
+// direct load.
+struct StagedRow {
+  int e0, e1;  // the finished row's CSR entries
+  int frow;    // its index among the CTA's 128 rows
+};
+
+template <typename T>
+__device__ __forceinline__ void finish_staged_row(const XferParams& P, const LayerSegs* lsegs,
+                                                  int c, const StagedRow& r, int kb,
+                                                  uint8_t* slot0) {
+  constexpr int kBK = Elem<T>::kBK;
+  constexpr int kPerChunk = 16 / sizeof(T);
+  const T* sender = reinterpret_cast<const T*>(P.sender);
+  uint8_t* slot1 = slot0 + kAtomABytes;
+  const int seg = kb / P.atoms_per_seg, kin = kb - seg * P.atoms_per_seg;
+  const int n_t = __ldg(&lsegs->n_terms[seg]);
+  const int la0 = __ldg(&lsegs->layer[seg][0]);
+  const int la1 = n_t > 1 ? __ldg(&lsegs->layer[seg][1]) : la0;
+  const float om0 = __ldg(&lsegs->w[seg][0]);
+  const float om1 = n_t > 1 ? __ldg(&lsegs->w[seg][1]) : 0.f;
+  const int64_t lrows = P.s_rows * P.d_s;
+  const int frow = r.frow, sw = frow & 7;
+  const int k0 = r.e1 > r.e0 ? P.col[r.e0] : -1;
+  const bool v0 = k0 >= 0 && k0 < P.T_s;
+  int k1 = -1;
+  if (n_t == 1 && r.e1 > r.e0 + 1) k1 = P.col[r.e0 + 1];
+  const bool v1 = n_t > 1 ? v0 : (k1 >= 0 && k1 < P.T_s);
+  const float w0 = v0 ? om0 * P.w[r.e0] : 0.f;
+  const float w1 = !v1 ? 0.f : (n_t > 1 ? om1 * P.w[r.e0] : om0 * P.w[r.e0 + 1]);
+  // two halves of four 16-byte chunks (fewer live registers)
+#pragma unroll 1
+  for (int h = 0; h < 2; ++h) {
+    float acc[kBK / 2];
+#pragma unroll
+    for (int i = 0; i < kBK / 2; ++i) acc[i] = 0.f;
+#pragma unroll
+    for (int k2 = 0; k2 < 4; ++k2) {
+      const int off = frow * 128 + (((4 * h + k2) ^ sw) << 4);
+      if (v0)
+        accum16(*reinterpret_cast<const uint4*>(slot0 + off), w0, acc + k2 * kPerChunk,
+                (const T*)nullptr);
+      if (v1)
+        accum16(*reinterpret_cast<const uint4*>(slot1 + off), w1, acc + k2 * kPerChunk,
+                (const T*)nullptr);
+    }
+    // the remaining (term, entry) pairs, loaded directly
+    const int e_first = n_t > 1 ? r.e0 + 1 : r.e0 + 2;
+    for (int e = e_first; e < r.e1; ++e) {
+      const int k = P.col[e];
+      if (k < 0 || k >= P.T_s) continue;  // flagged at plan creation
+      const int64_t kr = P.srow ? __ldg(P.srow + k) : k;
+      for (int ti = 0; ti < n_t; ++ti) {
+        const int la = ti == 0 ? la0 : la1;
+        const float wt = (ti == 0 ? om0 : om1) * P.w[e];
+        const uint4* src = reinterpret_cast<const uint4*>(
+                               sender + static_cast<int64_t>(la * 2 + c) * lrows + kr * P.d_s +
+                               kin * kBK) + 4 * h;
+        uint4 x[4];
+#pragma unroll
+        for (int k2 = 0; k2 < 4; ++k2) x[k2] = __ldg(src + k2);
+#pragma unroll
+        for (int k2 = 0; k2 < 4; ++k2) accum16(x[k2], wt, acc + k2 * kPerChunk, (const T*)nullptr);
+      }
+    }
+#pragma unroll
+    for (int k2 = 0; k2 < 4; ++k2)
+      put_chunk<T>(acc + k2 * kPerChunk, slot0, slot1, frow, 4 * h + k2);
+  }
+}
+
+template <typename T, int LAG, int kDirs>
+__device__ __forceinline__ void build_rows_staged(const XferParams* Ps, const DirTable<kDirs>& dt,
+                                                  int n_dir, uint8_t* sA, uint64_t* full_a,
+                                                  uint64_t* empty_a, volatile int* sAbort, int t,
+                                                  int lane, int row0, int total_tiles,
+                                                  int first_tile, int tile_step) {
+  constexpr int kBK = Elem<T>::kBK;
+  constexpr int kPerChunk = 16 / sizeof(T);
+  const bool by_slot = total_tiles >= 4 * tile_step;  // as in transfer_body
+  const int stages = Ps[0].stages_a;
+  const int slab = t >> 5, rsub = lane >> 3, ch = lane & 7;
+  int stage = 0;
+  uint32_t phase = 0;
+  bool ok = true;
+  for (int seq = 0, tile = tile_of(0, first_tile, tile_step, by_slot); tile < total_tiles && ok;
+       tile = tile_of(++seq, first_tile, tile_step, by_slot)) {
+    const int dd = dir_of(dt, n_dir, tile);
+    const XferParams& P = Ps[dd];
+    const int U = dt.U[dd];
+    const T* sender = reinterpret_cast<const T*>(P.sender);
+    int lc, m, n;
+    decode_tile(tile - dt.base[dd], dt.m_tiles[dd] * P.n_tiles_n, P.n_tiles_n, P.l0, &lc, &m, &n);
+    const int l = lc >> 1, c = lc & 1;
+    const LayerSegs* lsegs = P.segs + l;
+    const int64_t lrows = P.s_rows * P.d_s;
+    // cache rows of the first two entries of the eight rows this lane copies
+    int32_t kr0[8], kr1[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int u = min(m * kPairRows + row0 + slab * 32 + 4 * i + rsub, U - 1);
+      const int j0 = P.run_ptr[u];
+      const int e0 = P.row_ptr[j0], e1 = P.row_ptr[j0 + 1];
+      int k0 = e1 > e0 ? P.col[e0] : -1;
+      int k1 = e1 > e0 + 1 ? P.col[e0 + 1] : -1;
+      if (k0 >= P.T_s) k0 = -1;  // flagged at plan creation
+      if (k1 >= P.T_s) k1 = -1;
+      kr0[i] = k0 < 0 ? -1 : (P.srow ? __ldg(P.srow + k0) : k0);
+      kr1[i] = k1 < 0 ? -1 : (P.srow ? __ldg(P.srow + k1) : k1);
+    }
+    StagedRow fr;
+    fr.frow = slab * 32 + lane;
+    {
+      const int fu = min(m * kPairRows + row0 + fr.frow, U - 1);
+      const int fj0 = P.run_ptr[fu];
+      fr.e0 = P.row_ptr[fj0];
+      fr.e1 = P.row_ptr[fj0 + 1];
+    }
+    int pending = 0;  // stages issued and not yet finished (<= LAG)
+    for (int kb = 0; kb < P.n_kb; ++kb) {
+      if (!mbar_wait(smem_addr(&empty_a[stage]), phase ^ 1)) {
+        raise_timeout(P, sAbort);
+        ok = false;
+        break;
+      }
+      const int seg = kb / P.atoms_per_seg, kin = kb - seg * P.atoms_per_seg;
+      const int n_t = __ldg(&lsegs->n_terms[seg]);
+      const int la0 = __ldg(&lsegs->layer[seg][0]);
+      const int la1 = n_t > 1 ? __ldg(&lsegs->layer[seg][1]) : la0;
+      const T* b0 = sender + static_cast<int64_t>(la0 * 2 + c) * lrows + kin * kBK + ch * kPerChunk;
+      const T* b1 = sender + static_cast<int64_t>(la1 * 2 + c) * lrows + kin * kBK + ch * kPerChunk;
+      const uint32_t sa = smem_addr(sA + stage * kStageABytes);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int r = slab * 32 + 4 * i + rsub;
+        const uint32_t doff = static_cast<uint32_t>(r * 128 + ((ch ^ (r & 7)) << 4));
+        if (kr0[i] >= 0) {
+          cp_async_16(sa + doff, b0 + static_cast<int64_t>(kr0[i]) * P.d_s);
+          if (n_t > 1)
+            cp_async_16(sa + kAtomABytes + doff, b1 + static_cast<int64_t>(kr0[i]) * P.d_s);
+        }
+        if (n_t == 1 && kr1[i] >= 0)
+          cp_async_16(sa + kAtomABytes + doff, b0 + static_cast<int64_t>(kr1[i]) * P.d_s);
+      }
+      cp_async_commit();
+      if (pending == LAG) {
+        // stage kb - LAG (issued LAG stages ago) has landed for this thread;
+        // after the warp barrier, for the whole warp
+        cp_async_wait<LAG>();
+        __syncwarp();
+        const int st = (stage + stages - LAG) % stages;
+        finish_staged_row<T>(P, lsegs, c, fr, kb - LAG, sA + st * kStageABytes);
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) arrive_leader(smem_addr(&full_a[st]), row0);
+      } else {
+        ++pending;
+      }
+      if (++stage == stages) {
+        stage = 0;
+        phase ^= 1;
+      }
+    }
+    if (!ok) break;
+    // the tile's last `pending` stages: stage - pending .. stage - 1
+    cp_async_wait<0>();
+    __syncwarp();
+    for (int q = pending; q >= 1; --q) {
+      const int st = (stage + stages - q) % stages;
+      finish_staged_row<T>(P, lsegs, c, fr, P.n_kb - q, sA + st * kStageABytes);
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) arrive_leader(smem_addr(&full_a[st]), row0);
+    }
+  }
+}
+
 // The kernel body for one direction (kDirs = 1, the map and parameters are
 // kernel parameters) or several (tiles of all directions in one launch;
 // every role looks its tile's direction up and reads that direction's
@@ -1034,6 +1222,12 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
         case 4: gather_rows<T, 4, kDirs>(Ps, dt, n_dir, sA, full_a, empty_a, sAbort, t, lane, row0, total_tiles, first_tile, tile_step); break;
         default: gather_rows<T, 5, kDirs>(Ps, dt, n_dir, sA, full_a, empty_a, sAbort, t, lane, row0, total_tiles, first_tile, tile_step); break;
       }
+    } else if (P0.staged) {
+      switch (P0.lag) {
+        case 1: build_rows_staged<T, 1, kDirs>(Ps, dt, n_dir, sA, full_a, empty_a, sAbort, t, lane, row0, total_tiles, first_tile, tile_step); break;
+        case 2: build_rows_staged<T, 2, kDirs>(Ps, dt, n_dir, sA, full_a, empty_a, sAbort, t, lane, row0, total_tiles, first_tile, tile_step); break;
+        default: build_rows_staged<T, 3, kDirs>(Ps, dt, n_dir, sA, full_a, empty_a, sAbort, t, lane, row0, total_tiles, first_tile, tile_step); break;
+      }
     } else {
       // pooled CSR rows, blended sender layers and/or rotated sender keys:
       // thread t owns tile row t
@@ -1287,6 +1481,7 @@ hf_status make_xfer(hf_plan_s* p, const void* sender, void* receiver, int l_begi
   P.D_r = d.D_r;
   const int n_atoms = p->K / bk;  // 128-byte k-blocks per output row
   P.split = p->split ? 1 : 0;
+  P.staged = p->staged ? 1 : 0;
   P.atoms_per_stage = p->split ? 1 : kAtoms;
   P.n_batoms = n_atoms;
   P.n_kb = (n_atoms + P.atoms_per_stage - 1) / P.atoms_per_stage;
@@ -1340,7 +1535,7 @@ hf_status launch_transfer(hf_plan_s* p, const void* sender, void* receiver, cuda
 bool batch_compatible(const hf_plan_s* const* plans, int n) {
   for (int i = 1; i < n; ++i)
     if (plans[i]->desc.dtype != plans[0]->desc.dtype || plans[i]->gather != plans[0]->gather ||
-        plans[i]->split != plans[0]->split)
+        plans[i]->split != plans[0]->split || plans[i]->staged != plans[0]->staged)
       return false;
   return true;
 }
