@@ -230,7 +230,7 @@ class Desc:
             n_seg=n_seg, n_terms=n_terms,
             h_seg_layer=_as_i32p(self._segl) if self._segl is not None else None,
             h_seg_w=_f32_or_null(self._segw),
-            round_built_operands=int(bool(round_built_operands)))
+            round_built_operands=int(round_built_operands))
 
 
 def plan_workspace_size(desc: Desc) -> int:

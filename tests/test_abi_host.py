@@ -76,6 +76,7 @@ def _desc(B, **over):
     (dict(s_row0=[3], sender_rows=7), 1),             # span of 5 rows from row 3 > 7 rows
     (dict(s_row0=[-1], sender_rows=70), 1),
     (dict(sender_rows=4), 1),                         # fewer cache rows than sender tokens
+    (dict(round_built_operands=2), 1),                # a flag: 0 or 1
 ])
 def test_plan_create_rejects(B, over, status):
     d = _desc(B, **over)
