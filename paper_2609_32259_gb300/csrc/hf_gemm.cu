@@ -1,7 +1,8 @@
 // fp32 matrix products on the tcgen05 tensor cores, for hf_recolor_fit's
 // moments, Newton-Schulz roots and polar iterations (Section 3.2, Eq. 3-5).
 //
-// C = alpha op(A) op(B) + beta C with fp32 accuracy from bf16 products.
+// C = alpha op(A) op(B) + beta C_in + d I with fp32 accuracy from bf16
+// products (C_in may be C itself; d I adds d on the diagonal).
 // Every fp32 operand value x is split exactly into three bf16 parts,
 // x0 = bf16(x), x1 = bf16(x - x0), x2 = x - x0 - x1 (what is left has at
 // most 8 significant bits, so it is exact in bf16), and each part is stored
@@ -57,6 +58,8 @@ constexpr int kGTmemCols = 512;
 
 struct GemmParams {
   float* C;           // output, row-major with leading dimension ldc
+  const float* Cin;   // beta term's matrix (same layout as C; may be C)
+  float diag;         // added on the diagonal (row == column)
   int64_t ldc;
   float* partial;     // split-K partials [splits][M][N] (splits > 1)
   int32_t* err;       // error word (a wait ran out)
@@ -295,24 +298,30 @@ __global__ void __launch_bounds__(kGThreads, 1)
         }
       } else {
         float* dst = P.C + static_cast<int64_t>(row) * P.ldc + col0;
+        const float* cin = P.Cin + static_cast<int64_t>(row) * P.ldc + col0;
+        const int dcol = row - col0;  // this row's diagonal element, if in range
 #pragma unroll
         for (int i = 0; i < kGEpiCols; i += 4) {
           if (P.vec && col0 + i + 4 <= P.N) {
-            float4 o = make_float4(P.alpha * sum[i], P.alpha * sum[i + 1], P.alpha * sum[i + 2],
-                                   P.alpha * sum[i + 3]);
+            float o[4] = {P.alpha * sum[i], P.alpha * sum[i + 1], P.alpha * sum[i + 2],
+                          P.alpha * sum[i + 3]};
             if (P.beta != 0.f) {
-              const float4 c = *reinterpret_cast<const float4*>(dst + i);
-              o.x = fmaf(P.beta, c.x, o.x);
-              o.y = fmaf(P.beta, c.y, o.y);
-              o.z = fmaf(P.beta, c.z, o.z);
-              o.w = fmaf(P.beta, c.w, o.w);
+              const float4 c = *reinterpret_cast<const float4*>(cin + i);
+              o[0] = fmaf(P.beta, c.x, o[0]);
+              o[1] = fmaf(P.beta, c.y, o[1]);
+              o[2] = fmaf(P.beta, c.z, o[2]);
+              o[3] = fmaf(P.beta, c.w, o[3]);
             }
-            *reinterpret_cast<float4*>(dst + i) = o;
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+              if (dcol == i + k) o[k] += P.diag;
+            *reinterpret_cast<float4*>(dst + i) = make_float4(o[0], o[1], o[2], o[3]);
           } else {
             for (int k = 0; k < 4; ++k) {
               if (col0 + i + k >= P.N) continue;
               float o = P.alpha * sum[i + k];
-              if (P.beta != 0.f) o = fmaf(P.beta, dst[i + k], o);
+              if (P.beta != 0.f) o = fmaf(P.beta, cin[i + k], o);
+              if (dcol == i + k) o += P.diag;
               dst[i + k] = o;
             }
           }
@@ -335,17 +344,20 @@ __global__ void __launch_bounds__(kGThreads, 1)
   }
 }
 
-// C = alpha * sum_s partial[s] + beta * C.
+// C = alpha * sum_s partial[s] + beta * C_in + diag I.
 __global__ void gemm_reduce_kernel(const float* partial, int splits, int M, int N, float* C,
-                                   int64_t ldc, float alpha, float beta) {
+                                   const float* Cin, int64_t ldc, float alpha, float beta,
+                                   float diag) {
   const int64_t n_el = static_cast<int64_t>(M) * N;
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n_el;
        i += (int64_t)gridDim.x * blockDim.x) {
     float s = 0.f;
     for (int k = 0; k < splits; ++k) s += partial[k * n_el + i];
     const int64_t r = i / N, c = i - r * N;
-    float* dst = C + r * ldc + c;
-    *dst = beta != 0.f ? fmaf(beta, *dst, alpha * s) : alpha * s;
+    float o = alpha * s;
+    if (beta != 0.f) o = fmaf(beta, Cin[r * ldc + c], o);
+    if (r == c) o += diag;
+    C[r * ldc + c] = o;
   }
 }
 
@@ -447,7 +459,9 @@ size_t gemm_planes_bytes(int64_t rows, int64_t K) {
 
 hf_status gemm_f32(cudaStream_t s, const GemmWork& wk, int M, int N, int K, float alpha,
                    const float* A, int64_t a_i, int64_t a_k, const float* B, int64_t b_k,
-                   int64_t b_j, float beta, float* C, int64_t ldc) {
+                   int64_t b_j, float beta, float* C, int64_t ldc, const float* Cin,
+                   float diag) {
+  if (Cin == nullptr) Cin = C;
   if (M <= 0 || N <= 0) return HF_OK;
   if (K <= 0) {
     set_error("hf_recolor_fit: internal error: a product with K = 0");
@@ -485,6 +499,8 @@ hf_status gemm_f32(cudaStream_t s, const GemmWork& wk, int M, int N, int K, floa
   GemmParams P;
   std::memset(&P, 0, sizeof(P));
   P.C = C;
+  P.Cin = Cin;
+  P.diag = diag;
   P.ldc = ldc;
   P.err = wk.err;
   P.M = M;
@@ -502,7 +518,10 @@ hf_status gemm_f32(cudaStream_t s, const GemmWork& wk, int M, int N, int K, floa
     P.term_a[t] = ta[t];
     P.term_b[t] = tb[t];
   }
-  P.vec = (ldc % 4 == 0 && (reinterpret_cast<uintptr_t>(C) & 15u) == 0) ? 1 : 0;
+  P.vec = (ldc % 4 == 0 && ((reinterpret_cast<uintptr_t>(C) | reinterpret_cast<uintptr_t>(Cin)) &
+                             15u) == 0)
+              ? 1
+              : 0;
   P.alpha = alpha;
   P.beta = beta;
   const int pairs = std::max(1, device_sm_count() / 2);
@@ -538,7 +557,8 @@ hf_status gemm_f32(cudaStream_t s, const GemmWork& wk, int M, int N, int K, floa
   if (splits > 1) {
     const int64_t n_el = static_cast<int64_t>(M) * N;
     const int grid = static_cast<int>(std::min<int64_t>((n_el + 255) / 256, 4096));
-    gemm_reduce_kernel<<<grid, 256, 0, s>>>(wk.partial, splits, M, N, C, ldc, alpha, beta);
+    gemm_reduce_kernel<<<grid, 256, 0, s>>>(wk.partial, splits, M, N, C, Cin, ldc, alpha, beta,
+                                            diag);
     HF_CUDA_TRY(cudaGetLastError(), "hf_recolor_fit: product reduce launch");
   }
   return HF_OK;
@@ -605,7 +625,8 @@ extern "C" hf_status hf_debug_matmul_f32(int32_t M, int32_t N, int32_t K, float 
   wk.err = reinterpret_cast<int32_t*>(ws + L.err);
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   HF_CUDA_TRY(cudaMemsetAsync(wk.err, 0, sizeof(int32_t), s), "hf_debug_matmul_f32: clear");
-  const hf_status st = gemm_f32(s, wk, M, N, K, alpha, d_A, a_i, a_k, d_B, b_k, b_j, beta, d_C, ldc);
+  const hf_status st =
+      gemm_f32(s, wk, M, N, K, alpha, d_A, a_i, a_k, d_B, b_k, b_j, beta, d_C, ldc, d_C, 0.f);
   if (st != HF_OK) return st;
   if (h_err) {
     HF_CUDA_TRY(cudaMemcpyAsync(h_err, wk.err, sizeof(int32_t), cudaMemcpyDeviceToHost, s),

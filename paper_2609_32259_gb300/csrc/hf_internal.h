@@ -140,12 +140,14 @@ struct GemmWork {
 };
 // Bytes of the three bf16 planes of an operand with `rows` rows and K columns.
 size_t gemm_planes_bytes(int64_t rows, int64_t K);
-// C[M x N] = alpha op(A) op(B) + beta C (row-major C, leading dimension ldc),
-// op(A)(i, k) = A[i * a_i + k * a_k], op(B)(k, j) = B[k * b_k + j * b_j], in
-// fp32 accuracy on the tensor cores (hf_gemm.cu).  Asynchronous on s.
+// C[M x N] = alpha op(A) op(B) + beta C_in + diag I (row-major C and C_in,
+// leading dimension ldc; C_in NULL = C), op(A)(i, k) = A[i * a_i + k * a_k],
+// op(B)(k, j) = B[k * b_k + j * b_j], in fp32 accuracy on the tensor cores
+// (hf_gemm.cu).  Asynchronous on s.
 hf_status gemm_f32(cudaStream_t s, const GemmWork& wk, int M, int N, int K, float alpha,
                    const float* A, int64_t a_i, int64_t a_k, const float* B, int64_t b_k,
-                   int64_t b_j, float beta, float* C, int64_t ldc);
+                   int64_t b_j, float beta, float* C, int64_t ldc, const float* Cin = nullptr,
+                   float diag = 0.f);
 
 }  // namespace hf
 

@@ -36,8 +36,9 @@ constexpr size_t kPartialBytes = static_cast<size_t>(2) * 96 * 65536 * sizeof(fl
 
 hf_status sgemm(const GemmWork& h, cudaStream_t s, int M, int N, int K, float alpha,
                 const float* A, int64_t a_i, int64_t a_k, const float* B, int64_t b_k,
-                int64_t b_j, float beta, float* C, int64_t ldc) {
-  return gemm_f32(s, h, M, N, K, alpha, A, a_i, a_k, B, b_k, b_j, beta, C, ldc);
+                int64_t b_j, float beta, float* C, int64_t ldc, const float* Cin = nullptr,
+                float diag = 0.f) {
+  return gemm_f32(s, h, M, N, K, alpha, A, a_i, a_k, B, b_k, b_j, beta, C, ldc, Cin, diag);
 }
 
 // A product over the sample axis (K = N samples) in chunks of kMomentChunk:
@@ -57,7 +58,9 @@ hf_status moment_product(const GemmWork& h, cudaStream_t s, int M, int N, int64_
 __device__ __forceinline__ float ld(const __nv_bfloat16* p) { return __bfloat162float(*p); }
 __device__ __forceinline__ float ld(const float* p) { return *p; }
 
-// Column sums of w X and w Y, sum w, and sum w |x|^2 (fp64 accumulation).
+// Column sums of w X and w Y, sum w, and sum w |x|^2.  A thread sums its
+// column over the block's rows (at most a few hundred) in fp32; the partial
+// sums meet in fp64 (GB300's fp64 rate is a small fraction of fp32's).
 template <typename T>
 __global__ void rc_stats_kernel(const T* X, const T* Y, const float* w, int64_t N, int dx,
                                 int dy, double* sx, double* sy, double* sw_ss) {
@@ -65,19 +68,24 @@ __global__ void rc_stats_kernel(const T* X, const T* Y, const float* w, int64_t 
   const int col = blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t rows = (N + gridDim.y - 1) / gridDim.y;
   const int64_t n0 = blockIdx.y * rows, n1 = min(N, n0 + rows);
-  double s = 0.0, ssq = 0.0, swt = 0.0;
+  float s = 0.f, ssq = 0.f, swt = 0.f;
   if (col < d) {
     for (int64_t n = n0; n < n1; ++n) {
-      const double wn = w[n];
-      const double v = col < dx ? ld(X + n * dx + col) : ld(Y + n * dy + (col - dx));
-      s += wn * v;
-      if (col < dx) ssq += wn * v * v;
+      const float wn = w[n];
+      const float v = col < dx ? ld(X + n * dx + col) : ld(Y + n * dy + (col - dx));
+      const float wv = wn * v;
+      s += wv;
+      if (col < dx) ssq = fmaf(wv, v, ssq);
       if (col == 0) swt += wn;
     }
-    atomicAdd(col < dx ? sx + col : sy + (col - dx), s);
-    if (col < dx) atomicAdd(sw_ss + 1, ssq);
-    if (col == 0) atomicAdd(sw_ss, swt);
+    atomicAdd(col < dx ? sx + col : sy + (col - dx), static_cast<double>(s));
+    if (col == 0) atomicAdd(sw_ss, static_cast<double>(swt));
   }
+  // the shared sum of squares: every lane of the warp takes part (lanes
+  // past the columns hold 0), one fp64 atomic per warp
+  double q = ssq;
+  for (int o = 16; o > 0; o >>= 1) q += __shfl_xor_sync(0xffffffffu, q, o);
+  if ((threadIdx.x & 31) == 0 && q != 0.0) atomicAdd(sw_ss + 1, q);
 }
 
 // fp32 means mu_x (of X, not yet divided by r), mu_y, and [1 / W, 1 / r].
@@ -111,16 +119,19 @@ __global__ void rc_center_kernel(const T* X, const T* Y, const float* w, int64_t
   }
 }
 
-// S += reg * trace(S) / d * I  (one block).
+// S += reg * trace(S) / d * I  (one block of 256 threads).
 __global__ void rc_ridge_kernel(float* S, int d, float reg) {
-  __shared__ float tr;
-  if (threadIdx.x == 0) {
-    double t = 0.0;
-    for (int i = 0; i < d; ++i) t += S[static_cast<int64_t>(i) * d + i];
-    tr = static_cast<float>(t / d);
-  }
+  __shared__ double part[256];
+  double t = 0.0;
+  for (int i = threadIdx.x; i < d; i += blockDim.x) t += S[static_cast<int64_t>(i) * d + i];
+  part[threadIdx.x] = t;
   __syncthreads();
-  for (int i = threadIdx.x; i < d; i += blockDim.x) S[static_cast<int64_t>(i) * d + i] += reg * tr;
+  for (int o = blockDim.x / 2; o > 0; o >>= 1) {
+    if (threadIdx.x < o) part[threadIdx.x] += part[threadIdx.x + o];
+    __syncthreads();
+  }
+  const float add = reg * static_cast<float>(part[0] / d);
+  for (int i = threadIdx.x; i < d; i += blockDim.x) S[static_cast<int64_t>(i) * d + i] += add;
 }
 
 // out = a * in + b * I (square, or the leading square of a d x e matrix when
@@ -134,40 +145,71 @@ __global__ void rc_affine_kernel(float* out, const float* in, int64_t n_el, int 
   }
 }
 
-// sum of squares (fp64) of x, or of (x - I) when minus_identity.
+// sum of squares of x, or of (x - I) when minus_identity: fp32 per thread
+// (a few dozen elements each), fp64 across threads.
 __global__ void rc_sumsq_kernel(const float* x, int64_t n_el, int cols, int minus_identity,
                                 double* out) {
-  double s = 0.0;
+  float s = 0.f;
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n_el;
        i += (int64_t)gridDim.x * blockDim.x) {
     const int64_t r = i / cols, c = i - r * cols;
-    const double v = x[i] - (minus_identity && r == c ? 1.0 : 0.0);
-    s += v * v;
+    const float v = x[i] - (minus_identity && r == c ? 1.f : 0.f);
+    s = fmaf(v, v, s);
   }
-  for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-  if ((threadIdx.x & 31) == 0) atomicAdd(out, s);
+  double q = s;
+  for (int o = 16; o > 0; o >>= 1) q += __shfl_xor_sync(0xffffffffu, q, o);
+  if ((threadIdx.x & 31) == 0) atomicAdd(out, q);
 }
 
-// b = mu_y - mu_z A;  W_out = A^T in the output type.
+// W_out = A^T in the output type: 32 x 32 tiles through shared memory, read
+// and written along rows.
 template <typename T>
-__global__ void rc_output_kernel(const float* A, int dx, int dy, const double* sx,
-                                 const double* sy, const double* sw_ss, T* W_out, float* b_out) {
+__global__ void rc_transpose_kernel(const float* A, int dx, int dy, T* W_out) {
+  __shared__ float tile[32][33];
+  const int k0 = blockIdx.y * 32, j0 = blockIdx.x * 32;
+  for (int i = threadIdx.y; i < 32; i += blockDim.y) {
+    const int k = k0 + i, j = j0 + threadIdx.x;
+    if (k < dx && j < dy) tile[i][threadIdx.x] = A[static_cast<int64_t>(k) * dy + j];
+  }
+  __syncthreads();
+  for (int i = threadIdx.y; i < 32; i += blockDim.y) {
+    const int j = j0 + i, k = k0 + threadIdx.x;
+    if (k < dx && j < dy) W_out[static_cast<int64_t>(j) * dx + k] = T(tile[threadIdx.x][i]);
+  }
+}
+
+// b = mu_y - mu_z A, mu_z = mu_x / r.  Block (j-tile of 32 columns, slice of
+// 256 rows of A): thread (j, sub) sums 32 rows in fp64, the block combines its
+// eight partial sums and adds them to bacc[j] (cleared before).
+__global__ void rc_bias_partial_kernel(const float* A, int dx, int dy, const double* sx,
+                                       const double* sw_ss, double* bacc) {
+  __shared__ double part[8][33];
   const double W = sw_ss[0];
-  const double r = sqrt(sw_ss[1] / (static_cast<double>(dx) * W));
-  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < (int64_t)dx * dy;
-       i += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t j = i / dx, k = i - j * dx;  // W_out[j][k] = A[k][j]
-    W_out[i] = T(A[k * dy + j]);
+  const double inv = 1.0 / (W * sqrt(sw_ss[1] / (static_cast<double>(dx) * W)));
+  const int j = blockIdx.x * 32 + threadIdx.x;
+  const int kbase = blockIdx.y * 256 + threadIdx.y * 32;
+  double s = 0.0;
+  if (j < dy)
+    for (int k = kbase; k < min(dx, kbase + 32); ++k)
+      s = fma(sx[k] * inv, static_cast<double>(A[static_cast<int64_t>(k) * dy + j]), s);
+  part[threadIdx.y][threadIdx.x] = s;
+  __syncthreads();
+  if (threadIdx.y == 0 && j < dy) {
+    double t = 0.0;
+    for (int q = 0; q < 8; ++q) t += part[q][threadIdx.x];
+    atomicAdd(bacc + j, t);
   }
-  for (int j = blockIdx.x * blockDim.x + threadIdx.x; j < dy; j += gridDim.x * blockDim.x) {
-    double s = sy[j] / W;
-    for (int k = 0; k < dx; ++k) s -= (sx[k] / W / r) * A[static_cast<int64_t>(k) * dy + j];
-    b_out[j] = static_cast<float>(s);
-  }
+}
+
+__global__ void rc_bias_final_kernel(const double* sy, const double* sw_ss, const double* bacc,
+                                     int dy, float* b_out) {
+  const double W = sw_ss[0];
+  for (int j = blockIdx.x * blockDim.x + threadIdx.x; j < dy; j += gridDim.x * blockDim.x)
+    b_out[j] = static_cast<float>(sy[j] / W - bacc[j]);
 }
 
 struct Rc {
-  size_t stats, mu, xc, yc, sz, sy, szy, p1, p2, p3, p4, sz_ih, sy_ih, sy_h, m, x1, x2, xtx, a,
+  size_t stats, bacc, mu, xc, yc, sz, sy, szy, p1, p2, p3, p4, sz_ih, sy_ih, sy_h, m, x1, x2, xtx, a,
       planes_a, planes_b, partial, err, total;
   size_t planes_bytes;
 };
@@ -183,6 +225,7 @@ Rc rc_layout(int64_t N, int dx, int dy) {
   const size_t f = sizeof(float);
   const size_t dmax = static_cast<size_t>(dx > dy ? dx : dy);
   L.stats = take(sizeof(double) * (dx + dy + 4));
+  L.bacc = take(sizeof(double) * dy);
   L.mu = take(f * (dx + dy + 2));
   L.xc = take(f * N * dx);
   L.yc = take(f * N * dy);
@@ -252,8 +295,8 @@ hf_status ns_sqrt(cudaStream_t s, const GemmWork& h, const float* S, int d, floa
   double prev = 1e30;
   for (; it < kMaxIter; ++it) {
     // T = 1.5 I - 0.5 Z Y
-    rc_affine_kernel<<<grid, 256, 0, s>>>(T, nullptr, n_el, d, 0.f, 1.5f);
-    if ((st = sgemm(h, s, d, d, d, -0.5f, Z, d, 1, Y, d, 1, 1.f, T, d)) != HF_OK) return st;
+    if ((st = sgemm(h, s, d, d, d, -0.5f, Z, d, 1, Y, d, 1, 0.f, T, d, nullptr, 1.5f)) != HF_OK)
+      return st;
     if (it % 4 == 3) {
       double e2 = 0.0;
       HF_CUDA_TRY(cudaMemsetAsync(dscr, 0, sizeof(double), s), "clear");
@@ -305,8 +348,8 @@ hf_status ns_polar(cudaStream_t s, const GemmWork& h, const float* M, int dx, in
       if (converged(sqrt(e2 / dy), &prev)) break;
     }
     // X2 = 1.5 X - 0.5 X P
-    rc_affine_kernel<<<grid, 256, 0, s>>>(X2, X, n_el, dy, 1.5f, 0.f);
-    if ((st = sgemm(h, s, dx, dy, dy, -0.5f, X, dy, 1, P, dy, 1, 1.f, X2, dy)) != HF_OK) return st;
+    if ((st = sgemm(h, s, dx, dy, dy, -0.5f, X, dy, 1, P, dy, 1, 1.5f, X2, dy, X)) != HF_OK)
+      return st;
     std::swap(X, X2);
   }
   *iters = it;
@@ -338,7 +381,8 @@ hf_status recolor_typed(int64_t N, int dx, int dy, const void* Xv, const void* Y
   HF_CUDA_TRY(cudaMemsetAsync(h.err, 0, sizeof(int32_t), s), "clear");
   HF_CUDA_TRY(cudaMemsetAsync(stats, 0, sizeof(double) * (dx + dy + 4), s), "clear");
   const int d = dx + dy;
-  dim3 sgrid((d + 255) / 256, static_cast<unsigned>(std::min<int64_t>(N, 256)));
+  // at most ~128 rows per thread, so the per-thread fp32 sums stay short
+  dim3 sgrid((d + 255) / 256, static_cast<unsigned>(std::min<int64_t>((N + 127) / 128, 65535)));
   rc_stats_kernel<T><<<sgrid, 256, 0, s>>>(X, Y, w, N, dx, dy, sx, sy, sw_ss);
   float* mu = F(L.mu);
   rc_mean_kernel<<<(d + 255) / 256, 256, 0, s>>>(sx, sy, sw_ss, dx, dy, mu, mu + d);
@@ -376,8 +420,15 @@ hf_status recolor_typed(int64_t N, int dx, int dy, const void* Xv, const void* Y
   if ((st = sgemm(h, s, dx, dy, dx, 1.f, F(L.sz_ih), dx, 1, R, dy, 1, 0.f, tmp, dy)) != HF_OK) return st;
   if ((st = sgemm(h, s, dx, dy, dy, 1.f, tmp, dy, 1, F(L.sy_h), dy, 1, 0.f, F(L.a), dy)) != HF_OK)
     return st;
-  rc_output_kernel<T><<<1024, 256, 0, s>>>(F(L.a), dx, dy, sx, sy, sw_ss, static_cast<T*>(W_out),
-                                           b_out);
+  {
+    double* bacc = reinterpret_cast<double*>(ws + L.bacc);
+    HF_CUDA_TRY(cudaMemsetAsync(bacc, 0, sizeof(double) * dy, s), "clear");
+    rc_transpose_kernel<T><<<dim3((dy + 31) / 32, (dx + 31) / 32), dim3(32, 8), 0, s>>>(
+        F(L.a), dx, dy, static_cast<T*>(W_out));
+    rc_bias_partial_kernel<<<dim3((dy + 31) / 32, (dx + 255) / 256), dim3(32, 8), 0, s>>>(
+        F(L.a), dx, dy, sx, sw_ss, bacc);
+    rc_bias_final_kernel<<<(dy + 255) / 256, 256, 0, s>>>(sy, sw_ss, bacc, dy, b_out);
+  }
   HF_CUDA_TRY(cudaGetLastError(), "hf_recolor_fit: output launch");
   double hs[2];
   int32_t gemm_err = 0;
