@@ -54,6 +54,26 @@ def test_batch_mixing_operand_paths():
         assert torch.equal(c.job.receiver, ref), c.w.name
 
 
+def test_batch_mixing_layer_tables():
+    """A KV Ridge direction (an explicit eight-segment table), a paper3
+    direction and an interpolated one in one batch: each equals its single
+    transfer and stays within the parity tolerance of the oracle."""
+    ws = [W.qwen25_to_llama_kv_ridge(600),
+          W.qwen25_to_llama_batched(n_req=2, lo=100, hi=400, seed=44).with_(L_s=28, L_r=32),
+          W.llama_to_ministral(500).with_(L_s=5, L_r=6, layer_mode="interp")]
+    cases = [Case(w, sentinel=SENTINEL).run() for w in ws]
+    single = [c.job.receiver.clone() for c in cases]
+    for c in cases:
+        c.job.receiver.fill_(SENTINEL)
+    B.transfer_batch([c.job.plan for c in cases], [c.sender for c in cases],
+                     [c.job.receiver for c in cases])
+    torch.cuda.synchronize()
+    for c, ref in zip(cases, single):
+        assert torch.equal(c.job.receiver, ref), c.w.name
+    cases[0].check_parity(layers=[0, 13, 31])
+    cases[2].check_parity()
+
+
 def test_batch_of_one_and_empty_batch():
     c = Case(W.message_round(msg_tokens=40)[1], sentinel=SENTINEL).run()
     ref = c.job.receiver.clone()

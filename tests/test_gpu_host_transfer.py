@@ -31,6 +31,8 @@ CASES = {
     "paged_batched": (lambda: W.qwen25_to_llama_batched(n_req=3, lo=60, hi=500, seed=8)
                       .with_(L_s=4, L_r=5), (2, 5)),
     "interp_f32": (W.tiny, (4,)),
+    "kv_ridge_paged": (lambda: W.qwen25_to_llama_kv_ridge(1).with_(paged=True,
+                                                                r_tokens=(300, 77)), (3, 32)),
 }
 
 

@@ -255,6 +255,24 @@ EDGE = {
     "message_span_rotated_overlap": lambda: W.llama_to_ministral(150).with_(
         L_s=3, L_r=3, span_gap=2000, sender_k_rotated=True, s_pos0=(2000,),
         align_mode="overlap_mean", r_pos0=(1500,)),
+    # KV Ridge's eight one-layer segments with a paged receiver cache (an
+    # empty request in the middle), and with fp32 caches and maps
+    "kv_ridge_batched_paged": lambda: W.qwen25_to_llama_kv_ridge(1).with_(
+        paged=True, r_tokens=(420, 0, 129)),
+    "kv_ridge_f32": lambda: W.qwen25_to_llama_kv_ridge(300).with_(dtype="f32"),
+    # eight computed segments, paged receiver, fp32
+    "explicit_eight_segments_paged_f32": lambda: _explicit(
+        W.qwen25_to_llama_batched(n_req=3, lo=30, hi=250, seed=33).with_(
+            L_s=9, L_r=3, dtype="f32"), n_seg=8, n_terms=2),
+    # the staged operand builder (computed bf16 rows) with paging and spans,
+    # with key norm and a caller RoPE table, and with same-index pairing
+    "interp_batched_paged_spans": lambda: W.qwen25_to_llama_batched(
+        n_req=3, lo=40, hi=300, seed=41).with_(L_s=5, L_r=4, layer_mode="interp",
+                                               span_gap=500),
+    "interp_knorm_rope_table": lambda: W.llama_to_ministral(900).with_(
+        L_s=6, L_r=5, layer_mode="interp", knorm=True, rope_table=True, r_pos0=(4000,)),
+    "interp_same_index": lambda: W.llama_to_qwen25(517).with_(
+        L_s=7, L_r=3, layer_mode="interp", align_mode="same_index"),
 }
 
 
