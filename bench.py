@@ -42,6 +42,9 @@ def parse():
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--round-built-operands", action="store_true",
                     help="computed operand rows rounded once to bf16 (no value + residual pair)")
+    ap.add_argument("--pool-before-map", action="store_true",
+                    help="overlap mean pooling before the map (pooled operand rows per distinct "
+                         "row) instead of pooling the mapped sender rows")
     return ap.parse_args()
 
 
@@ -182,14 +185,17 @@ def kernel_sources_sha256():
 def algorithmic_work(w, tok, U, n_distinct_cols):
     """FLOPs and bytes a transfer cannot avoid.
 
-    FLOP: 2 * (2 L_r) * U * K * d_r, U = distinct alignment rows (rows with
-    identical inputs share one map output before RoPE).
+    FLOP: 2 * (2 L_r) * min(U, S) * K * d_r, U = distinct alignment rows
+    (rows with identical inputs share one map output before RoPE), S = the
+    sender tokens the alignment references: the map is linear, so the
+    pooling can come before it (U rows) or after it (S rows), whichever is
+    fewer.
     Bytes: the receiver cache written once; every referenced sender row read
     once per sender layer (the three-layer neighbourhoods of these depth
     pairs touch every sender layer); the maps and biases read once; the CSR
     and per-row metadata."""
     e = 2 if w.dtype == "bf16" else 4
-    flops = 2.0 * 2 * w.L_r * U * w.K * w.d_r
+    flops = 2.0 * 2 * w.L_r * min(U, n_distinct_cols) * w.K * w.d_r
     T_r = tok.T_r
     # sender layers the layer table reads (all of them for Eq. 1 and the
     # interpolation on these depth pairs; the selected ones for an explicit table)
@@ -249,10 +255,33 @@ class OracleSample:
                                H_r=w.H_r, D_r=w.D_r, pos=self.pos, inv_freq_r=self.inv)
 
 
-def _copied_operands(w):
+def _pool_after_map(w, pool_before_map=False):
+    """Overlap mean pooling applied to the mapped sender rows (the library's
+    choice unless the caller asks otherwise or the pooled row itself is
+    needed: key norm, sender keys rotated back per position)."""
+    return (w.align_mode == "overlap_mean" and not pool_before_map and not w.knorm
+            and not w.sender_k_rotated)
+
+
+def launches_per_step(w, pool_before_map=False):
+    """Kernel launches of one hf_align_build + hf_plan_create + hf_transfer:
+    alignment (TA: sender check, match, max-scan; same-index: one kernel;
+    overlap: sender check, count, scan, fill), plan (init, layer table,
+    rows, scan, runs; sender positions or span rows; window key scan and
+    windows when the pooling follows the map), one transfer kernel."""
+    align = {"ta": 3, "same_index": 1, "overlap_mean": 4}[w.align_mode]
+    plan = (5 + (1 if (w.sender_k_rotated or w.span_gap) else 0)
+            + (2 if _pool_after_map(w, pool_before_map) else 0))
+    return align + plan + 1
+
+
+def _copied_operands(w, pool_before_map=False):
     """Every map input row is a copy of one sender row: one-entry alignment
-    rows, segments of one sender layer of weight 1, keys without RoPE."""
-    if w.align_mode == "overlap_mean" or w.layer_mode == "interp" or w.sender_k_rotated:
+    rows (or sender rows whose maps are pooled afterwards), segments of one
+    sender layer of weight 1, keys without RoPE."""
+    if w.layer_mode == "interp" or w.sender_k_rotated:
+        return False
+    if w.align_mode == "overlap_mean" and not _pool_after_map(w, pool_before_map):
         return False
     if w.layer_mode == "explicit":
         return all(len(terms) == 1 and float(terms[0]) == 1.0
@@ -349,7 +378,8 @@ def run_ours(args):
     Wm, b, r = W.maps(w, dev)
     paged = W.paged_layout(w, tok) if w.paged else None
     job = pipeline.job_from_workload(w, tok, sender, Wm, b, r, paged=paged, device=dev,
-                                     round_built_operands=args.round_built_operands)
+                                     round_built_operands=args.round_built_operands,
+                                     pool_before_map=args.pool_before_map)
     stream = torch.cuda.current_stream(dev)
 
     for _ in range(max(3, args.warmup)):
@@ -518,7 +548,7 @@ def run_ours(args):
                "sample": (f"{samp.n_rows} contiguous receiver rows x {w.L_r} layers x K/V "
                           f"of {w.name} (dense fp64 numpy oracle as written)")}
 
-    launches_per_step = 3 + 4 + 1  # align (3 kernels), plan (4), transfer (1)
+    launches = launches_per_step(w, args.pool_before_map)
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_ms,
@@ -529,7 +559,10 @@ def run_ours(args):
                    "distinct_rows": U, "sender": f"{w.L_s}x{w.H_s}x{w.D_s}",
                    "receiver": f"{w.L_r}x{w.H_r}x{w.D_r}",
                    "mode": f"{w.align_mode}+{w.layer_mode}",
-                   "operands": ("copied sender rows" if _copied_operands(w)
+                   "pooling": ("after the map (mapped sender rows pooled in the epilogue)"
+                               if _pool_after_map(w, args.pool_before_map) else
+                               "before the map" if w.align_mode == "overlap_mean" else None),
+                   "operands": ("copied sender rows" if _copied_operands(w, args.pool_before_map)
                                 else "computed rows rounded once to bf16"
                                 if args.round_built_operands or w.dtype != "bf16"
                                 else "computed rows as bf16 value + residual"),
@@ -537,7 +570,7 @@ def run_ours(args):
                           "256 MB L2 flush write between steps (outside the timed events)"),
                    "parallelism": "replicas" if world > 1 else "single"},
         "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
-        "gpu_launches": launches_per_step * args.steps, "device_status": status,
+        "gpu_launches": launches * args.steps, "device_status": status,
     }
     if rank == 0:
         print(json.dumps(line), flush=True)
@@ -642,7 +675,8 @@ def run_batch(args):
                    "l2": "maps (1.2 GB) larger than L2 (no flush)",
                    "parallelism": "single"},
         "roofline": roof, "cpu_baseline": None, "e2e": None, "clocks": clk,
-        "gpu_launches": (8 * len(jobs)) * args.steps, "device_status": status,
+        "gpu_launches": (sum(launches_per_step(w) - 1 for w in ws) + 1) * args.steps,
+        "device_status": status,
     }
     print(json.dumps(line), flush=True)
     for j in jobs:

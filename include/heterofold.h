@@ -110,6 +110,11 @@ typedef enum {
 #define HF_CHECK_CAPACITY      0x10 /* the CSR did not fit the given capacity */
 #define HF_CHECK_TIMEOUT       0x20 /* a pipeline wait gave up (internal error) */
 #define HF_CHECK_INTERNAL      0x40 /* a launch invariant did not hold (internal error) */
+#define HF_CHECK_POOL_WINDOW   0x80 /* pooling after the map: a CSR row's columns do not
+                                       fit its 128-token window (rows whose first
+                                       columns decrease, or a row spanning 128 or more
+                                       sender tokens); create the plan with
+                                       pool_before_map = 1 */
 
 /*
  * hf_align_build — alignment CSR from character-end offsets (Section 3.1,
@@ -239,6 +244,22 @@ typedef struct {
      feature, which at 1e9 outputs can exceed 2e-2 absolute).  Ignored for
      copied rows and fp32 plans. */
   int32_t round_built_operands;
+
+  /* Overlap mean pooling (HF_ALIGN_OVERLAP_MEAN) is linear, so the map
+     commutes with it: y_j = (sum_e w_e x_{col_e} / r) A + b
+                           = sum_e w_e (x_{col_e} A) / r + b.
+     0 (default): plans in that mode without key norm or rotated sender keys
+     map sender rows and pool the mapped rows in the epilogue (pooling after
+     the map): the map input rows are sender rows (copied, or blended across
+     layers), windows of 128 consecutive aligned sender tokens with a stride
+     of 128 - h (h = the widest row's column span), and each receiver row is
+     pooled from the window holding its columns.  Needs rows whose first
+     columns do not decrease and that span fewer than 128 sender tokens
+     (as hf_align_build makes them); otherwise HF_CHECK_POOL_WINDOW is set
+     and the rows that do not fit are left incomplete (every access stays
+     inside the caches).  1: pool before the map (map input rows computed
+     per distinct CSR row), with no such limit. */
+  int32_t pool_before_map;
 } hf_plan_desc;
 
 typedef struct hf_plan_s* hf_plan;

@@ -32,7 +32,7 @@ DTYPES = {"bf16": 0, "f32": 1}
 CHECK_BITS = {
     0x01: "HF_CHECK_BAD_OFFSETS", 0x02: "HF_CHECK_BAD_COLUMN", 0x04: "HF_CHECK_BAD_ROW",
     0x08: "HF_CHECK_BAD_BLOCK", 0x10: "HF_CHECK_CAPACITY", 0x20: "HF_CHECK_TIMEOUT",
-    0x40: "HF_CHECK_INTERNAL",
+    0x40: "HF_CHECK_INTERNAL", 0x80: "HF_CHECK_POOL_WINDOW",
 }
 
 EXPORTED = ("hf_align_build", "hf_plan_workspace_size", "hf_plan_create", "hf_transfer",
@@ -69,6 +69,7 @@ class PlanDesc(ctypes.Structure):
         ("n_seg", ctypes.c_int32), ("n_terms", ctypes.c_int32),
         ("h_seg_layer", _i32p), ("h_seg_w", _f32p),
         ("round_built_operands", ctypes.c_int32),
+        ("pool_before_map", ctypes.c_int32),
     ]
 
 
@@ -193,7 +194,7 @@ class Desc:
                  n_blocks=0, max_blocks_per_req=0, d_block_table=None, inv_freq_r=None,
                  sender_k_rotated=False, theta_s=0.0, inv_freq_s=None, s_pos0=None,
                  seg_layer=None, seg_w=None, s_row0=None, sender_rows=0,
-                 round_built_operands=False):
+                 round_built_operands=False, pool_before_map=False):
         self._s = _host_i32(s_tok_ptr)
         self._r = _host_i32(r_tok_ptr)
         self._pos0 = None if r_pos0 is None else _host_i32(r_pos0)
@@ -230,7 +231,8 @@ class Desc:
             n_seg=n_seg, n_terms=n_terms,
             h_seg_layer=_as_i32p(self._segl) if self._segl is not None else None,
             h_seg_w=_f32_or_null(self._segw),
-            round_built_operands=int(round_built_operands))
+            round_built_operands=int(round_built_operands),
+            pool_before_map=int(pool_before_map))
 
 
 def plan_workspace_size(desc: Desc) -> int:

@@ -49,6 +49,11 @@ struct WorkspaceLayout {
   size_t pos;        // int32[T_r]: RoPE position of each receiver row
   size_t dst_row;    // int32[T_r]: destination row of each receiver row
   size_t new_flag;   // int32[T_r]: 1 where a receiver row starts a new distinct row
+  // pooling after the map (overlap mean pooling): windows of 128 aligned
+  // sender tokens with stride S = 128 - h, h the widest row's column span
+  size_t win_info;   // int32[4]: h, S, number of windows, unused
+  size_t row_key;    // int32[T_r]: first column of each row, then its running maximum
+  size_t win_ptr;    // int32[T_s + 2]: first receiver row of each window
   size_t total;
 };
 
@@ -93,6 +98,7 @@ struct hf_plan_s {
   bool rope;    // receiver keys get RoPE
   bool unrot;   // sender keys carry RoPE and are rotated back in the builder
   bool span;    // aligned sender tokens are spans inside a longer sender cache
+  bool pam;     // pooling after the map: map input rows are sender rows in windows
   int64_t s_rows;  // sender-cache rows per (layer, role)
   char* ws;
   size_t ws_bytes;
@@ -120,8 +126,8 @@ hf_status plan_build(const hf_plan_desc* desc, void* d_workspace, size_t workspa
 // launch ends through the bounded waits with HF_CHECK_TIMEOUT.
 hf_status launch_transfer(hf_plan_s* p, const void* sender, void* receiver, cudaStream_t stream,
                           int l_begin = 0, int l_end = -1, bool stall = false);
-// Several plans in one launch: they must share the dtype and the operand
-// path (batch_compatible); n <= kMaxBatch.
+// Several plans in one launch: they must share the dtype, the operand path
+// and where the pooling happens (batch_compatible); n <= kMaxBatch.
 bool batch_compatible(const hf_plan_s* const* plans, int n);
 hf_status launch_transfer_batch(hf_plan_s* const* plans, const void* const* senders,
                                 void* const* receivers, int n, cudaStream_t stream);

@@ -44,6 +44,10 @@ WorkspaceLayout workspace_layout(const hf_plan_desc& d) {
   const int64_t T_r = d.r_tok_ptr[n_req];
   const int64_t n_spos = d.sender_k_rotated ? d.s_tok_ptr[n_req] : 0;
   const int64_t n_srow = d.s_row0 ? d.s_tok_ptr[n_req] : 0;
+  // pooling after the map may apply (the plan decides): window tables
+  const bool pam = d.align_mode == HF_ALIGN_OVERLAP_MEAN && d.pool_before_map == 0;
+  const int64_t n_key = pam ? T_r : 0;
+  const int64_t n_win = pam ? d.s_tok_ptr[n_req] + 2 : 0;
   WorkspaceLayout w{};
   size_t off = 0;
   auto take = [&](size_t bytes) {
@@ -70,6 +74,9 @@ WorkspaceLayout workspace_layout(const hf_plan_desc& d) {
   w.pos = take(sizeof(int32_t) * (size_t)(T_r > 0 ? T_r : 1));
   w.dst_row = take(sizeof(int32_t) * (size_t)(T_r > 0 ? T_r : 1));
   w.new_flag = take(sizeof(int32_t) * (size_t)(T_r > 0 ? T_r : 1));
+  w.win_info = take(sizeof(int32_t) * 4);
+  w.row_key = take(sizeof(int32_t) * (size_t)(n_key > 0 ? n_key : 1));
+  w.win_ptr = take(sizeof(int32_t) * (size_t)(n_win > 0 ? n_win : 1));
   w.total = off;
   return w;
 }
@@ -96,6 +103,9 @@ struct PlanDev {
   int32_t* pos;
   int32_t* dst_row;
   int32_t* new_flag;
+  int32_t* win_info;
+  int32_t* row_key;
+  int32_t* win_ptr;
 };
 
 PlanDev plan_dev(const hf_plan_s* p) {
@@ -120,6 +130,9 @@ PlanDev plan_dev(const hf_plan_s* p) {
   d.pos = reinterpret_cast<int32_t*>(at(p->lay.pos));
   d.dst_row = reinterpret_cast<int32_t*>(at(p->lay.dst_row));
   d.new_flag = reinterpret_cast<int32_t*>(at(p->lay.new_flag));
+  d.win_info = reinterpret_cast<int32_t*>(at(p->lay.win_info));
+  d.row_key = reinterpret_cast<int32_t*>(at(p->lay.row_key));
+  d.win_ptr = reinterpret_cast<int32_t*>(at(p->lay.win_ptr));
   return d;
 }
 
@@ -133,6 +146,7 @@ __global__ void plan_init_kernel(const __grid_constant__ PlanConsts t, PlanDev d
     *d.status = 0;
     *d.n_distinct = 0;
   }
+  if (tid < 4) d.win_info[tid] = 0;
   for (int i = tid; i < 2 * t.L_r; i += blockDim.x) d.inv_r[i] = t.inv_r[i];
   for (int i = tid; i < t.D_r / 2; i += blockDim.x) d.inv_freq[i] = t.inv_freq[i];
   for (int i = tid; i <= t.n_req; i += blockDim.x) d.r_tok_ptr[i] = t.r_tok_ptr[i];
@@ -178,6 +192,7 @@ struct RowArgs {
   int paged, block_size, n_blocks, max_blocks;
   int single_entry;  // rows must be one entry of weight 1
   int span;          // map sender tokens to cache rows through d.srow
+  int pam;           // pooling after the map: row keys and the widest column span
 };
 
 __device__ __forceinline__ void flag(int32_t* status, int bits) { atomicOr(status, bits); }
@@ -208,9 +223,21 @@ __global__ void plan_rows_kernel(RowArgs a) {
     const int32_t e0 = a.row_ptr[j], e1 = a.row_ptr[j + 1];
     if (e1 <= e0) flag(d.status, HF_CHECK_BAD_ROW);
     if (a.single_entry && (e1 - e0 != 1 || a.w[e0] != 1.0f)) flag(d.status, HF_CHECK_BAD_ROW);
+    int32_t kmin = INT_MAX, kmax = -1;
     for (int32_t e = e0; e < e1; ++e) {
       const int32_t k = a.col[e];
-      if (k < 0 || k >= a.T_s) flag(d.status, HF_CHECK_BAD_COLUMN);
+      if (k < 0 || k >= a.T_s) {
+        flag(d.status, HF_CHECK_BAD_COLUMN);
+      } else {
+        kmin = min(kmin, k);
+        kmax = max(kmax, k);
+      }
+    }
+    if (a.pam) {
+      // the row's first valid column (-1: none); made a running maximum by
+      // a scan, it assigns the row to a window
+      d.row_key[j] = kmax >= 0 ? kmin : -1;
+      if (kmax >= 0) atomicMax(&d.win_info[0], kmax - kmin);
     }
     int is_new = (j == r0) ? 1 : 0;
     if (!is_new) {
@@ -251,6 +278,48 @@ __global__ void plan_runs_kernel(RowArgs a) {
     if (j == a.T_r - 1) {
       d.run_ptr[incl] = static_cast<int32_t>(a.T_r);
       *d.n_distinct = incl;
+    }
+  }
+}
+
+// Pooling after the map: window w holds the aligned sender tokens
+// [w S, w S + 128), S = 128 - h with h the widest row's column span, so a
+// row whose first column c satisfies w = floor(c / S) has every column in
+// window w.  After the max-scan row_key[j] is the largest first column of
+// rows 0..j (non-decreasing); window w takes the rows j with
+// floor(row_key[j] / S) = w, win_ptr[w] the first of them.  A row whose
+// columns leave its window (first columns that decrease, or h >= 128) is
+// flagged.
+__global__ void plan_windows_kernel(RowArgs a) {
+  const PlanDev& d = a.d;
+  const int32_t h = d.win_info[0];
+  const bool too_wide = h >= 128;
+  const int32_t S = too_wide ? 1 : 128 - h;
+  const int32_t last = d.row_key[a.T_r - 1];
+  const int32_t n_win = last < 0 ? 0 : last / S + 1;
+  if (blockIdx.x == 0 && threadIdx.x == 0) {
+    d.win_info[1] = S;
+    d.win_info[2] = n_win;
+    if (too_wide) flag(d.status, HF_CHECK_POOL_WINDOW);
+  }
+  const int64_t n = a.T_r > (int64_t)n_win + 1 ? a.T_r : (int64_t)n_win + 1;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    if (i < a.T_r) {
+      const int32_t key = d.row_key[i];
+      if (key >= 0) {
+        const int64_t lo = (int64_t)(key / S) * S;
+        for (int32_t e = a.row_ptr[i]; e < a.row_ptr[i + 1]; ++e) {
+          const int32_t k = a.col[e];
+          if (k >= 0 && k < a.T_s && (k < lo || k >= lo + 128)) flag(d.status, HF_CHECK_POOL_WINDOW);
+        }
+      }
+    }
+    if (i <= n_win) {
+      const int64_t x = i * (int64_t)S;
+      d.win_ptr[i] = x > INT_MAX ? static_cast<int32_t>(a.T_r)
+                                 : lower_bound_i32(d.row_key, static_cast<int>(a.T_r),
+                                                   static_cast<int32_t>(x));
     }
   }
 }
@@ -380,6 +449,8 @@ hf_status validate(const hf_plan_desc* d) {
   }
   if (d->round_built_operands != 0 && d->round_built_operands != 1)
     return bad("round_built_operands must be 0 or 1");
+  if (d->pool_before_map != 0 && d->pool_before_map != 1)
+    return bad("pool_before_map must be 0 or 1");
   if (d->paged) {
     if (d->block_size < 1 || d->n_blocks < 1 || d->max_blocks_per_req < 1 || !d->d_block_table)
       return bad("paged layout needs block_size, n_blocks, max_blocks_per_req, d_block_table");
@@ -424,6 +495,7 @@ hf_status launch_plan_kernels(hf_plan_s* p, const PlanTables& tables, cudaStream
   a.max_blocks = p->desc.max_blocks_per_req;
   a.single_entry = p->desc.align_mode != HF_ALIGN_OVERLAP_MEAN;
   a.span = p->span ? 1 : 0;
+  a.pam = p->pam ? 1 : 0;
   const int64_t want = (p->T_r + 255) / 256;
   const int grid = static_cast<int>(std::min<int64_t>(want, 8LL * device_sm_count()));
   plan_rows_kernel<<<grid, 256, 0, stream>>>(a);
@@ -435,6 +507,13 @@ hf_status launch_plan_kernels(hf_plan_s* p, const PlanTables& tables, cudaStream
                                                    p->span ? 1 : 0);
   }
   plan_runs_kernel<<<grid, 256, 0, stream>>>(a);
+  if (p->pam) {
+    scan_inplace_kernel<ScanMax><<<1, kScanThreads, 0, stream>>>(d.row_key, p->T_r, nullptr);
+    const int64_t n_w = std::max<int64_t>(p->T_r, p->T_s + 2);
+    const int grid_w = static_cast<int>(
+        std::min<int64_t>((n_w + 255) / 256, 8LL * device_sm_count()));
+    plan_windows_kernel<<<grid_w, 256, 0, stream>>>(a);
+  }
   HF_CUDA_TRY(cudaGetLastError(), "plan kernels launch");
   return HF_OK;
 }
@@ -489,12 +568,20 @@ hf_status plan_build(const hf_plan_desc* desc, void* d_workspace, size_t workspa
   }
   p->unrot = desc->sender_k_rotated == 1;
   p->rope = desc->theta_r > 0.0 || desc->h_inv_freq_r != nullptr;
-  p->gather = one_layer_segments && desc->align_mode != HF_ALIGN_OVERLAP_MEAN && !p->unrot;
+  // overlap mean pooling commutes with the map (it is linear): unless the
+  // pooled row itself is needed (key norm, sender keys rotated back per
+  // position) or the caller asks otherwise, the map input rows are sender
+  // rows and the epilogue pools the mapped rows
+  p->pam = desc->align_mode == HF_ALIGN_OVERLAP_MEAN && desc->pool_before_map == 0 &&
+           !p->unrot && desc->d_knorm_w == nullptr;
+  const bool one_entry = desc->align_mode != HF_ALIGN_OVERLAP_MEAN || p->pam;
+  p->gather = one_layer_segments && one_entry && !p->unrot;
   p->split = !p->gather && desc->dtype == HF_BF16 && desc->round_built_operands == 0;
-  // one-entry rows (Token Alignment, same-index) have at most two (term,
-  // entry) pairs per segment, both staged by cp.async; pooled rows have more,
-  // whose direct loads stall the warp anyway (measured slower staged)
-  p->staged = p->split && !p->unrot && desc->align_mode != HF_ALIGN_OVERLAP_MEAN;
+  // one-entry rows (Token Alignment, same-index, sender rows of pooling
+  // after the map) have at most two (term, entry) pairs per segment, both
+  // staged by cp.async; pooled rows have more, whose direct loads stall the
+  // warp anyway (measured slower staged)
+  p->staged = p->split && !p->unrot && one_entry;
   p->ws = static_cast<char*>(d_workspace);
   p->ws_bytes = workspace_bytes;
   p->lay = lay;

@@ -87,6 +87,14 @@ struct XferParams {
   // (atoms_per_stage = 1); otherwise kAtoms atoms of K per A stage
   int split, atoms_per_stage, n_batoms;  // n_batoms: B atoms (map atoms of K) per tile
   int staged;  // split one-entry rows built by build_rows_staged
+  // pooling after the map: the tile rows of CTA rank k in pair tile m are the
+  // aligned sender tokens of window w = 2m + k, [w S, w S + 128) (S =
+  // win_info[1]); the receiver rows [win_ptr[w], win_ptr[w+1]) are pooled
+  // from them in the epilogue
+  int pam;
+  const int32_t* win_info;  // h, S, number of windows
+  const int32_t* win_ptr;
+  const int32_t* pos;       // RoPE position of every receiver row
   int stages_a, stages_b, lag;  // A ring (stages), B ring (atoms), loader groups in flight
   int rope, paged, knorm, unrot, D_s;
   int stall;  // test hook: the map producer withholds its first atom (hf_debug_transfer_stalled)
@@ -131,6 +139,23 @@ __device__ __forceinline__ void decode_tile(int tile, int tiles_per_lc, int n_ti
 __device__ __forceinline__ void raise_timeout(const XferParams& P, volatile int* abort_flag) {
   atomicOr(P.status, HF_CHECK_TIMEOUT);
   *abort_flag = 1;
+}
+
+// Pooling after the map: the aligned sender token of row r (0..127) of the
+// window of CTA row0 in pair tile m, w = 2m + row0/128, token w S + r (the
+// last token past the end; those rows are never pooled).
+__device__ __forceinline__ int pam_token(const XferParams& P, int m, int row0, int r) {
+  const int w = (m * kPairRows + row0) >> 7;
+  const int64_t k = static_cast<int64_t>(w) * __ldg(P.win_info + 1) + r;
+  return static_cast<int>(k < P.T_s ? k : P.T_s - 1);
+}
+
+// Kernel variants fix pooling after the map at compile time (kPam 0: off,
+// 1: on) so that neither path carries the other's registers; kPam 2 reads
+// it from the parameters (fp32 and multi-direction launches).
+template <int kPam>
+__device__ __forceinline__ bool pam_on(const XferParams& P) {
+  return kPam == 2 ? P.pam != 0 : kPam == 1;
 }
 
 // Accumulates w * (8 bf16 | 4 fp32 values) into acc.
@@ -374,6 +399,140 @@ __device__ __forceinline__ void copy_epilogue(const XferParams& P, uint32_t ta,
   }
 }
 
+// Pooling after the map, one lane's receiver rows [jb, je) of a window
+// whose first aligned sender token is `base`: the staged rows hold
+// z_i / r (i = token - base) for four rotation pairs of up to two heads, and
+// y_j = sum_e w_e z_{col_e} / r + b, rotated at the receiver position of j
+// for keys.  Positions of consecutive rows of a request are consecutive, so
+// the angles advance by one position per row (re-anchored every 16 rows and
+// wherever the position jumps).
+template <typename T>
+__device__ __forceinline__ void pam_walk(int jb, int je, int base, const float* stg, int qq,
+                                         bool two_heads, bool do_rope, const float* f,
+                                         const float* C1, const float* S1, const float4* bias4,
+                                         const XferParams& P, T* out_lc, int ocol, int q,
+                                         int half) {
+  if (jb >= je) return;
+  int expect = INT_MIN;  // position for which cs/sn are valid
+  float cs[4] = {1.f, 1.f, 1.f, 1.f}, sn[4] = {0.f, 0.f, 0.f, 0.f};
+  int e1 = __ldg(P.row_ptr + jb);
+  for (int j = jb; j < je; ++j) {
+    const int e0 = e1;
+    e1 = __ldg(P.row_ptr + j + 1);
+    float4 x0 = make_float4(0.f, 0.f, 0.f, 0.f), y0 = x0, x1 = x0, y1 = x0;
+    for (int e = e0; e < e1; ++e) {
+      const int loc = __ldg(P.col + e) - base;
+      if (loc < 0 || loc >= kBM) continue;  // flagged at plan creation
+      const float wt = __ldg(P.w + e);
+      const float* urow = stg + loc * 64;
+      const int sw = loc & 7;
+      const float4 a = *reinterpret_cast<const float4*>(urow + ((qq ^ sw) << 2));
+      const float4 b = *reinterpret_cast<const float4*>(urow + (((4 + qq) ^ sw) << 2));
+      x0 = make_float4(fmaf(wt, a.x, x0.x), fmaf(wt, a.y, x0.y), fmaf(wt, a.z, x0.z),
+                       fmaf(wt, a.w, x0.w));
+      y0 = make_float4(fmaf(wt, b.x, y0.x), fmaf(wt, b.y, y0.y), fmaf(wt, b.z, y0.z),
+                       fmaf(wt, b.w, y0.w));
+      if (two_heads) {
+        const float4 a1 = *reinterpret_cast<const float4*>(urow + 32 + ((qq ^ sw) << 2));
+        const float4 b1 = *reinterpret_cast<const float4*>(urow + 32 + (((4 + qq) ^ sw) << 2));
+        x1 = make_float4(fmaf(wt, a1.x, x1.x), fmaf(wt, a1.y, x1.y), fmaf(wt, a1.z, x1.z),
+                         fmaf(wt, a1.w, x1.w));
+        y1 = make_float4(fmaf(wt, b1.x, y1.x), fmaf(wt, b1.y, y1.y), fmaf(wt, b1.z, y1.z),
+                         fmaf(wt, b1.w, y1.w));
+      }
+    }
+    x0 = make_float4(x0.x + bias4[0].x, x0.y + bias4[0].y, x0.z + bias4[0].z, x0.w + bias4[0].w);
+    y0 = make_float4(y0.x + bias4[1].x, y0.y + bias4[1].y, y0.z + bias4[1].z, y0.w + bias4[1].w);
+    x1 = make_float4(x1.x + bias4[2].x, x1.y + bias4[2].y, x1.z + bias4[2].z, x1.w + bias4[2].w);
+    y1 = make_float4(y1.x + bias4[3].x, y1.y + bias4[3].y, y1.z + bias4[3].z, y1.w + bias4[3].w);
+    if (do_rope) {
+      const int p = __ldg(P.pos + j);
+      if (p != expect || ((j - jb) & 15) == 0) {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) rope_sincos(p, f[k], &sn[k], &cs[k]);
+      } else {  // advance every angle by one position
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const float t = cs[k] * C1[k] - sn[k] * S1[k];
+          sn[k] = sn[k] * C1[k] + cs[k] * S1[k];
+          cs[k] = t;
+        }
+      }
+      expect = p + 1;
+      rotate4(x0, y0, cs, sn);
+      if (two_heads) rotate4(x1, y1, cs, sn);
+    }
+    const int drow = P.paged ? __ldg(P.dst_row + j) : j;
+    if (drow >= 0) {
+      T* o = out_lc + static_cast<int64_t>(drow) * P.d_r + ocol + q + 4 * qq;
+      store4(o, x0);
+      store4(o + half, y0);
+      if (two_heads) {
+        store4(o + 2 * half, x1);
+        store4(o + 3 * half, y1);
+      }
+    }
+  }
+}
+
+// Epilogue of a tile with pooling after the map (both roles): TMEM row i of
+// this CTA is the product of aligned sender token base + i; per 16 rotation
+// pairs of a head pair, warp (g, sp), e < 8, stages z / r of TMEM lane
+// quarter sp, head 2*hp+g, and the ten warps pool, rotate (keys) and store
+// the window's receiver rows [jb, je), split into slices as in the rotated
+// epilogue.
+template <typename T>
+__device__ __forceinline__ void pam_epilogue(const XferParams& P, uint32_t ta,
+                                             const float* bias_tile, float inv_r, int base,
+                                             int jb, int je, float* sStg, int e, int g, int row,
+                                             int lane, bool do_rope, T* out_lc, int ocol0) {
+  const int D = P.D_r, half = P.D_r / 2;
+  const int n_heads = P.BN / D;
+  const bool two_heads = n_heads >= 2;
+  const int n_pairs = two_heads ? n_heads / 2 : 1;
+  const bool stages_head = e < 8 && (g == 0 || two_heads);
+  const int ps = lane >> 2, qq = lane & 3;
+  const int per = (je - jb + kEpiWarps - 1) / kEpiWarps;
+  const int wjb = min(je, jb + e * per), wje = min(je, wjb + per);
+  const int per_slot = (wje - wjb + 7) >> 3;
+  const int ljb = min(wje, wjb + ps * per_slot), lje = min(wje, ljb + per_slot);
+  for (int hp = 0; hp < n_pairs; ++hp) {
+    const int tcol = (2 * hp + g) * D;
+    for (int q = 0; q < half; q += 16) {
+      float f[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) f[k] = do_rope ? __ldg(P.inv_freq + q + 4 * qq + k) : 0.f;
+      if (stages_head) {
+        uint32_t v[32];
+        tmem_load_2x16(ta + tcol + q, ta + tcol + half + q, v);
+        float* srow = sStg + row * 64 + g * 32;
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+          *reinterpret_cast<float4*>(srow + ((k ^ (row & 7)) << 2)) = make_float4(
+              __uint_as_float(v[4 * k]) * inv_r, __uint_as_float(v[4 * k + 1]) * inv_r,
+              __uint_as_float(v[4 * k + 2]) * inv_r, __uint_as_float(v[4 * k + 3]) * inv_r);
+      }
+      named_barrier_sync(1, kEpiThreads);
+      const float* bb = bias_tile + 2 * hp * D + q + 4 * qq;
+      float4 bias4[4];
+      bias4[0] = __ldg(reinterpret_cast<const float4*>(bb));
+      bias4[1] = __ldg(reinterpret_cast<const float4*>(bb + half));
+      bias4[2] = two_heads ? __ldg(reinterpret_cast<const float4*>(bb + D)) : make_float4(0.f, 0.f, 0.f, 0.f);
+      bias4[3] = two_heads ? __ldg(reinterpret_cast<const float4*>(bb + D + half)) : make_float4(0.f, 0.f, 0.f, 0.f);
+      float C1[4], S1[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        C1[k] = 1.f;
+        S1[k] = 0.f;
+        if (do_rope) rope_sincos(1, f[k], &S1[k], &C1[k]);  // one step = one row
+      }
+      pam_walk<T>(ljb, lje, base, sStg, qq, two_heads, do_rope, f, C1, S1, bias4, P, out_lc,
+                  ocol0 + 2 * hp * D, q, half);
+      named_barrier_sync(1, kEpiThreads);
+    }
+  }
+}
+
 // Last u in [0, nrows) with srun[u] <= j.
 __device__ __forceinline__ int find_row(const int32_t* srun, int nrows, int j) {
   int lo = 0, hi = nrows - 1;
@@ -388,11 +547,13 @@ __device__ __forceinline__ int find_row(const int32_t* srun, int nrows, int j) {
 // [kin*kBK, (kin+1)*kBK) of segment `seg`, i.e. sum over the segment's
 // sender layers (weight om) and the row's CSR entries (weight w) of the
 // sender rows, accumulated in fp32 and written into the swizzled layout,
-// rounded once, or as value + residual atoms when lo_atom is given.
+// rounded once, or as value + residual atoms when lo_atom is given.  With
+// tok >= 0 the row is that one aligned sender token, weight 1 (pooling
+// after the map), and the CSR range is not read.
 template <typename T>
 __device__ __forceinline__ void build_atom(const XferParams& P, const LayerSegs& segs, int seg,
-                                           int kin, int c, int e0, int e1, uint8_t* atom,
-                                           uint8_t* lo_atom, int t) {
+                                           int kin, int c, int e0, int e1, int tok,
+                                           uint8_t* atom, uint8_t* lo_atom, int t) {
   constexpr int kBK = Elem<T>::kBK;
   constexpr int kPerChunk = 16 / sizeof(T);
   const T* sender = reinterpret_cast<const T*>(P.sender);
@@ -403,10 +564,11 @@ __device__ __forceinline__ void build_atom(const XferParams& P, const LayerSegs&
     const int tl = segs.layer[seg][ti];
     const float om = segs.w[seg][ti];
     const T* base = sender + (static_cast<int64_t>(tl * 2 + c) * P.s_rows) * P.d_s + kin * kBK;
-    for (int e = e0; e < e1; ++e) {
-      const int k = P.col[e];
+    const int n_e = tok >= 0 ? 1 : e1 - e0;
+    for (int ie = 0; ie < n_e; ++ie) {
+      const int k = tok >= 0 ? tok : P.col[e0 + ie];
       if (k < 0 || k >= P.T_s) continue;  // flagged at plan creation
-      const float wt = om * P.w[e];
+      const float wt = tok >= 0 ? om : om * P.w[e0 + ie];
       const int64_t kr = P.srow ? __ldg(P.srow + k) : k;
       const uint4* src = reinterpret_cast<const uint4*>(base + kr * P.d_s);
       uint4 x[8];
@@ -537,7 +699,9 @@ __device__ __forceinline__ void build_stage_unrotated(const XferParams& P, const
 
 // Tiles of several transfer directions in one launch: direction d owns the
 // launch's tiles [base[d], base[d + 1]) (2 x its slots, so a slot's two
-// roles stay together), m_tiles[d] row blocks of U[d] distinct rows.
+// roles stay together), m_tiles[d] row blocks of U[d] distinct rows (with
+// pooling after the map, 128 rows per window: one window per CTA of a pair
+// tile).
 template <int kDirs>
 struct DirTable {
   int base[kDirs + 1];
@@ -545,11 +709,11 @@ struct DirTable {
   int U[kDirs];
 };
 
-template <int kDirs>
+template <int kDirs, int kPam>
 __device__ __forceinline__ int build_dirs(const XferParams* Ps, int n_dir, DirTable<kDirs>* dt) {
   int total = 0;
   for (int d = 0; d < (kDirs == 1 ? 1 : n_dir); ++d) {
-    const int U = *Ps[d].n_distinct;
+    const int U = pam_on<kPam>(Ps[d]) ? 128 * __ldg(Ps[d].win_info + 2) : *Ps[d].n_distinct;
     const int mt = (U + kPairRows - 1) / kPairRows;
     dt->U[d] = U;
     dt->m_tiles[d] = mt;
@@ -584,7 +748,7 @@ __device__ __forceinline__ void arrive_leader(uint32_t bar, int row0) {
 // layout.  A thread keeps LAG groups in flight: after committing k-block i
 // it waits for k-block i-LAG and fences it to the async proxy; then one lane
 // per warp arrives on that stage's barrier in the leader CTA of the pair.
-template <typename T, int LAG, int kDirs>
+template <typename T, int LAG, int kDirs, int kPam>
 __device__ __forceinline__ void gather_rows(const XferParams* Ps, const DirTable<kDirs>& dt,
                                             int n_dir, uint8_t* sA, uint64_t* full_a,
                                             uint64_t* empty_a, volatile int* sAbort, int t,
@@ -622,8 +786,14 @@ __device__ __forceinline__ void gather_rows(const XferParams* Ps, const DirTable
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
       const int r = slab * 32 + 4 * i + rsub;
-      const int u = min(m * kPairRows + row0 + r, U - 1);
-      roff[i] = static_cast<int64_t>(P.ucol[u]) * P.d_s + ch * kPerChunk;
+      int64_t kr;  // sender-cache row
+      if (pam_on<kPam>(P)) {
+        const int k = pam_token(P, m, row0, r);
+        kr = P.srow ? __ldg(P.srow + k) : k;
+      } else {
+        kr = P.ucol[min(m * kPairRows + row0 + r, U - 1)];
+      }
+      roff[i] = kr * P.d_s + ch * kPerChunk;
       doff[i] = static_cast<uint32_t>(r * 128 + ((ch ^ (r & 7)) << 4));
     }
     int seg = 0, kin = 0;  // segment of the next atom, and the atom within it
@@ -686,6 +856,7 @@ __device__ __forceinline__ void gather_rows(const XferParams* Ps, const DirTable
 // direct load.
 struct StagedRow {
   int e0, e1;  // the finished row's CSR entries
+  int tok;     // >= 0: the row is this aligned sender token, weight 1 (pooling after the map)
   int frow;    // its index among the CTA's 128 rows
 };
 
@@ -705,13 +876,15 @@ __device__ __forceinline__ void finish_staged_row(const XferParams& P, const Lay
   const float om1 = n_t > 1 ? __ldg(&lsegs->w[seg][1]) : 0.f;
   const int64_t lrows = P.s_rows * P.d_s;
   const int frow = r.frow, sw = frow & 7;
-  const int k0 = r.e1 > r.e0 ? P.col[r.e0] : -1;
+  const bool one = r.tok >= 0;
+  const int k0 = one ? r.tok : (r.e1 > r.e0 ? P.col[r.e0] : -1);
   const bool v0 = k0 >= 0 && k0 < P.T_s;
   int k1 = -1;
-  if (n_t == 1 && r.e1 > r.e0 + 1) k1 = P.col[r.e0 + 1];
+  if (!one && n_t == 1 && r.e1 > r.e0 + 1) k1 = P.col[r.e0 + 1];
   const bool v1 = n_t > 1 ? v0 : (k1 >= 0 && k1 < P.T_s);
-  const float w0 = v0 ? om0 * P.w[r.e0] : 0.f;
-  const float w1 = !v1 ? 0.f : (n_t > 1 ? om1 * P.w[r.e0] : om0 * P.w[r.e0 + 1]);
+  const float e_w0 = one ? 1.f : (v0 ? P.w[r.e0] : 0.f);
+  const float w0 = v0 ? om0 * e_w0 : 0.f;
+  const float w1 = !v1 ? 0.f : (n_t > 1 ? om1 * e_w0 : om0 * P.w[r.e0 + 1]);
   // two halves of four 16-byte chunks (fewer live registers)
 #pragma unroll 1
   for (int h = 0; h < 2; ++h) {
@@ -730,7 +903,8 @@ __device__ __forceinline__ void finish_staged_row(const XferParams& P, const Lay
     }
     // the remaining (term, entry) pairs, loaded directly
     const int e_first = n_t > 1 ? r.e0 + 1 : r.e0 + 2;
-    for (int e = e_first; e < r.e1; ++e) {
+    const int e_end = one ? e_first : r.e1;
+    for (int e = e_first; e < e_end; ++e) {
       const int k = P.col[e];
       if (k < 0 || k >= P.T_s) continue;  // flagged at plan creation
       const int64_t kr = P.srow ? __ldg(P.srow + k) : k;
@@ -753,7 +927,7 @@ __device__ __forceinline__ void finish_staged_row(const XferParams& P, const Lay
   }
 }
 
-template <typename T, int LAG, int kDirs>
+template <typename T, int LAG, int kDirs, int kPam>
 __device__ __forceinline__ void build_rows_staged(const XferParams* Ps, const DirTable<kDirs>& dt,
                                                   int n_dir, uint8_t* sA, uint64_t* full_a,
                                                   uint64_t* empty_a, volatile int* sAbort, int t,
@@ -782,11 +956,16 @@ __device__ __forceinline__ void build_rows_staged(const XferParams* Ps, const Di
     int32_t kr0[8], kr1[8];
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
-      const int u = min(m * kPairRows + row0 + slab * 32 + 4 * i + rsub, U - 1);
-      const int j0 = P.run_ptr[u];
-      const int e0 = P.row_ptr[j0], e1 = P.row_ptr[j0 + 1];
-      int k0 = e1 > e0 ? P.col[e0] : -1;
-      int k1 = e1 > e0 + 1 ? P.col[e0 + 1] : -1;
+      int k0, k1 = -1;
+      if (pam_on<kPam>(P)) {
+        k0 = pam_token(P, m, row0, slab * 32 + 4 * i + rsub);
+      } else {
+        const int u = min(m * kPairRows + row0 + slab * 32 + 4 * i + rsub, U - 1);
+        const int j0 = P.run_ptr[u];
+        const int e0 = P.row_ptr[j0], e1 = P.row_ptr[j0 + 1];
+        k0 = e1 > e0 ? P.col[e0] : -1;
+        k1 = e1 > e0 + 1 ? P.col[e0 + 1] : -1;
+      }
       if (k0 >= P.T_s) k0 = -1;  // flagged at plan creation
       if (k1 >= P.T_s) k1 = -1;
       kr0[i] = k0 < 0 ? -1 : (P.srow ? __ldg(P.srow + k0) : k0);
@@ -794,7 +973,11 @@ __device__ __forceinline__ void build_rows_staged(const XferParams* Ps, const Di
     }
     StagedRow fr;
     fr.frow = slab * 32 + lane;
-    {
+    fr.e0 = fr.e1 = 0;
+    fr.tok = -1;
+    if (pam_on<kPam>(P)) {
+      fr.tok = pam_token(P, m, row0, fr.frow);
+    } else {
       const int fu = min(m * kPairRows + row0 + fr.frow, U - 1);
       const int fj0 = P.run_ptr[fu];
       fr.e0 = P.row_ptr[fj0];
@@ -864,7 +1047,7 @@ __device__ __forceinline__ void build_rows_staged(const XferParams* Ps, const Di
 // every role looks its tile's direction up and reads that direction's
 // parameters).  All directions share the dtype, the operand path and the
 // ring depths; a B stage is stage_b_stride bytes (the widest direction's).
-template <typename T, bool kGather, int kDirs>
+template <typename T, bool kGather, int kDirs, int kPam>
 __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const XferParams* Ps,
                                               int n_dir, int stage_b_stride) {
   constexpr int kBK = Elem<T>::kBK;
@@ -931,7 +1114,7 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
   const uint32_t tmem_base = *sTmem;
 
   DirTable<kDirs> dt;
-  const int total_tiles = build_dirs<kDirs>(Ps, n_dir, &dt);
+  const int total_tiles = build_dirs<kDirs, kPam>(Ps, n_dir, &dt);
   const bool by_slot = total_tiles >= 4 * tile_step;
 
   if (warp == 0) {
@@ -1107,7 +1290,18 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
       tc_fence_after_sync();
       const int u0 = m * kPairRows + row0;
       const int nrows = min(kBM, U - u0);  // <= 0: this CTA has no rows in the tile
-      if (nrows > 0) {
+      if (nrows > 0 && pam_on<kPam>(P)) {
+        const int w = u0 >> 7;  // this CTA's window
+        const int base = w * __ldg(P.win_info + 1);
+        const int jb = __ldg(P.win_ptr + w), je = __ldg(P.win_ptr + w + 1);
+        T* const out_lc = reinterpret_cast<T*>(P.receiver) +
+                          (static_cast<int64_t>(lc) * P.recv_rows) * P.d_r;
+        pam_epilogue<T>(P,
+                        tmem_base + static_cast<uint32_t>(acc * 256) +
+                            (static_cast<uint32_t>(sp * 32) << 16),
+                        P.bias + static_cast<int64_t>(lc) * P.d_r + n * P.BN, P.inv_r[lc], base,
+                        jb, je, sStg, e, g, row, lane, P.rope && c == 0, out_lc, n * P.BN);
+      } else if (nrows > 0) {
         for (int i = tid_e; i <= nrows; i += kEpiThreads) {
           sRun[i] = P.run_ptr[u0 + i];
           sUpos[i] = i < nrows ? P.upos[u0 + i] : 0;
@@ -1216,17 +1410,17 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
     const int t = threadIdx.x - 64 - kEpiThreads;  // 0..127
     if (kGather) {
       switch (P0.lag) {
-        case 1: gather_rows<T, 1, kDirs>(Ps, dt, n_dir, sA, full_a, empty_a, sAbort, t, lane, row0, total_tiles, first_tile, tile_step); break;
-        case 2: gather_rows<T, 2, kDirs>(Ps, dt, n_dir, sA, full_a, empty_a, sAbort, t, lane, row0, total_tiles, first_tile, tile_step); break;
-        case 3: gather_rows<T, 3, kDirs>(Ps, dt, n_dir, sA, full_a, empty_a, sAbort, t, lane, row0, total_tiles, first_tile, tile_step); break;
-        case 4: gather_rows<T, 4, kDirs>(Ps, dt, n_dir, sA, full_a, empty_a, sAbort, t, lane, row0, total_tiles, first_tile, tile_step); break;
-        default: gather_rows<T, 5, kDirs>(Ps, dt, n_dir, sA, full_a, empty_a, sAbort, t, lane, row0, total_tiles, first_tile, tile_step); break;
+        case 1: gather_rows<T, 1, kDirs, kPam>(Ps, dt, n_dir, sA, full_a, empty_a, sAbort, t, lane, row0, total_tiles, first_tile, tile_step); break;
+        case 2: gather_rows<T, 2, kDirs, kPam>(Ps, dt, n_dir, sA, full_a, empty_a, sAbort, t, lane, row0, total_tiles, first_tile, tile_step); break;
+        case 3: gather_rows<T, 3, kDirs, kPam>(Ps, dt, n_dir, sA, full_a, empty_a, sAbort, t, lane, row0, total_tiles, first_tile, tile_step); break;
+        case 4: gather_rows<T, 4, kDirs, kPam>(Ps, dt, n_dir, sA, full_a, empty_a, sAbort, t, lane, row0, total_tiles, first_tile, tile_step); break;
+        default: gather_rows<T, 5, kDirs, kPam>(Ps, dt, n_dir, sA, full_a, empty_a, sAbort, t, lane, row0, total_tiles, first_tile, tile_step); break;
       }
     } else if (P0.staged) {
       switch (P0.lag) {
-        case 1: build_rows_staged<T, 1, kDirs>(Ps, dt, n_dir, sA, full_a, empty_a, sAbort, t, lane, row0, total_tiles, first_tile, tile_step); break;
-        case 2: build_rows_staged<T, 2, kDirs>(Ps, dt, n_dir, sA, full_a, empty_a, sAbort, t, lane, row0, total_tiles, first_tile, tile_step); break;
-        default: build_rows_staged<T, 3, kDirs>(Ps, dt, n_dir, sA, full_a, empty_a, sAbort, t, lane, row0, total_tiles, first_tile, tile_step); break;
+        case 1: build_rows_staged<T, 1, kDirs, kPam>(Ps, dt, n_dir, sA, full_a, empty_a, sAbort, t, lane, row0, total_tiles, first_tile, tile_step); break;
+        case 2: build_rows_staged<T, 2, kDirs, kPam>(Ps, dt, n_dir, sA, full_a, empty_a, sAbort, t, lane, row0, total_tiles, first_tile, tile_step); break;
+        default: build_rows_staged<T, 3, kDirs, kPam>(Ps, dt, n_dir, sA, full_a, empty_a, sAbort, t, lane, row0, total_tiles, first_tile, tile_step); break;
       }
     } else {
       // pooled CSR rows, blended sender layers and/or rotated sender keys:
@@ -1243,9 +1437,15 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
                     &n);
         const int l = lc >> 1, c = lc & 1;
         const LayerSegs segs = P.segs[l];
-        const int u = min(m * kPairRows + row0 + t, dt.U[dd] - 1);
-        const int j0 = P.run_ptr[u];
-        const int e0 = P.row_ptr[j0], e1 = P.row_ptr[j0 + 1];
+        int e0 = 0, e1 = 0, tok = -1;
+        if (pam_on<kPam>(P)) {  // sender token of this row of the CTA's window
+          tok = pam_token(P, m, row0, t);
+        } else {
+          const int u = min(m * kPairRows + row0 + t, dt.U[dd] - 1);
+          const int j0 = P.run_ptr[u];
+          e0 = P.row_ptr[j0];
+          e1 = P.row_ptr[j0 + 1];
+        }
         const bool unrot_k = P.unrot && c == 0;
         int seg = 0, kin = 0;  // segment of the next atom, and the atom within it
         for (int kb = 0; kb < P.n_kb; ++kb) {
@@ -1260,7 +1460,7 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
             if (unrot_k)
               build_atom_unrotated<T>(P, segs, seg, kin, c, e0, e1, st, st + kAtomABytes, t);
             else
-              build_atom<T>(P, segs, seg, kin, c, e0, e1, st, st + kAtomABytes, t);
+              build_atom<T>(P, segs, seg, kin, c, e0, e1, tok, st, st + kAtomABytes, t);
             if (++kin == P.atoms_per_seg) {
               kin = 0;
               ++seg;
@@ -1276,7 +1476,7 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
           } else {
             const int na = kb == P.n_kb - 1 ? P.last_atoms : kAtoms;
             for (int a = 0; a < na; ++a) {
-              build_atom<T>(P, segs, seg, kin, c, e0, e1, st + a * kAtomABytes, nullptr, t);
+              build_atom<T>(P, segs, seg, kin, c, e0, e1, tok, st + a * kAtomABytes, nullptr, t);
               if (++kin == P.atoms_per_seg) {
                 kin = 0;
                 ++seg;
@@ -1309,11 +1509,11 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
   }
 }
 
-template <typename T, bool kGather>
+template <typename T, bool kGather, int kPam>
 __global__ void __launch_bounds__(kThreads, 1)
     transfer_kernel(const __grid_constant__ CUtensorMap tmap_w,
                     const __grid_constant__ XferParams P) {
-  transfer_body<T, kGather, 1>(&tmap_w, &P, 1, (P.BN / 2) * 128);
+  transfer_body<T, kGather, 1, kPam>(&tmap_w, &P, 1, (P.BN / 2) * 128);
 }
 
 // Several directions in one launch (hf_transfer_batch).
@@ -1325,10 +1525,10 @@ struct BatchParams {
 };
 static_assert(sizeof(BatchParams) < 32000, "BatchParams must fit the kernel parameter space");
 
-template <typename T, bool kGather>
+template <typename T, bool kGather, int kPam>
 __global__ void __launch_bounds__(kThreads, 1)
     transfer_batch_kernel(const __grid_constant__ BatchParams B) {
-  transfer_body<T, kGather, kMaxBatch>(B.maps, B.P, B.n_dir, B.stage_b_stride);
+  transfer_body<T, kGather, kMaxBatch, kPam>(B.maps, B.P, B.n_dir, B.stage_b_stride);
 }
 
 // ---------------------------------------------------------------------------
@@ -1482,6 +1682,10 @@ hf_status make_xfer(hf_plan_s* p, const void* sender, void* receiver, int l_begi
   const int n_atoms = p->K / bk;  // 128-byte k-blocks per output row
   P.split = p->split ? 1 : 0;
   P.staged = p->staged ? 1 : 0;
+  P.pam = p->pam ? 1 : 0;
+  P.win_info = reinterpret_cast<const int32_t*>(ws + p->lay.win_info);
+  P.win_ptr = reinterpret_cast<const int32_t*>(ws + p->lay.win_ptr);
+  P.pos = reinterpret_cast<const int32_t*>(ws + p->lay.pos);
   P.atoms_per_stage = p->split ? 1 : kAtoms;
   P.n_batoms = n_atoms;
   P.n_kb = (n_atoms + P.atoms_per_stage - 1) / P.atoms_per_stage;
@@ -1499,15 +1703,16 @@ hf_status make_xfer(hf_plan_s* p, const void* sender, void* receiver, int l_begi
   P.knorm = d.d_knorm_w ? 1 : 0;
   P.knorm_eps = d.knorm_eps;
   P.idesc = make_idesc(f32 ? 2u : 1u, kPairRows, p->BN);
-  *max_pair_tiles =
-      2LL * P.n_l * ((p->T_r + kPairRows - 1) / kPairRows) * static_cast<int64_t>(P.n_tiles_n);
+  // pooling after the map: at most T_s windows (stride >= 1), two per pair tile
+  const int64_t row_blocks = p->pam ? (p->T_s + 1) / 2 : (p->T_r + kPairRows - 1) / kPairRows;
+  *max_pair_tiles = 2LL * P.n_l * row_blocks * static_cast<int64_t>(P.n_tiles_n);
   return HF_OK;
 }
 
-template <typename T, bool kGather>
+template <typename T, bool kGather, int kPam>
 hf_status launch_batch_typed(const BatchParams& B, int64_t max_pair_tiles, size_t smem,
                              cudaStream_t stream) {
-  return launch_pairs(transfer_batch_kernel<T, kGather>, max_pair_tiles, smem, stream, B);
+  return launch_pairs(transfer_batch_kernel<T, kGather, kPam>, max_pair_tiles, smem, stream, B);
 }
 
 }  // namespace
@@ -1525,17 +1730,23 @@ hf_status launch_transfer(hf_plan_s* p, const void* sender, void* receiver, cuda
   P.stall = stall ? 1 : 0;
   const size_t smem = smem_bytes(p->BN, P.stages_a, P.stages_b);
   if (d.dtype == HF_F32)
-    return p->gather ? launch_pairs(transfer_kernel<float, true>, max_pair_tiles, smem, stream, mw, P)
-                     : launch_pairs(transfer_kernel<float, false>, max_pair_tiles, smem, stream, mw, P);
+    return p->gather
+               ? launch_pairs(transfer_kernel<float, true, 2>, max_pair_tiles, smem, stream, mw, P)
+               : launch_pairs(transfer_kernel<float, false, 2>, max_pair_tiles, smem, stream, mw, P);
+  if (p->pam)
+    return p->gather
+               ? launch_pairs(transfer_kernel<__nv_bfloat16, true, 1>, max_pair_tiles, smem, stream, mw, P)
+               : launch_pairs(transfer_kernel<__nv_bfloat16, false, 1>, max_pair_tiles, smem, stream, mw, P);
   return p->gather
-             ? launch_pairs(transfer_kernel<__nv_bfloat16, true>, max_pair_tiles, smem, stream, mw, P)
-             : launch_pairs(transfer_kernel<__nv_bfloat16, false>, max_pair_tiles, smem, stream, mw, P);
+             ? launch_pairs(transfer_kernel<__nv_bfloat16, true, 0>, max_pair_tiles, smem, stream, mw, P)
+             : launch_pairs(transfer_kernel<__nv_bfloat16, false, 0>, max_pair_tiles, smem, stream, mw, P);
 }
 
 bool batch_compatible(const hf_plan_s* const* plans, int n) {
   for (int i = 1; i < n; ++i)
     if (plans[i]->desc.dtype != plans[0]->desc.dtype || plans[i]->gather != plans[0]->gather ||
-        plans[i]->split != plans[0]->split || plans[i]->staged != plans[0]->staged)
+        plans[i]->split != plans[0]->split || plans[i]->staged != plans[0]->staged ||
+        plans[i]->pam != plans[0]->pam)
       return false;
   return true;
 }
@@ -1576,11 +1787,14 @@ hf_status launch_transfer_batch(hf_plan_s* const* plans, const void* const* send
   const size_t smem = smem_bytes(max_bn, sa, sb);
   hf_status s;
   if (plans[0]->desc.dtype == HF_F32)
-    s = plans[0]->gather ? launch_batch_typed<float, true>(*B, tiles, smem, stream)
-                         : launch_batch_typed<float, false>(*B, tiles, smem, stream);
+    s = plans[0]->gather ? launch_batch_typed<float, true, 2>(*B, tiles, smem, stream)
+                         : launch_batch_typed<float, false, 2>(*B, tiles, smem, stream);
+  else if (plans[0]->pam)
+    s = plans[0]->gather ? launch_batch_typed<__nv_bfloat16, true, 1>(*B, tiles, smem, stream)
+                         : launch_batch_typed<__nv_bfloat16, false, 1>(*B, tiles, smem, stream);
   else
-    s = plans[0]->gather ? launch_batch_typed<__nv_bfloat16, true>(*B, tiles, smem, stream)
-                         : launch_batch_typed<__nv_bfloat16, false>(*B, tiles, smem, stream);
+    s = plans[0]->gather ? launch_batch_typed<__nv_bfloat16, true, 0>(*B, tiles, smem, stream)
+                         : launch_batch_typed<__nv_bfloat16, false, 0>(*B, tiles, smem, stream);
   delete B;
   return s;
 }

@@ -46,13 +46,16 @@ def test_llama_to_ministral_32k_sampled():
     print(c.report())
 
 
-# The register-built operand path (pooled rows, blended layers): the fp32
-# pooling or blend is rounded once to bf16 before the tensor core, so its
-# error grows with the number of outputs compared; these run it on the real
-# model shapes (whole 4K transfers, and the 32K transfer sampled as above).
+# Overlap mean pooling on the real model shapes (whole 4K transfers, and the
+# 32K transfer sampled as above).  By default the pooling follows the map
+# (sender rows mapped, the mapped rows pooled in the epilogue; blended
+# layers as value + residual operand rows); pool_before_map builds the
+# pooled rows first (value + residual operand rows per distinct row).
 @pytest.mark.parametrize("layer_mode", ["paper3", "interp"])
-def test_llama_to_qwen25_4k_overlap_full(layer_mode):
-    c = Case(W.llama_to_qwen25(4096).with_(align_mode="overlap_mean", layer_mode=layer_mode)).run()
+@pytest.mark.parametrize("pool_before_map", [False, True])
+def test_llama_to_qwen25_4k_overlap_full(layer_mode, pool_before_map):
+    c = Case(W.llama_to_qwen25(4096).with_(align_mode="overlap_mean", layer_mode=layer_mode),
+             pool_before_map=pool_before_map).run()
     c.check_csr()
     c.check_parity()
     print(c.report())
@@ -349,6 +352,114 @@ def test_device_flags_bad_block_and_column():
     c2.job.transfer()
     torch.cuda.synchronize()
     assert c2.job.device_status() & 0x02
+
+
+# ---------------------------------------------------------------- pooling after the map
+# Overlap mean pooling commutes with the map: plans in that mode map
+# windows of 128 aligned sender tokens (stride 128 - h, h the widest row's
+# column span) and pool the mapped rows in the epilogue.
+PAM_EDGE = {
+    # ten receiver rows per sender token: ~1,300 receiver rows per window
+    "long_runs": lambda: W.llama_to_ministral(3000).with_(
+        L_s=4, L_r=3, mean_s=12.0, mean_r=1.2, r_pos0=(3000,), align_mode="overlap_mean"),
+    # one-character sender tokens, 13-character receiver tokens: every row
+    # spans 13 sender tokens (window stride 116)
+    "wide_rows": lambda: W.llama_to_ministral(600).with_(
+        L_s=4, L_r=3, mean_s=1.0, mean_r=13.0, align_mode="overlap_mean"),
+    "batched_paged_spans": lambda: W.qwen25_to_llama_batched(
+        n_req=3, lo=40, hi=400, seed=51).with_(L_s=4, L_r=3, align_mode="overlap_mean",
+                                               span_gap=300),
+    # blended layers (staged value + residual rows), paged, with an empty
+    # and a one-token request
+    "interp_batched_paged": lambda: W.qwen25_to_llama_batched(
+        n_req=4, lo=1, hi=300, seed=52).with_(L_s=5, L_r=4, align_mode="overlap_mean",
+                                              layer_mode="interp", r_tokens=(250, 0, 1, 300)),
+    "paper3_f32": lambda: W.llama_to_ministral(500).with_(L_s=4, L_r=3, dtype="f32",
+                                                          align_mode="overlap_mean"),
+    "head64": lambda: W.llama_to_ministral(333).with_(L_s=3, L_r=2, H_r=4, D_r=64,
+                                                      align_mode="overlap_mean"),
+    "one_head_d128": lambda: W.llama_to_ministral(333).with_(L_s=3, L_r=2, H_r=1, D_r=128,
+                                                             align_mode="overlap_mean"),
+    "explicit_two_terms": lambda: _explicit(
+        W.llama_to_ministral(500).with_(L_s=5, L_r=3, align_mode="overlap_mean"),
+        n_seg=2, n_terms=2),
+    "one_token": lambda: W.llama_to_ministral(1).with_(L_s=3, L_r=3, align_mode="overlap_mean"),
+    "rope_table_pos0": lambda: W.llama_to_ministral(700).with_(
+        L_s=4, L_r=3, align_mode="overlap_mean", rope_table=True, r_pos0=(90000,)),
+}
+
+
+@pytest.mark.parametrize("name", sorted(PAM_EDGE))
+def test_pool_after_map_edge_case(name):
+    c = Case(PAM_EDGE[name]()).run()
+    c.check_csr()
+    c.check_parity()
+
+
+def test_pool_after_map_rounded_blend():
+    """Blended rows rounded once (the builder path with one sender token per
+    operand row)."""
+    c = Case(PAM_EDGE["interp_batched_paged"](), round_built_operands=True).run()
+    c.check_parity()
+
+
+def _crafted_csr(c, rows):
+    """Replaces the job's alignment CSR by rows (lists of sender columns,
+    mean weights) and keeps the oracle's copy in step."""
+    T = c.tok.T_r
+    assert len(rows) == T
+    rp = np.zeros(T + 1, np.int64)
+    rp[1:] = np.cumsum([len(r) for r in rows])
+    col = np.concatenate([np.asarray(r, np.int64) for r in rows])
+    w = np.concatenate([np.full(len(r), 1.0 / len(r)) for r in rows])
+    assert rp[-1] <= c.job.nnz_capacity
+    c.job.align()
+    c.job.row_ptr.copy_(torch.as_tensor(rp.astype(np.int32)))
+    c.job.col[: len(col)].copy_(torch.as_tensor(col.astype(np.int32)))
+    c.job.w[: len(w)].copy_(torch.as_tensor(w.astype(np.float32)))
+    c.csr = O.CSR(rp, col, w)
+    c.job.make_plan()
+    c.job.transfer()
+    torch.cuda.synchronize()
+
+
+@pytest.mark.parametrize("kind", ["span_150", "decreasing"])
+def test_pool_after_map_flags_rows_outside_their_window(kind):
+    """A row spanning 150 sender tokens, or rows whose first columns
+    decrease: pooling after the map flags HF_CHECK_POOL_WINDOW (the
+    transfer stays in bounds); pooling before the map takes the same CSR
+    and matches the oracle."""
+    w = W.llama_to_ministral(100).with_(L_s=3, L_r=2, mean_s=1.0, mean_r=3.6,
+                                        align_mode="overlap_mean")
+    for before in (False, True):
+        c = Case(w, pool_before_map=before)
+        T, Ts = c.tok.T_r, c.tok.T_s
+        assert Ts >= 3 * T
+        rows = [[3 * j] for j in range(T)]
+        if kind == "span_150":
+            rows[3] = list(range(9, 159))
+        else:  # row 60's window starts at sender token 128 (stride 127 or 128)
+            rows[60] = [5, 6]
+        _crafted_csr(c, rows)
+        status = c.job.device_status()
+        if before:
+            assert status == 0, hex(status)
+            c.check_parity()
+        else:
+            assert status & 0x80, hex(status)
+
+
+def test_pool_after_map_wide_row_fits():
+    """One row spanning 100 sender tokens: the window stride drops to 29
+    and the transfer stays exact."""
+    w = W.llama_to_ministral(100).with_(L_s=3, L_r=2, mean_s=1.0, mean_r=3.6,
+                                        align_mode="overlap_mean")
+    c = Case(w)
+    rows = [[j] for j in range(c.tok.T_r)]
+    rows[5] = list(range(5, 105))
+    _crafted_csr(c, rows)
+    assert c.job.device_status() == 0
+    c.check_parity()
 
 
 def test_empty_final_row_is_flagged_not_read():

@@ -46,9 +46,25 @@ def test_copied_operand_label():
     assert bench._copied_operands(bench.workload("llama_to_ministral_32k"))
     assert bench._copied_operands(bench.workload("qwen25_to_llama_kv_ridge_4k"))
     assert not bench._copied_operands(bench.workload("llama_to_ministral_32k_interp"))
-    assert not bench._copied_operands(bench.workload("llama_to_qwen25_4k_overlap"))
+    # overlap pooling after the map copies sender rows; before it, pooled rows are computed
+    assert bench._copied_operands(bench.workload("llama_to_qwen25_4k_overlap"))
+    assert not bench._copied_operands(bench.workload("llama_to_qwen25_4k_overlap"),
+                                      pool_before_map=True)
+    assert not bench._copied_operands(bench.workload("llama_to_qwen25_4k_overlap_interp"))
     w = W.llama_to_ministral(64).with_(sender_k_rotated=True)
     assert not bench._copied_operands(w)
+    assert not bench._copied_operands(w.with_(align_mode="overlap_mean"))
+
+
+def test_launches_per_step():
+    """Align + plan + transfer kernels, by mode (the bench's gpu_launches)."""
+    assert bench.launches_per_step(bench.workload("llama_to_ministral_32k")) == 3 + 5 + 1
+    ov = bench.workload("llama_to_qwen25_4k_overlap")
+    assert bench.launches_per_step(ov) == 4 + 7 + 1
+    assert bench.launches_per_step(ov, pool_before_map=True) == 4 + 5 + 1
+    assert bench.launches_per_step(ov.with_(knorm=True)) == 4 + 5 + 1
+    assert bench.launches_per_step(W.llama_to_ministral(64).with_(
+        align_mode="same_index", span_gap=10)) == 1 + 6 + 1
 
 
 def test_kv_ridge_selection_stand_in():
