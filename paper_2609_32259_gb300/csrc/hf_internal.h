@@ -99,6 +99,7 @@ struct hf_plan_s {
   bool unrot;   // sender keys carry RoPE and are rotated back in the builder
   bool span;    // aligned sender tokens are spans inside a longer sender cache
   bool pam;     // pooling after the map: map input rows are sender rows in windows
+  bool wide;    // tiles of two 256-column blocks (operand rows built by the loader warps)
   int64_t s_rows;  // sender-cache rows per (layer, role)
   char* ws;
   size_t ws_bytes;

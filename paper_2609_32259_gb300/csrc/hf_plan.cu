@@ -582,6 +582,9 @@ hf_status plan_build(const hf_plan_desc* desc, void* d_workspace, size_t workspa
   // staged by cp.async; pooled rows have more, whose direct loads stall the
   // warp anyway (measured slower staged)
   p->staged = p->split && !p->unrot && one_entry;
+  // built operand rows bound their paths: a tile covering two 256-column
+  // blocks (both TMEM accumulators) builds each A stage once for both
+  p->wide = !p->gather && p->d_r % 512 == 0;
   p->ws = static_cast<char*>(d_workspace);
   p->ws_bytes = workspace_bytes;
   p->lay = lay;

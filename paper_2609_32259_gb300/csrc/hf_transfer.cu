@@ -87,6 +87,11 @@ struct XferParams {
   // (atoms_per_stage = 1); otherwise kAtoms atoms of K per A stage
   int split, atoms_per_stage, n_batoms;  // n_batoms: B atoms (map atoms of K) per tile
   int staged;  // split one-entry rows built by build_rows_staged
+  // wide tiles (operand rows built by the loader warps, which bound those
+  // paths): a tile covers two 256-column blocks, one per TMEM accumulator,
+  // so every built A stage feeds twice the MMAs; the epilogue drains both
+  // before the next tile's MMAs start
+  int wide;
   // pooling after the map: the tile rows of CTA rank k in pair tile m are the
   // aligned sender tokens of window w = 2m + k, [w S, w S + 128) (S =
   // win_info[1]); the receiver rows [win_ptr[w], win_ptr[w+1]) are pooled
@@ -1137,19 +1142,23 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
         int lc, m, n;
         decode_tile(tile - dt.base[dd], dt.m_tiles[dd] * P.n_tiles_n, P.n_tiles_n, P.l0, &lc, &m,
                     &n);
-        const int n_atoms = P.n_batoms;
-        for (int at = 0; at < n_atoms; ++at) {
+        // a wide tile takes each map atom for its two column blocks in turn
+        const int n_half = P.wide ? 2 : 1;
+        const int n_loads = P.n_batoms * n_half;
+        for (int ab = 0; ab < n_loads; ++ab) {
+          const int at = ab / n_half, h = ab - at * n_half;
           if (!mbar_wait(smem_addr(&empty_b[stage]), phase ^ 1)) {
             raise_timeout(P, sAbort);
             ok = false;
             break;
           }
           const uint32_t fb = mapa_shared(smem_addr(&full_b[stage]), 0);
-          if (!(P.stall && seq == 0 && at == 0)) {  // the test hook leaves this stage empty
+          if (!(P.stall && seq == 0 && ab == 0)) {  // the test hook leaves this stage empty
             mbar_arrive_expect_tx_cluster(fb, atom_b_bytes);
             tma_load_2d_pair_hint(smem_addr(sB + stage * stage_b_bytes), tmap, at * kBK,
-                                  lc * P.d_r + n * P.BN + static_cast<int>(rank) * half_bn, fb,
-                                  pol_b);
+                                  lc * P.d_r + (n * n_half + h) * P.BN +
+                                      static_cast<int>(rank) * half_bn,
+                                  fb, pol_b);
           }
           if (++stage == stages_b) {
             stage = 0;
@@ -1184,12 +1193,15 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
         const uint32_t idesc = P.idesc;
         const int n_kb = P.n_kb, last_atoms = P.last_atoms, per_stage = P.atoms_per_stage;
         const bool split = P.split != 0;
-        if (!mbar_wait(smem_addr(&tempty[acc]), acc_phase ^ 1)) {
+        const bool wide = !kGather && P.wide != 0;  // both accumulators, one per column block
+        const int n_half = wide ? 2 : 1;
+        bool free_acc = mbar_wait(smem_addr(&tempty[wide ? 0 : acc]), acc_phase ^ 1);
+        if (free_acc && wide) free_acc = mbar_wait(smem_addr(&tempty[1]), acc_phase ^ 1);
+        if (!free_acc) {
           raise_timeout(P, sAbort);
           break;
         }
         tc_fence_after_sync();
-        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * 256);
         uint32_t accumulate = 0;
         for (int kb = 0; kb < n_kb && ok; ++kb) {
           if (!mbar_wait(full_a0 + 8 * sa, pa)) {
@@ -1201,12 +1213,14 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
 #pragma unroll
           for (int a = 0; a < kAtoms; ++a) {
             if (a >= na) break;
+           for (int h = 0; h < n_half; ++h) {
             if (!mbar_wait(full_b0 + 8 * sb, pb)) {
               raise_timeout(P, sAbort);
               ok = false;
               break;
             }
             tc_fence_after_sync();
+            const uint32_t d_tmem = tmem_base + static_cast<uint32_t>((wide ? h : acc) * 256);
             const uint64_t ad = desc_a0 + sa * step_a + a * atom_a;
             const uint64_t bd = desc_b0 + sb * step_b;
             // four 32-byte K steps per 128-byte atom (descriptor units of 16 bytes)
@@ -1228,12 +1242,14 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
               mma_tf32_pair(d_tmem, ad + 4, bd + 4, idesc, 1);
               mma_tf32_pair(d_tmem, ad + 6, bd + 6, idesc, 1);
             }
-            accumulate = 1;
             tc_commit_pair(empty_b0 + 8 * sb, 0x3);
             if (++sb == stages_b) {
               sb = 0;
               pb ^= 1;
             }
+           }
+            if (!ok) break;
+            accumulate = 1;
           }
           if (!ok) break;
           tc_commit_pair(empty_a0 + 8 * sa, 0x3);
@@ -1243,9 +1259,15 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
           }
         }
         if (!ok) break;
-        tc_commit_pair(smem_addr(&tfull[acc]), 0x3);
-        acc ^= 1;
-        if (acc == 0) acc_phase ^= 1;
+        if (wide) {
+          tc_commit_pair(smem_addr(&tfull[0]), 0x3);
+          tc_commit_pair(smem_addr(&tfull[1]), 0x3);
+          acc_phase ^= 1;
+        } else {
+          tc_commit_pair(smem_addr(&tfull[acc]), 0x3);
+          acc ^= 1;
+          if (acc == 0) acc_phase ^= 1;
+        }
       }
       // every issued MMA has completed before TMEM is released
       tc_commit_pair(smem_addr(drain), 0x3);
@@ -1283,8 +1305,16 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
       decode_tile(tile - dt.base[dd], dt.m_tiles[dd] * P.n_tiles_n, P.n_tiles_n, P.l0, &lc, &m,
                   &n);
       const int c = lc & 1;
-      if (!mbar_wait(smem_addr(&tfull[acc]), acc_phase)) {
+      // a wide tile's two column blocks are drained in turn, one per accumulator
+      const bool wide = !kGather && P.wide != 0;
+      const int n_half = wide ? 2 : 1;
+      bool timed_out = false;
+      for (int h = 0; h < n_half; ++h) {
+      const int ac = wide ? h : acc;        // TMEM accumulator
+      const int nb = wide ? 2 * n + h : n;  // 256-column block of the map and the receiver
+      if (!mbar_wait(smem_addr(&tfull[ac]), acc_phase)) {
         raise_timeout(P, sAbort);
+        timed_out = true;
         break;
       }
       tc_fence_after_sync();
@@ -1297,10 +1327,10 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
         T* const out_lc = reinterpret_cast<T*>(P.receiver) +
                           (static_cast<int64_t>(lc) * P.recv_rows) * P.d_r;
         pam_epilogue<T>(P,
-                        tmem_base + static_cast<uint32_t>(acc * 256) +
+                        tmem_base + static_cast<uint32_t>(ac * 256) +
                             (static_cast<uint32_t>(sp * 32) << 16),
-                        P.bias + static_cast<int64_t>(lc) * P.d_r + n * P.BN, P.inv_r[lc], base,
-                        jb, je, sStg, e, g, row, lane, P.rope && c == 0, out_lc, n * P.BN);
+                        P.bias + static_cast<int64_t>(lc) * P.d_r + nb * P.BN, P.inv_r[lc], base,
+                        jb, je, sStg, e, g, row, lane, P.rope && c == 0, out_lc, nb * P.BN);
       } else if (nrows > 0) {
         for (int i = tid_e; i <= nrows; i += kEpiThreads) {
           sRun[i] = P.run_ptr[u0 + i];
@@ -1319,18 +1349,18 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
         const float* bias = P.bias + static_cast<int64_t>(lc) * P.d_r;
         const bool do_rope = P.rope && c == 0;
         const bool do_knorm = P.knorm && c == 0;
-        const uint32_t ta = tmem_base + static_cast<uint32_t>(acc * 256) +
+        const uint32_t ta = tmem_base + static_cast<uint32_t>(ac * 256) +
                             (static_cast<uint32_t>(sp * 32) << 16);
         T* const out_lc = reinterpret_cast<T*>(P.receiver) +
                           (static_cast<int64_t>(lc) * P.recv_rows) * P.d_r;
         if (c == 1 || (!P.rope && !P.knorm)) {
-          copy_epilogue<T>(P, ta, bias + n * P.BN, inv_r, nrows, sRun,
-                           reinterpret_cast<uint8_t*>(sStg), g, row, e, lane, out_lc, n * P.BN);
+          copy_epilogue<T>(P, ta, bias + nb * P.BN, inv_r, nrows, sRun,
+                           reinterpret_cast<uint8_t*>(sStg), g, row, e, lane, out_lc, nb * P.BN);
         } else
         for (int hp = 0; hp < n_pairs; ++hp) {
           const bool stages_head = stager && (g == 0 || two_heads);
           const int tcol = (2 * hp + g) * D;            // accumulator column of this warp's head
-          const int ocol_pair = n * P.BN + 2 * hp * D;  // receiver feature of the pair's first head
+          const int ocol_pair = nb * P.BN + 2 * hp * D;  // receiver feature of the pair's first head
           float rn = 1.0f;
           if (do_knorm && stages_head) {
             float ss = 0.0f;
@@ -1340,7 +1370,7 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
 #pragma unroll
               for (int i = 0; i < 16; ++i) {
                 const float y = fmaf(__uint_as_float(v[i]), inv_r,
-                                     __ldg(bias + n * P.BN + tcol + q2 + i));
+                                     __ldg(bias + nb * P.BN + tcol + q2 + i));
                 ss = fmaf(y, y, ss);
               }
             }
@@ -1356,7 +1386,7 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
               // step 1: pairs q..q+15 of head 2*hp+g for this warp's 32 rows
               uint32_t v[32];
               tmem_load_2x16(ta + tcol + q, ta + tcol + half + q, v);
-              const float* bcol = bias + n * P.BN + tcol;
+              const float* bcol = bias + nb * P.BN + tcol;
               float y[32];
 #pragma unroll
               for (int i = 0; i < 16; i += 4) {
@@ -1401,9 +1431,15 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
       }
       tc_fence_before_sync();
       __syncwarp();
-      if (lane == 0) arrive_leader(smem_addr(&tempty[acc]), row0);
-      acc ^= 1;
-      if (acc == 0) acc_phase ^= 1;
+      if (lane == 0) arrive_leader(smem_addr(&tempty[ac]), row0);
+      }
+      if (timed_out) break;
+      if (wide) {
+        acc_phase ^= 1;
+      } else {
+        acc ^= 1;
+        if (acc == 0) acc_phase ^= 1;
+      }
     }
   } else {
     // ------------------------------------------------------------ A builders
@@ -1692,7 +1728,8 @@ hf_status make_xfer(hf_plan_s* p, const void* sender, void* receiver, int l_begi
   P.last_atoms = n_atoms - P.atoms_per_stage * (P.n_kb - 1);
   P.atoms_per_seg = p->d_s / bk;
   P.BN = p->BN;
-  P.n_tiles_n = p->d_r / p->BN;
+  P.wide = p->wide ? 1 : 0;
+  P.n_tiles_n = p->d_r / (p->BN * (p->wide ? 2 : 1));
   pick_rings(p->BN, &P.stages_a, &P.stages_b, &P.lag);
   P.rope = p->rope ? 1 : 0;
   P.unrot = p->unrot ? 1 : 0;
@@ -1746,7 +1783,7 @@ bool batch_compatible(const hf_plan_s* const* plans, int n) {
   for (int i = 1; i < n; ++i)
     if (plans[i]->desc.dtype != plans[0]->desc.dtype || plans[i]->gather != plans[0]->gather ||
         plans[i]->split != plans[0]->split || plans[i]->staged != plans[0]->staged ||
-        plans[i]->pam != plans[0]->pam)
+        plans[i]->pam != plans[0]->pam || plans[i]->wide != plans[0]->wide)
       return false;
   return true;
 }
