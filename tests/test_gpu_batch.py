@@ -54,6 +54,29 @@ def test_batch_mixing_operand_paths():
         assert torch.equal(c.job.receiver, ref), c.w.name
 
 
+def test_batch_of_built_operand_rows():
+    """Directions whose operand rows the loader warps build (layers blended
+    per sender token, overlap pooling after the map; a Qwen2.5-shaped
+    receiver is one 512-column wide tile) in one launch: each equals its
+    single transfer and the oracle."""
+    ws = [W.llama_to_ministral(700).with_(L_s=5, L_r=4, layer_mode="interp",
+                                          align_mode="overlap_mean"),
+          W.llama_to_qwen25(500).with_(L_s=6, L_r=3, layer_mode="interp",
+                                       align_mode="overlap_mean"),
+          W.qwen25_to_llama_batched(n_req=2, lo=80, hi=300, seed=61).with_(
+              L_s=4, L_r=3, layer_mode="interp", align_mode="overlap_mean")]
+    cases = [Case(w, sentinel=SENTINEL).run() for w in ws]
+    single = [c.job.receiver.clone() for c in cases]
+    for c in cases:
+        c.job.receiver.fill_(SENTINEL)
+    B.transfer_batch([c.job.plan for c in cases], [c.sender for c in cases],
+                     [c.job.receiver for c in cases])
+    torch.cuda.synchronize()
+    for c, ref in zip(cases, single):
+        assert torch.equal(c.job.receiver, ref), c.w.name
+        c.check_parity()
+
+
 def test_batch_mixing_layer_tables():
     """A KV Ridge direction (an explicit eight-segment table), a paper3
     direction and an interpolated one in one batch: each equals its single
