@@ -42,6 +42,9 @@ def parse():
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--round-built-operands", action="store_true",
                     help="computed operand rows rounded once to bf16 (no value + residual pair)")
+    ap.add_argument("--graph", action="store_true",
+                    help="replay the step as CUDA graphs (alignment + plan, transfer) recorded "
+                         "once before the timed steps")
     ap.add_argument("--pool-before-map", action="store_true",
                     help="overlap mean pooling before the map (pooled operand rows per distinct "
                          "row) instead of pooling the mapped sender rows")
@@ -407,6 +410,10 @@ def run_ours(args):
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
+    if args.graph:
+        job.capture()
+        job.replay()
+        torch.cuda.synchronize()
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
     t_start.record(stream)
@@ -414,10 +421,16 @@ def run_ours(args):
         if flush is not None:
             flush.fill_(i & 0xff)
         st[i][0].record(stream)
-        job.align(stream)
-        job.make_plan(stream)
+        if args.graph:
+            job.replay(prep=True, xfer=False)
+        else:
+            job.align(stream)
+            job.make_plan(stream)
         ev[i][0].record(stream)
-        job.transfer(stream)
+        if args.graph:
+            job.replay(prep=False, xfer=True)
+        else:
+            job.transfer(stream)
         ev[i][1].record(stream)
         st[i][1].record(stream)
     t_end.record(stream)
@@ -568,6 +581,8 @@ def run_ours(args):
                                 else "computed rows as bf16 value + residual"),
                    "l2": ("inputs larger than L2 (no flush)" if flush is None else
                           "256 MB L2 flush write between steps (outside the timed events)"),
+                   "launch": ("CUDA graph replay (align + plan, transfer)" if args.graph
+                              else "stream launches"),
                    "parallelism": "replicas" if world > 1 else "single"},
         "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
         "gpu_launches": launches * args.steps, "device_status": status,

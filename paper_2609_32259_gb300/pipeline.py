@@ -112,6 +112,35 @@ class TransferJob:
         self.make_plan(stream)
         self.transfer(stream)
 
+    # -- CUDA graphs ------------------------------------------------------------
+    def capture(self) -> None:
+        """Records one step as two CUDA graphs: ``prep`` (hf_align_build and
+        hf_plan_create) and ``xfer`` (hf_transfer).  Every call of the step
+        is stream-ordered and allocation-free, so the graphs replay the same
+        kernels on the job's buffers: replays see the current contents of the
+        sender cache, the offsets and the maps, and write the receiver cache
+        and the plan workspace.  The plan created while recording is the
+        job's plan afterwards (its host arrays went into the recorded kernel
+        parameters)."""
+        import torch
+        self.step(torch.cuda.current_stream())  # kernel attributes, lazy module loading
+        torch.cuda.synchronize()
+        self.g_prep = torch.cuda.CUDAGraph()
+        self.g_xfer = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(self.g_prep):
+            s = torch.cuda.current_stream()
+            self.align(s)
+            self.make_plan(s)
+        with torch.cuda.graph(self.g_xfer):
+            self.transfer(torch.cuda.current_stream())
+
+    def replay(self, prep: bool = True, xfer: bool = True) -> None:
+        """Replays the recorded step on the current stream."""
+        if prep:
+            self.g_prep.replay()
+        if xfer:
+            self.g_xfer.replay()
+
     # -- inspection -------------------------------------------------------------
     def csr(self):
         nnz = int(self.info[0].item())
