@@ -638,6 +638,20 @@ def run_batch(args):
         batch()
         sequential()
     torch.cuda.synchronize()
+    if args.graph:  # the six alignments + plans, and the one batched transfer, as graphs
+        g_prep, g_batch = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g_prep):
+            for j in jobs:
+                j.align(torch.cuda.current_stream())
+                j.make_plan(torch.cuda.current_stream())
+        with torch.cuda.graph(g_batch):
+            B.transfer_batch([j.plan for j in jobs], [j.sender for j in jobs],
+                             [j.receiver for j in jobs], torch.cuda.current_stream())
+        prepare = g_prep.replay
+        batch = g_batch.replay
+        prepare()
+        batch()
+        torch.cuda.synchronize()
     status = max(j.device_status() for j in jobs)
     flops = bytes_ = 0.0
     T_total = 0
@@ -688,6 +702,8 @@ def run_batch(args):
                    "sequential_kernel_ms": res["sequential"][1],
                    "sequential_step_ms": res["sequential"][0],
                    "l2": "maps (1.2 GB) larger than L2 (no flush)",
+                   "launch": ("CUDA graph replay (align + plan of the six directions, batched "
+                              "transfer)" if args.graph else "stream launches"),
                    "parallelism": "single"},
         "roofline": roof, "cpu_baseline": None, "e2e": None, "clocks": clk,
         "gpu_launches": (sum(launches_per_step(w) - 1 for w in ws) + 1) * args.steps,
