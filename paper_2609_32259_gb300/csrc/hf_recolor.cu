@@ -134,6 +134,20 @@ __global__ void rc_ridge_kernel(float* S, int d, float reg) {
   for (int i = threadIdx.x; i < d; i += blockDim.x) S[static_cast<int64_t>(i) * d + i] += add;
 }
 
+// *out = trace(S) (one block of 256 threads).
+__global__ void rc_trace_kernel(const float* S, int d, double* out) {
+  __shared__ double part[256];
+  double t = 0.0;
+  for (int i = threadIdx.x; i < d; i += blockDim.x) t += S[static_cast<int64_t>(i) * d + i];
+  part[threadIdx.x] = t;
+  __syncthreads();
+  for (int o = blockDim.x / 2; o > 0; o >>= 1) {
+    if (threadIdx.x < o) part[threadIdx.x] += part[threadIdx.x + o];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) *out = part[0];
+}
+
 // out = a * in + b * I (square, or the leading square of a d x e matrix when
 // only scaling: b = 0).
 __global__ void rc_affine_kernel(float* out, const float* in, int64_t n_el, int cols, float a,
@@ -274,8 +288,20 @@ bool converged(double e, double* prev) {
 }
 
 // Newton-Schulz square root and inverse square root of the SPD matrix S
-// (d x d): root = S^{1/2}, inv_root = S^{-1/2}.  Y, Z, T, U are d x d work.
-hf_status ns_sqrt(cudaStream_t s, const GemmWork& h, const float* S, int d, float* Y, float* Z, float* T, float* U,
+// (d x d): root = S^{1/2} (when root is not null), inv_root = S^{-1/2}; Y, Z, T, U
+// are d x d work buffers distinct from both.
+// The coupled iteration Y <- Y T, Z <- T Z, T = (3I - Z Y) / 2 acts on each
+// eigenvalue x^2 of Z Y (x the corresponding eigenvalue of (S/c)^{1/2}
+// polynomials) as the cubic sign iteration x <- x (3 - x^2) / 2, which
+// lifts small x by only 1.5 per step.  With a lower bound l <= x <= 1 (the
+// ridge reg * trace / d bounds the smallest eigenvalue of S from below),
+// each step first scales Y and Z by b = sqrt(3 / (l^2 + l + 1)), the factor
+// for which the cubic maps [b l, b] onto [p(b l), 1] with p(b l) = p(b)
+// (the scaled Newton-Schulz step that maximises the new lower bound): small
+// x then grow by ~2.6 per step, and b -> 1 as l -> 1.  Scaling Y and Z
+// together keeps Y = (S/c) Z, so the limits are unchanged.  With reg = 0
+// there is no bound and the plain iteration runs.
+hf_status ns_sqrt(cudaStream_t s, const GemmWork& h, const float* S, int d, float reg, float* Y, float* Z, float* T, float* U,
                   float* root, float* inv_root, double* dscr, int* iters) {
   const int64_t n_el = static_cast<int64_t>(d) * d;
   const int grid = 1024;
@@ -289,15 +315,27 @@ hf_status ns_sqrt(cudaStream_t s, const GemmWork& h, const float* S, int d, floa
     set_error("hf_recolor_fit: a covariance is zero");
     return HF_ERR_INVALID_ARGUMENT;
   }
+  double l = 0.0;  // lower bound of the eigenvalues x of (Z Y)^{1/2}
+  if (reg > 0.f) {
+    rc_trace_kernel<<<1, 256, 0, s>>>(S, d, dscr);
+    double tr = 0.0;
+    if ((st = read_double(s, dscr, &tr)) != HF_OK) return st;
+    // S = S0 + reg tr(S0)/d I with S0 >= 0 and tr(S) = (1 + reg) tr(S0)
+    const double lam_lo = reg * tr / (static_cast<double>(d) * (1.0 + reg));
+    if (lam_lo > 0.0) l = std::min(1.0, sqrt(lam_lo / c));
+  }
   rc_affine_kernel<<<grid, 256, 0, s>>>(Y, S, n_el, d, static_cast<float>(1.0 / c), 0.f);
   rc_affine_kernel<<<grid, 256, 0, s>>>(Z, nullptr, n_el, d, 0.f, 1.f);
   int it = 0;
   double prev = 1e30;
   for (; it < kMaxIter; ++it) {
-    // T = 1.5 I - 0.5 Z Y
-    if ((st = sgemm(h, s, d, d, d, -0.5f, Z, d, 1, Y, d, 1, 0.f, T, d, nullptr, 1.5f)) != HF_OK)
+    const double b = l > 0.0 ? sqrt(3.0 / (l * l + l + 1.0)) : 1.0;
+    // T = 1.5 I - 0.5 b^2 Z Y
+    if ((st = sgemm(h, s, d, d, d, static_cast<float>(-0.5 * b * b), Z, d, 1, Y, d, 1, 0.f, T,
+                    d, nullptr, 1.5f)) != HF_OK)
       return st;
-    if (it % 4 == 3) {
+    // the residual |I - Z Y| = 2 |T - I| holds for unscaled steps
+    if (it % 4 == 3 && b < 1.0 + 1e-6) {
       double e2 = 0.0;
       HF_CUDA_TRY(cudaMemsetAsync(dscr, 0, sizeof(double), s), "clear");
       // |I - Z Y| = 2 |T - I|
@@ -305,15 +343,20 @@ hf_status ns_sqrt(cudaStream_t s, const GemmWork& h, const float* S, int d, floa
       if ((st = read_double(s, dscr, &e2)) != HF_OK) return st;
       if (converged(2.0 * sqrt(e2 / d), &prev)) break;
     }
-    if ((st = sgemm(h, s, d, d, d, 1.f, Y, d, 1, T, d, 1, 0.f, U, d)) != HF_OK) return st;  // Y T
+    const float bf = static_cast<float>(b);
+    if ((st = sgemm(h, s, d, d, d, bf, Y, d, 1, T, d, 1, 0.f, U, d)) != HF_OK) return st;  // b Y T
     std::swap(Y, U);
-    if ((st = sgemm(h, s, d, d, d, 1.f, T, d, 1, Z, d, 1, 0.f, U, d)) != HF_OK) return st;  // T Z
+    if ((st = sgemm(h, s, d, d, d, bf, T, d, 1, Z, d, 1, 0.f, U, d)) != HF_OK) return st;  // b T Z
     std::swap(Z, U);
+    l = std::min(1.0, b * l * (3.0 - b * b * l * l) / 2.0);
   }
   *iters = it;
-  rc_affine_kernel<<<grid, 256, 0, s>>>(root, Y, n_el, d, static_cast<float>(sqrt(c)), 0.f);
+  // inv_root first: root may be null (not wanted), and neither may alias the
+  // work buffers, which Y and Z rotate through
   rc_affine_kernel<<<grid, 256, 0, s>>>(inv_root, Z, n_el, d, static_cast<float>(1.0 / sqrt(c)),
                                         0.f);
+  if (root)
+    rc_affine_kernel<<<grid, 256, 0, s>>>(root, Y, n_el, d, static_cast<float>(sqrt(c)), 0.f);
   HF_CUDA_TRY(cudaGetLastError(), "hf_recolor_fit: iteration launch");
   return HF_OK;
 }
@@ -401,10 +444,10 @@ hf_status recolor_typed(int64_t N, int dx, int dy, const void* Xv, const void* Y
     rc_ridge_kernel<<<1, 256, 0, s>>>(F(L.sy), dy, reg);
   }
   int it1 = 0, it2 = 0, it3 = 0;
-  if ((st = ns_sqrt(s, h, F(L.sz), dx, F(L.p1), F(L.p2), F(L.p3), F(L.p4), F(L.p4) /*unused root*/,
+  if ((st = ns_sqrt(s, h, F(L.sz), dx, reg, F(L.p1), F(L.p2), F(L.p3), F(L.p4), nullptr,
                     F(L.sz_ih), dscr, &it1)) != HF_OK)
     return st;
-  if ((st = ns_sqrt(s, h, F(L.sy), dy, F(L.p1), F(L.p2), F(L.p3), F(L.p4), F(L.sy_h), F(L.sy_ih),
+  if ((st = ns_sqrt(s, h, F(L.sy), dy, reg, F(L.p1), F(L.p2), F(L.p3), F(L.p4), F(L.sy_h), F(L.sy_ih),
                     dscr, &it2)) != HF_OK)
     return st;
   // M = Sigma_Z^{-1/2} Sigma_ZY Sigma_Y^{-1/2}
