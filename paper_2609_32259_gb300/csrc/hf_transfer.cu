@@ -27,8 +27,16 @@
 //               three-layer neighbourhood) they copy the 128 sender rows with
 //               cp.async, eight lanes per 128-byte row; for pooled or blended
 //               rows they sum weighted sender rows in fp32 registers and round
-//               once.  Both write the 128-byte swizzled layout and fence it to
-//               the async proxy before arriving on the stage barrier.
+//               once, or write the rounded row and its rounding residual as
+//               two atoms (split operands).  Both write the 128-byte swizzled
+//               layout and fence it to the async proxy before arriving on the
+//               stage barrier.
+// Overlap mean pooling is linear, so by default it follows the map: the
+// tile rows of a CTA are a window of 128 consecutive aligned sender tokens
+// and the epilogue pools the mapped rows of each receiver row's columns
+// (pam_epilogue).  Plans whose rows the builders compute use wide tiles:
+// two 256-column blocks per tile in the two accumulators, so each built A
+// stage feeds twice the MMAs.
 // Pipeline hand-offs use mbarriers with bounded waits; nothing traps.
 #include <algorithm>
 #include <climits>
