@@ -135,6 +135,20 @@ struct Elem<float> {
 // alternate; with fewer, it takes tiles first, first + step, ... (the two
 // roles of a slot on different pairs).  lc = 2 * l + c indexes the maps,
 // biases and receiver cache.
+// Slot order needs at least two slots per CTA pair, and is kept unless tile
+// order fills the last round of tiles clearly better: a pair's share is
+// whole slots (two tiles) in slot order, single tiles otherwise (at 1K
+// receiver tokens, 256 slots over 76 pairs leave the last round 37% full,
+// 512 tiles 74%).
+__device__ __forceinline__ bool slot_order(int total_tiles, int tile_step) {
+  if (total_tiles < 4 * tile_step) return false;
+  const int slots = total_tiles >> 1;
+  const float fill_slots =
+      static_cast<float>(slots) / static_cast<float>(((slots + tile_step - 1) / tile_step) * tile_step);
+  const float fill_tiles = static_cast<float>(total_tiles) /
+                           static_cast<float>(((total_tiles + tile_step - 1) / tile_step) * tile_step);
+  return fill_slots >= fill_tiles - 0.03f;
+}
 __device__ __forceinline__ int tile_of(int seq, int first, int step, bool by_slot) {
   return by_slot ? 2 * (first + (seq >> 1) * step) + (seq & 1) : first + seq * step;
 }
@@ -768,7 +782,7 @@ __device__ __forceinline__ void gather_rows(const XferParams* Ps, const DirTable
                                             int lane, int row0, int total_tiles, int first_tile,
                                             int tile_step) {
   constexpr int kBK = Elem<T>::kBK;
-  const bool by_slot = total_tiles >= 4 * tile_step;  // as in transfer_body
+  const bool by_slot = slot_order(total_tiles, tile_step);
   constexpr int kPerChunk = 16 / sizeof(T);
   const int stages = Ps[0].stages_a;
   const int slab = t >> 5, rsub = lane >> 3, ch = lane & 7;
@@ -948,7 +962,7 @@ __device__ __forceinline__ void build_rows_staged(const XferParams* Ps, const Di
                                                   int first_tile, int tile_step) {
   constexpr int kBK = Elem<T>::kBK;
   constexpr int kPerChunk = 16 / sizeof(T);
-  const bool by_slot = total_tiles >= 4 * tile_step;  // as in transfer_body
+  const bool by_slot = slot_order(total_tiles, tile_step);
   const int stages = Ps[0].stages_a;
   const int slab = t >> 5, rsub = lane >> 3, ch = lane & 7;
   int stage = 0;
@@ -1128,7 +1142,7 @@ __device__ __forceinline__ void transfer_body(const CUtensorMap* maps, const Xfe
 
   DirTable<kDirs> dt;
   const int total_tiles = build_dirs<kDirs, kPam>(Ps, n_dir, &dt);
-  const bool by_slot = total_tiles >= 4 * tile_step;
+  const bool by_slot = slot_order(total_tiles, tile_step);
 
   if (warp == 0) {
     // ------------------------------------------------------------ map tiles
