@@ -362,8 +362,13 @@ hf_status ns_sqrt(cudaStream_t s, const GemmWork& h, const float* S, int d, floa
 }
 
 // Orthogonal polar factor of M (dx x dy, dx >= dy, full column rank):
-// X <- X (3I - X^T X) / 2 from X_0 = M / |M|_F.  Result in *out (one of the
-// two buffers).
+// X <- X (3I - X^T X) / 2 from X_0 = M / min(|M|_F, 1).  M is the whitened
+// cross-covariance Sigma_Z^{-1/2} Sigma_ZY Sigma_Y^{-1/2} of one weighted
+// sample set, so its singular values (canonical correlations; the ridges
+// only lower them) are at most 1 (Cauchy-Schwarz), and the iteration needs
+// no smaller scale: dividing by |M|_F = sqrt(sum of squared correlations)
+// would only shrink them and add ~log_1.5 |M|_F steps.  Result in *out (one
+// of the two buffers).
 hf_status ns_polar(cudaStream_t s, const GemmWork& h, const float* M, int dx, int dy, float* X, float* X2,
                    float* P, double* dscr, float** out, int* iters) {
   const int64_t n_el = static_cast<int64_t>(dx) * dy, p_el = static_cast<int64_t>(dy) * dy;
@@ -377,7 +382,8 @@ hf_status ns_polar(cudaStream_t s, const GemmWork& h, const float* M, int dx, in
     set_error("hf_recolor_fit: the cross-covariance is zero");
     return HF_ERR_INVALID_ARGUMENT;
   }
-  rc_affine_kernel<<<grid, 256, 0, s>>>(X, M, n_el, dy, static_cast<float>(1.0 / sqrt(m2)), 0.f);
+  rc_affine_kernel<<<grid, 256, 0, s>>>(X, M, n_el, dy,
+                                        static_cast<float>(1.0 / std::min(sqrt(m2), 1.0)), 0.f);
   int it = 0;
   double prev = 1e30;
   for (; it < kMaxIter; ++it) {
