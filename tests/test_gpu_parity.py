@@ -386,6 +386,12 @@ PAM_EDGE = {
     "one_token": lambda: W.llama_to_ministral(1).with_(L_s=3, L_r=3, align_mode="overlap_mean"),
     "rope_table_pos0": lambda: W.llama_to_ministral(700).with_(
         L_s=4, L_r=3, align_mode="overlap_mean", rope_table=True, r_pos0=(90000,)),
+    # fp32 blends per sender token (the register builder) in wide tiles
+    "interp_f32_wide": lambda: W.llama_to_ministral(400).with_(
+        L_s=4, L_r=3, dtype="f32", align_mode="overlap_mean", layer_mode="interp"),
+    # key norm needs the pooled row: overlap pooling stays before the map
+    "knorm_pools_first": lambda: W.llama_to_ministral(600).with_(
+        L_s=4, L_r=3, align_mode="overlap_mean", knorm=True, r_pos0=(321,)),
 }
 
 
